@@ -1,0 +1,160 @@
+/*
+ * sparsecoder.h -- C ABI of the GB300 (sm_103a) hot path of SparseCoder
+ * (arXiv 2310.07109): Longformer-style sparse attention fused with learned
+ * token pruning, one layer or a pruned stack of layers.
+ *
+ * Conventions
+ * -----------
+ * - All tensors are caller-owned DEVICE memory unless a field says "host".
+ *   The library allocates nothing; scratch lives in a caller-supplied
+ *   workspace of sc_workspace_size() bytes (device memory, 256-byte aligned).
+ * - bf16 tensors are passed as uint16_t bit patterns.  Q/K/V/O rows are
+ *   [.., token, head, 64] with the head dimension fixed at SC_HEAD_DIM = 64;
+ *   every such pointer must be 16-byte aligned.
+ * - Every call is asynchronous on `stream` (a cudaStream_t passed as void*;
+ *   NULL = legacy default stream).  No call synchronises the host, and no
+ *   current length ever travels back to the host: layer l+1 reads the
+ *   lengths layer l wrote, on the device.
+ * - Arguments are validated on the host before anything is launched; a bad
+ *   argument returns an SC_ERR_* code with nothing enqueued.  CUDA launch
+ *   errors return SC_ERR_CUDA.  No C++ exception crosses this interface.
+ * - Every wait inside a kernel is bounded (about 2 s).  A wait that expires
+ *   makes the kernel record SC_ERR_TIMEOUT in the workspace status word and
+ *   return; sc_workspace_status() reports (and clears) it.
+ *
+ * The method (paper sections / equations cited on each call):
+ *   current tokens c = 0..n-1 of one sequence, original positions p(c);
+ *   G = global original positions; a token is global when p(c) is in G.
+ *   Allowed keys of row i: all n tokens if i is global, otherwise
+ *   {j : |i - j| <= w} U {global j}  (Sec. "Sparse Attention": unit i is
+ *   attended by units i-w..i+w; Sec. "Extractor of Attention Scores": special
+ *   tokens attend to every token and are attended by every token).
+ *   P_h = row-wise softmax of q.k / sqrt(64) over the allowed keys (Fig. 1
+ *   caption); O_h[i] = sum_j P_h[i,j] v_j.
+ *   s_j = (1/(H n)) sum_h sum_i P_h[i,j]: probabilities accumulated
+ *   vertically (Sec. "Pruning"; Fig. 1 caption), averaged over heads and rows.
+ *   keep_j = (j == 0) || s_j >= theta  (Sec. "Token Pruning", Step 2, the
+ *   binarised mask, read as >= and with the first token always kept);
+ *   kept tokens are compacted in order (Step 3, hard pruning).
+ */
+#ifndef SPARSECODER_H
+#define SPARSECODER_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SC_HEAD_DIM 64
+#define SC_MAX_LEN 4096   /* longest supported (padded) sequence */
+#define SC_MAX_GLOBAL 16  /* most global positions per call */
+#define SC_MAX_WINDOW 256 /* widest one-sided window when L > 640 */
+
+typedef enum {
+  SC_OK = 0,
+  SC_ERR_INVALID_ARG = 1, /* null pointer, bad size, misaligned pointer, bad global set */
+  SC_ERR_UNSUPPORTED = 2, /* L > SC_MAX_LEN, too many globals, window too wide */
+  SC_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed */
+  SC_ERR_TIMEOUT = 4,     /* a bounded device-side wait expired (from sc_workspace_status) */
+  SC_ERR_WORKSPACE = 5    /* workspace missing, too small or misaligned */
+} sc_status;
+
+/*
+ * One layer on tokens already in current (compacted) order.
+ *
+ * Q, K, V    bf16 [B][L][H][64]; row c of sequence b holds current token c.
+ *            Rows at or beyond len[b] are never read.
+ * len        int32 [B]: current length n_b (0 <= n_b <= L).
+ * pos        int32 [B][L]: original position of each current token, strictly
+ *            increasing within [0, n_b).  Decides which tokens are global and
+ *            is what pos_out is compacted from.
+ * w          one-sided window (>= 0).
+ * global_pos HOST int32 [n_global]: sorted, distinct original positions,
+ *            0 <= g < L, n_global <= SC_MAX_GLOBAL (may be 0).
+ * alpha      theta_b = alpha / n_b for every sequence (threshold schedule of
+ *            Sec. "RQ4": thresholds scaled linearly across layers; the caller
+ *            supplies alpha for this layer).  Ignored when theta != NULL.
+ * theta      optional float [B]: absolute thresholds per sequence.
+ * O          bf16 [B][L][H][64] out: attention output of every current token
+ *            (all n_b tokens, before pruning) at its current slot.
+ * scores     float [B][L] out: s_j at current slot j.
+ * pos_out    int32 [B][L] out: original positions of the kept tokens, in order.
+ * len_out    int32 [B] out: number of kept tokens.
+ * Slots at or beyond the current (resp. kept) length are left untouched.
+ * pos_out/len_out must not alias pos/len.
+ */
+typedef struct {
+  int B, L, H, w;
+  const uint16_t* Q;
+  const uint16_t* K;
+  const uint16_t* V;
+  const int32_t* len;
+  const int32_t* pos;
+  const int32_t* global_pos;
+  int n_global;
+  float alpha;
+  const float* theta;
+  uint16_t* O;
+  float* scores;
+  int32_t* pos_out;
+  int32_t* len_out;
+} sc_layer_args;
+
+/*
+ * A pruned stack of n_layers layers over inputs in ORIGINAL-position order.
+ *
+ * Q, K, V    bf16 [n_layers][B][L][H][64]: layer l reads, for each token that
+ *            survived layers 0..l-1, the row at its original position.
+ * pad_mask   uint8 [B][L] (1 = real token) or NULL (no padding).  Padding
+ *            tokens are removed before layer 0 (Fig. "experiment" caption:
+ *            shorter inputs are padded to max_length).
+ * w, global_pos, n_global   as for sc_layer_args.
+ * alpha      HOST float [n_layers]: theta_{l,b} = alpha[l] / n_{l,b}.
+ * O          bf16 [n_layers][B][L][H][64] out (current slots of each layer).
+ * scores     float [n_layers][B][L] out.
+ * pos        int32 [n_layers+1][B][L] out: pos[0] = real tokens after padding
+ *            removal, pos[l+1] = survivors of layer l.
+ * len        int32 [n_layers+1][B] out.
+ */
+typedef struct {
+  int n_layers, B, L, H, w;
+  const uint16_t* Q;
+  const uint16_t* K;
+  const uint16_t* V;
+  const uint8_t* pad_mask;
+  const int32_t* global_pos;
+  int n_global;
+  const float* alpha;
+  uint16_t* O;
+  float* scores;
+  int32_t* pos;
+  int32_t* len;
+} sc_stack_args;
+
+/* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
+size_t sc_workspace_size(int B, int L, int H);
+
+/* One layer (Sec. "Sparse Attention" + Sec. "Token Pruning").  Errors: see sc_status. */
+int sc_layer_forward(const sc_layer_args* args, void* workspace, size_t workspace_bytes,
+                     void* stream);
+
+/* The pruned stack (Fig. "sparsecoder": sparse attention with layer-wise
+ * token pruning, 12 layers in the paper's encoder).  Errors: see sc_status. */
+int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
+                     void* stream);
+
+/* Synchronises `stream`, returns SC_ERR_TIMEOUT if any kernel since the last
+ * query recorded an expired wait (else SC_OK, or SC_ERR_CUDA), and clears
+ * the status word. */
+int sc_workspace_status(void* workspace, size_t workspace_bytes, void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* sc_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPARSECODER_H */

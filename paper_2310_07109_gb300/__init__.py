@@ -1,0 +1,11 @@
+"""SparseCoder hot path on GB300 (sm_103a): Longformer-style sparse attention
+fused with learned token pruning, behind the C ABI of include/sparsecoder.h.
+
+The Python surface is a thin ctypes binding (``binding``); the arithmetic runs
+in ``libsparsecoder.so`` (``csrc/``), built in-tree by ``build.build_library``.
+"""
+from .binding import (SparseCoderError, layer_forward, load, new_workspace, stack_forward,
+                      status_string, workspace_size, workspace_status)
+
+__all__ = ["SparseCoderError", "layer_forward", "load", "new_workspace", "stack_forward",
+           "status_string", "workspace_size", "workspace_status"]

@@ -1,0 +1,181 @@
+"""ctypes binding of ``libsparsecoder.so`` (include/sparsecoder.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  PyTorch provides device memory and the current stream.  There is no
+CPU fallback: if the library cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+SC_HEAD_DIM = 64
+SC_MAX_LEN = 4096
+SC_MAX_GLOBAL = 16
+SC_MAX_WINDOW = 256
+
+SC_OK, SC_ERR_INVALID_ARG, SC_ERR_UNSUPPORTED, SC_ERR_CUDA, SC_ERR_TIMEOUT, SC_ERR_WORKSPACE = range(6)
+
+
+class SparseCoderError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(msg)
+        self.code = code
+
+
+class LayerArgs(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("L", ctypes.c_int), ("H", ctypes.c_int), ("w", ctypes.c_int),
+                ("Q", ctypes.c_void_p), ("K", ctypes.c_void_p), ("V", ctypes.c_void_p),
+                ("len", ctypes.c_void_p), ("pos", ctypes.c_void_p),
+                ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
+                ("alpha", ctypes.c_float), ("theta", ctypes.c_void_p),
+                ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
+                ("pos_out", ctypes.c_void_p), ("len_out", ctypes.c_void_p)]
+
+
+class StackArgs(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int), ("B", ctypes.c_int), ("L", ctypes.c_int),
+                ("H", ctypes.c_int), ("w", ctypes.c_int),
+                ("Q", ctypes.c_void_p), ("K", ctypes.c_void_p), ("V", ctypes.c_void_p),
+                ("pad_mask", ctypes.c_void_p),
+                ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
+                ("alpha", ctypes.POINTER(ctypes.c_float)),
+                ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
+                ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p)]
+
+
+EXPORTED = ["sc_layer_forward", "sc_stack_forward", "sc_workspace_size", "sc_workspace_status",
+            "sc_status_string"]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False):
+    """Load the CUDA library (optionally building it first); raise if unavailable."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if build_if_missing and not os.path.exists(path):
+            _build.build_library()
+        if not os.path.exists(path):
+            raise RuntimeError(
+                "libsparsecoder.so is not built (run __graft_entry__.build() or "
+                "python -m paper_2310_07109_gb300.build); there is no fallback path")
+        lib = ctypes.CDLL(path)
+        lib.sc_workspace_size.restype = ctypes.c_size_t
+        lib.sc_workspace_size.argtypes = [ctypes.c_int] * 3
+        lib.sc_layer_forward.restype = ctypes.c_int
+        lib.sc_layer_forward.argtypes = [ctypes.POINTER(LayerArgs), ctypes.c_void_p,
+                                         ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_stack_forward.restype = ctypes.c_int
+        lib.sc_stack_forward.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
+                                         ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_workspace_status.restype = ctypes.c_int
+        lib.sc_workspace_status.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_status_string.restype = ctypes.c_char_p
+        lib.sc_status_string.argtypes = [ctypes.c_int]
+        _lib = lib
+        return lib
+
+
+def status_string(code: int) -> str:
+    return load().sc_status_string(int(code)).decode()
+
+
+def _check(code: int):
+    if code != SC_OK:
+        raise SparseCoderError(code, status_string(code))
+
+
+def workspace_size(B: int, L: int, H: int) -> int:
+    return int(load().sc_workspace_size(int(B), int(L), int(H)))
+
+
+def new_workspace(B: int, L: int, H: int, device=None) -> torch.Tensor:
+    n = workspace_size(B, L, H)
+    if n == 0:
+        raise SparseCoderError(SC_ERR_INVALID_ARG, "invalid workspace sizes")
+    ws = torch.zeros(n + 256, dtype=torch.uint8, device=device or "cuda")
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + n]
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream_handle(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _int32_host(values):
+    vals = [int(v) for v in values]
+    arr = (ctypes.c_int32 * max(1, len(vals)))(*vals)
+    return arr, len(vals)
+
+
+def layer_forward(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *, O=None,
+                  scores=None, pos_out=None, len_out=None, workspace=None, stream=None):
+    """One layer on current-order inputs (``sc_layer_forward``).
+
+    Q, K, V: bf16 [B, L, H, 64] cuda tensors; length: int32 [B]; pos: int32 [B, L].
+    Returns (O, scores, pos_out, len_out).
+    """
+    B, L, H, D = Q.shape
+    dev = Q.device
+    O = O if O is not None else torch.empty((B, L, H, D), dtype=torch.bfloat16, device=dev)
+    scores = scores if scores is not None else torch.empty((B, L), dtype=torch.float32, device=dev)
+    pos_out = pos_out if pos_out is not None else torch.empty((B, L), dtype=torch.int32, device=dev)
+    len_out = len_out if len_out is not None else torch.empty((B,), dtype=torch.int32, device=dev)
+    ws = workspace if workspace is not None else new_workspace(B, L, H, dev)
+    garr, ng = _int32_host(global_pos)
+    a = LayerArgs(B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(length), _ptr(pos),
+                  ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, float(alpha),
+                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out))
+    _check(load().sc_layer_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
+    return O, scores, pos_out, len_out
+
+
+def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
+                  stream=None):
+    """The pruned layer stack (``sc_stack_forward``).
+
+    Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
+    pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers].
+    Returns a dict with O, scores, pos, len (device tensors).
+    """
+    nl, B, L, H, D = Q.shape
+    dev = Q.device
+    if out is None:
+        out = {"O": torch.empty((nl, B, L, H, D), dtype=torch.bfloat16, device=dev),
+               "scores": torch.empty((nl, B, L), dtype=torch.float32, device=dev),
+               "pos": torch.empty((nl + 1, B, L), dtype=torch.int32, device=dev),
+               "len": torch.empty((nl + 1, B), dtype=torch.int32, device=dev)}
+    ws = workspace if workspace is not None else new_workspace(B, L, H, dev)
+    garr, ng = _int32_host(global_pos)
+    al = (ctypes.c_float * nl)(*[float(x) for x in alpha])
+    a = StackArgs(nl, B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(pad_mask),
+                  ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
+                  ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
+                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]))
+    _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
+    return out
+
+
+def workspace_status(workspace, stream=None) -> int:
+    """Synchronise and return (then clear) the workspace status code."""
+    return int(load().sc_workspace_status(_ptr(workspace), workspace.numel(),
+                                          _stream_handle(stream)))

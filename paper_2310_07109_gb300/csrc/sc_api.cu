@@ -1,0 +1,289 @@
+// sc_api.cu -- the C ABI declared in include/sparsecoder.h: argument checks,
+// workspace layout, TMA descriptors and the launch sequence of one layer or
+// of the pruned layer stack.  All launches go to the caller's stream; nothing
+// here synchronises the host except sc_workspace_status().
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/sparsecoder.h"
+#include "sc_internal.cuh"
+
+namespace sc {
+cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st);
+cudaError_t configure_kernels();
+cudaError_t launch_layer(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
+                         const LayerParams& p, cudaStream_t st);
+}  // namespace sc
+
+namespace {
+
+using namespace sc;
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+struct WsLayout {
+  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, total;
+};
+
+bool ws_layout(int B, int L, int H, WsLayout* w) {
+  if (B < 1 || L < 1 || H < 1 || L > kMaxLen) return false;
+  const size_t T = (L + kTile - 1) / kTile;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes);
+    return at;
+  };
+  w->status = take(kAlign);
+  w->lse = take(sizeof(float) * B * H * (size_t)L);
+  w->acc = take(sizeof(float) * B * H * (size_t)L);
+  w->gpart = take(sizeof(float) * B * H * T * kMaxGlobal);
+  w->gstat = take(sizeof(float) * B * H * T * kMaxGlobal * 2);
+  w->og = take(sizeof(float) * B * H * kMaxGlobal * kHeadDim);
+  w->keep = take(sizeof(uint8_t) * B * (size_t)L);
+  w->cnt_tile = take(sizeof(uint32_t) * B * T);
+  w->cnt_seq = take(sizeof(uint32_t) * B);
+  w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
+  w->ng = take(sizeof(int32_t) * 2 * B);
+  w->total = off;
+  return true;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* ptr = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 2-D view [rows][64] of a bf16 tensor whose rows are (.., token, head); one
+// TMA box is a single 128-byte row, gathered four at a time.
+bool encode_rows(CUtensorMap* m, const void* base, long long rows) {
+  auto enc = get_encoder();
+  if (!enc) return false;
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+  cuuint64_t gstride[1] = {static_cast<cuuint64_t>(kHeadDim * 2)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kHeadDim), 1};
+  cuuint32_t estride[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box,
+             estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int ensure_configured() {
+  static std::mutex mu;
+  static bool done[256] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return SC_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    if (configure_kernels() != cudaSuccess) return SC_ERR_CUDA;
+    done[dev] = true;
+  }
+  return SC_OK;
+}
+
+int check_common(int B, int L, int H, int w, const int32_t* gpos, int ngl) {
+  if (B < 1 || L < 1 || H < 1 || w < 0 || ngl < 0) return SC_ERR_INVALID_ARG;
+  if (L > SC_MAX_LEN) return SC_ERR_UNSUPPORTED;
+  if (ngl > SC_MAX_GLOBAL) return SC_ERR_UNSUPPORTED;
+  if (ngl > 0 && gpos == nullptr) return SC_ERR_INVALID_ARG;
+  for (int g = 0; g < ngl; ++g) {
+    if (gpos[g] < 0 || gpos[g] >= L) return SC_ERR_INVALID_ARG;
+    if (g > 0 && gpos[g] <= gpos[g - 1]) return SC_ERR_INVALID_ARG;
+  }
+  // one 128-row tile must reach at most five 128-key tiles
+  if (L > kMaxBandTiles * kTile && w > SC_MAX_WINDOW) return SC_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * L * H > (1ll << 30)) return SC_ERR_UNSUPPORTED;
+  return SC_OK;
+}
+
+void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
+  p->status = reinterpret_cast<int*>(ws + lay.status);
+  p->lse = reinterpret_cast<float*>(ws + lay.lse);
+  p->acc = reinterpret_cast<float*>(ws + lay.acc);
+  p->gpart = reinterpret_cast<float*>(ws + lay.gpart);
+  p->gstat = reinterpret_cast<float*>(ws + lay.gstat);
+  p->og = reinterpret_cast<float*>(ws + lay.og);
+  p->keep = reinterpret_cast<uint8_t*>(ws + lay.keep);
+  p->cnt_tile = reinterpret_cast<uint32_t*>(ws + lay.cnt_tile);
+  p->cnt_seq = reinterpret_cast<uint32_t*>(ws + lay.cnt_seq);
+  int32_t* gcur = reinterpret_cast<int32_t*>(ws + lay.gcur);
+  int32_t* ng = reinterpret_cast<int32_t*>(ws + lay.ng);
+  p->gcur = gcur + slot * p->B * kMaxGlobal;
+  p->gcur_out = gcur + (1 - slot) * p->B * kMaxGlobal;
+  p->ng = ng + slot * p->B;
+  p->ng_out = ng + (1 - slot) * p->B;
+}
+
+int reset_counters(char* ws, const WsLayout& lay, cudaStream_t st) {
+  // the counters reset themselves after each layer; clearing them per call
+  // keeps a call independent of any earlier call that was cut short
+  if (cudaMemsetAsync(ws + lay.cnt_tile, 0, lay.gcur - lay.cnt_tile, st) != cudaSuccess)
+    return SC_ERR_CUDA;
+  return SC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t sc_workspace_size(int B, int L, int H) {
+  WsLayout lay;
+  if (!ws_layout(B, L, H, &lay)) return 0;
+  return lay.total;
+}
+
+const char* sc_status_string(int status) {
+  switch (status) {
+    case SC_OK: return "SC_OK";
+    case SC_ERR_INVALID_ARG: return "SC_ERR_INVALID_ARG: invalid argument";
+    case SC_ERR_UNSUPPORTED: return "SC_ERR_UNSUPPORTED: size or option outside the supported range";
+    case SC_ERR_CUDA: return "SC_ERR_CUDA: a CUDA call failed";
+    case SC_ERR_TIMEOUT: return "SC_ERR_TIMEOUT: a bounded device-side wait expired";
+    case SC_ERR_WORKSPACE: return "SC_ERR_WORKSPACE: workspace missing, too small or misaligned";
+    default: return "unknown sparsecoder status";
+  }
+}
+
+int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if (!a->Q || !a->K || !a->V || !a->len || !a->pos || !a->O || !a->scores || !a->pos_out ||
+      !a->len_out)
+    return SC_ERR_INVALID_ARG;
+  if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
+    return SC_ERR_INVALID_ARG;
+  if (a->pos_out == a->pos || a->len_out == a->len) return SC_ERR_INVALID_ARG;
+  WsLayout lay;
+  ws_layout(a->B, a->L, a->H, &lay);
+  if (!workspace || ws_bytes < lay.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
+    return SC_ERR_WORKSPACE;
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+
+  const long long rows = static_cast<long long>(a->B) * a->L * a->H;
+  CUtensorMap mq, mk, mv;
+  if (!encode_rows(&mq, a->Q, rows) || !encode_rows(&mk, a->K, rows) ||
+      !encode_rows(&mv, a->V, rows))
+    return SC_ERR_CUDA;
+  if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
+
+  LayerParams p{};
+  p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
+  p.T = (a->L + kTile - 1) / kTile;
+  p.gather = 0;
+  p.row_base = 0;
+  p.len = a->len;
+  p.pos = a->pos;
+  p.O = a->O;
+  p.scores = a->scores;
+  p.pos_out = a->pos_out;
+  p.len_out = a->len_out;
+  p.alpha = a->alpha;
+  p.theta = a->theta;
+  fill_workspace(&p, ws, lay, 0);
+
+  PrepParams pp{};
+  pp.B = a->B; pp.L = a->L;
+  pp.pos_in = a->pos;
+  pp.len_in = a->len;
+  pp.gcur = const_cast<int32_t*>(p.gcur);
+  pp.ng = const_cast<int32_t*>(p.ng);
+  pp.n_global = a->n_global;
+  for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
+  if (launch_prep(pp, st) != cudaSuccess) return SC_ERR_CUDA;
+  if (launch_layer(mq, mk, mv, p, st) != cudaSuccess) return SC_ERR_CUDA;
+  return SC_OK;
+}
+
+int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
+    return SC_ERR_INVALID_ARG;
+  if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
+    return SC_ERR_INVALID_ARG;
+  const long long rows = static_cast<long long>(a->n_layers) * a->B * a->L * a->H;
+  if (rows > (1ll << 31) - 1) return SC_ERR_UNSUPPORTED;
+  WsLayout lay;
+  ws_layout(a->B, a->L, a->H, &lay);
+  if (!workspace || ws_bytes < lay.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
+    return SC_ERR_WORKSPACE;
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+
+  CUtensorMap mq, mk, mv;
+  if (!encode_rows(&mq, a->Q, rows) || !encode_rows(&mk, a->K, rows) ||
+      !encode_rows(&mv, a->V, rows))
+    return SC_ERR_CUDA;
+  if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
+
+  const size_t BL = static_cast<size_t>(a->B) * a->L;
+  LayerParams p{};
+  p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
+  p.T = (a->L + kTile - 1) / kTile;
+  p.gather = 1;
+  p.theta = nullptr;
+  fill_workspace(&p, ws, lay, 0);
+
+  PrepParams pp{};
+  pp.B = a->B; pp.L = a->L;
+  pp.pad_mask = a->pad_mask;
+  pp.pos_out = a->pos;
+  pp.len_out = a->len;
+  pp.gcur = const_cast<int32_t*>(p.gcur);
+  pp.ng = const_cast<int32_t*>(p.ng);
+  pp.n_global = a->n_global;
+  for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
+  if (launch_prep(pp, st) != cudaSuccess) return SC_ERR_CUDA;
+
+  for (int l = 0; l < a->n_layers; ++l) {
+    fill_workspace(&p, ws, lay, l & 1);
+    p.row_base = static_cast<long long>(l) * a->B * a->L * a->H;
+    p.len = a->len + static_cast<size_t>(l) * a->B;
+    p.len_out = a->len + static_cast<size_t>(l + 1) * a->B;
+    p.pos = a->pos + static_cast<size_t>(l) * BL;
+    p.pos_out = a->pos + static_cast<size_t>(l + 1) * BL;
+    p.O = a->O + static_cast<size_t>(l) * BL * a->H * kHeadDim;
+    p.scores = a->scores + static_cast<size_t>(l) * BL;
+    p.alpha = a->alpha[l];
+    if (launch_layer(mq, mk, mv, p, st) != cudaSuccess) return SC_ERR_CUDA;
+  }
+  return SC_OK;
+}
+
+int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {
+  if (!workspace || ws_bytes < kAlign) return SC_ERR_WORKSPACE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return SC_ERR_CUDA;
+  int word = 0;
+  if (cudaMemcpy(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return SC_ERR_CUDA;
+  if (word == 0) return SC_OK;
+  if (cudaMemset(workspace, 0, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  return (word & kStatusTimeout) ? SC_ERR_TIMEOUT : SC_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,68 @@
+// sc_internal.cuh -- parameter block shared by the host launcher and the
+// kernels of the sparse-attention + token-pruning layer.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+
+namespace sc {
+
+constexpr int kHeadDim = 64;
+constexpr int kTile = 128;         // rows (queries or keys) per tile
+constexpr int kMaxBandTiles = 5;   // key (query) tiles touched by one 128-row tile
+constexpr int kMaxGlobal = 16;     // global tokens per sequence (one 16-wide MMA tile)
+constexpr int kMaxLen = 4096;
+constexpr int kMaxTiles = kMaxLen / kTile;
+constexpr int kThreads = 192;      // 4 softmax warps + 1 load warp + 1 MMA warp
+constexpr uint32_t kTileBytes = kTile * kHeadDim * 2;   // 16 KB bf16 tile
+constexpr uint32_t kGTileBytes = kMaxGlobal * kHeadDim * 2;
+
+// status word bits (workspace)
+constexpr int kStatusTimeout = 1;
+
+// log2(e) / sqrt(64): logits are kept in base-2 units, x = (q.k) * kLogitScale2.
+constexpr float kLogitScale2 = 0.125f * 1.4426950408889634f;
+
+struct LayerParams {
+  int B, L, H, w;
+  int T;                 // tiles per padded sequence = ceil(L / 128)
+  int gather;            // 1: row of current token c is at original position pos[b][c]
+  long long row_base;    // first tensor-map row of this layer's [B][L][H] block
+  const int32_t* len;    // [B] current lengths
+  const int32_t* pos;    // [B][L] original positions of current tokens
+  const int32_t* gcur;   // [B][kMaxGlobal] current indices of global tokens (increasing)
+  const int32_t* ng;     // [B] number of global tokens present
+  uint16_t* O;           // [B][L][H][64] bf16 out
+  float* scores;         // [B][L] out
+  int32_t* pos_out;      // [B][L] out
+  int32_t* len_out;      // [B] out
+  int32_t* gcur_out;     // [B][kMaxGlobal] out (next layer)
+  int32_t* ng_out;       // [B] out
+  float alpha;           // theta_b = alpha / n_b unless theta != nullptr
+  const float* theta;    // [B] absolute thresholds or nullptr
+  // workspace
+  float* lse;            // [B][H][L] per-row log2-sum-exp2 (+inf for global rows)
+  float* acc;            // [B][H][L] per-head column sums: band rows + global rows
+  float* gpart;          // [B][H][T][kMaxGlobal] column sums of global keys over far rows
+  float* gstat;          // [B][H][T][kMaxGlobal][2] (max, sum) of global rows per key tile
+  float* og;             // [B][H][kMaxGlobal][64] fp32 outputs of global rows
+  uint8_t* keep;         // [B][L]
+  uint32_t* cnt_tile;    // [B][T]
+  uint32_t* cnt_seq;     // [B]
+  int* status;
+};
+
+struct PrepParams {
+  int B, L;
+  const uint8_t* pad_mask;   // [B][L] or nullptr (stack mode)
+  const int32_t* pos_in;     // [B][L] given positions (layer mode) or nullptr
+  const int32_t* len_in;     // [B] (layer mode)
+  int32_t* pos_out;          // [B][L] (stack mode)
+  int32_t* len_out;          // [B] (stack mode)
+  int32_t* gcur;             // [B][kMaxGlobal]
+  int32_t* ng;               // [B]
+  int n_global;
+  int global_pos[kMaxGlobal];
+};
+
+}  // namespace sc

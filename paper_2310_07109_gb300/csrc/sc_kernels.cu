@@ -1,0 +1,889 @@
+// sc_kernels.cu -- device code of one sparse-attention + learned-token-pruning
+// layer on sm_103a.
+//
+// Per layer, per sequence b (n current tokens, original positions pos[b][*]):
+//
+//   rows kernel   (one CTA per (128-query-row tile, head, sequence))
+//     S = Q K^T over the band key tiles and one 16-wide tile of global keys,
+//     tensor cores (tcgen05, bf16 -> fp32 in tensor memory), operands gathered
+//     by TMA (gather4) straight from the original-position rows.  Row softmax
+//     in fp32 (base-2, lazily rescaled running max), P (bf16) V accumulated in
+//     tensor memory.  Writes O, the row log-sum-exp LSE_i, the far-row column
+//     sums of the global keys, and (max, sum) of the global rows over this
+//     tile's keys.
+//
+//   cols kernel   (one CTA per (128-key tile, head, sequence))
+//     S^T = K Q^T for the query tiles whose band reaches this key tile, then
+//     P[i,j] = exp2(S_ij - LSE_i) summed over the rows i of each key column j
+//     (each thread owns one key column, so no cross-thread reduction), plus the
+//     global rows' probabilities and their P V outputs.  The last CTA of a key
+//     tile sums the heads in a fixed order and applies the threshold; the last
+//     tile of a sequence compacts the survivors in order.  No wait on other
+//     CTAs: the "last" CTA is found by an atomic counter.
+//
+// The method (allowed sets, row softmax, vertical accumulation, >= threshold,
+// order-preserving removal) is Sec. "Sparse Attention", Sec. "Extractor of
+// Attention Scores in Sparse Attention Matrix" and Sec. "Token Pruning".
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "sc_internal.cuh"
+#include "sm103_primitives.cuh"
+
+namespace sc {
+
+// ---------------------------------------------------------------------------
+// small helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void named_sync_softmax() {
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Bounded wait that ignores the abort flag: used in teardown to make sure no
+// asynchronous copy or MMA is still writing into this CTA's memory.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  int dummy = 0;
+  mbar_wait(bar, parity, &dummy, 1000000000ull);
+}
+
+// Wait used by the softmax warps: the outcome is made uniform across the warp
+// so that an expired wait can never leave lanes diverged at a warp vote.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
+}
+
+// Tensor-map row of (sequence b, row src of that sequence, head h).
+__device__ __forceinline__ int tmap_row(const LayerParams& p, int b, int src, int h) {
+  return static_cast<int>(p.row_base + (static_cast<long long>(b) * p.L + src) * p.H + h);
+}
+
+__device__ __forceinline__ int src_row(const LayerParams& p, int b, int c) {
+  return p.gather ? __ldg(p.pos + static_cast<size_t>(b) * p.L + c) : c;
+}
+
+// The load warp gathers a 128-row tile (rows first_c .. first_c+127 of the
+// current sequence, clamped to n-1) of one tensor into `dst`; each lane moves
+// four rows with one gather4.
+__device__ __forceinline__ void load_tile(const LayerParams& p, const CUtensorMap* map,
+                                          uint8_t* dst, int b, int h, int first_c, int n,
+                                          uint64_t* bar, int lane) {
+  int r[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    int c = min(first_c + 4 * lane + k, n - 1);
+    r[k] = tmap_row(p, b, src_row(p, b, c), h);
+  }
+  tma_gather4(dst + 512 * lane, map, 0, r[0], r[1], r[2], r[3], bar);
+}
+
+// The 16 global rows (current indices gc[0..ng-1], the last repeated).
+__device__ __forceinline__ void load_globals(const LayerParams& p, const CUtensorMap* map,
+                                             uint8_t* dst, int b, int h, const int* gc, int ng,
+                                             uint64_t* bar, int lane) {
+  if (lane < 4) {
+    int r[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      int g = min(4 * lane + k, ng - 1);
+      r[k] = tmap_row(p, b, src_row(p, b, gc[g]), h);
+    }
+    tma_gather4(dst + 512 * lane, map, 0, r[0], r[1], r[2], r[3], bar);
+  }
+}
+
+// Issue D[128 x N] (+)= A[128 x 64] * B[N x 64]^T with both operands K-major
+// 128B-swizzled tiles (A rows and B rows are 128-byte lines).
+__device__ __forceinline__ void mma_qk(uint32_t d_tmem, uint32_t a_smem, uint32_t b_smem, int N) {
+  const uint32_t idesc = (N == 128) ? idesc_bf16(128, 128, false, false)
+                                    : idesc_bf16(128, 16, false, false);
+#pragma unroll
+  for (int k = 0; k < kHeadDim / 16; ++k)
+    umma_bf16(d_tmem, sdesc_sw128(a_smem + 32 * k), sdesc_sw128(b_smem + 32 * k), idesc, k > 0);
+}
+
+// Issue D[128 x 64] (+)= P[128 x 16*ksteps] * V[16*ksteps x 64]: P is a K-major
+// 128B-swizzled tile in two 64-key halves of 16 KB, V an MN-major tile of
+// 128-byte key rows.
+__device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_t v_smem,
+                                       int ksteps, bool accumulate) {
+  const uint32_t idesc = idesc_bf16(128, 64, false, true);
+  for (int k = 0; k < ksteps; ++k)
+    umma_bf16(d_tmem, sdesc_sw128(p_smem + (k >> 2) * 16384 + (k & 3) * 32),
+              sdesc_sw128(v_smem + k * 2048), idesc, (accumulate || k > 0) ? 1u : 0u);
+}
+
+// ---------------------------------------------------------------------------
+// rows kernel
+// ---------------------------------------------------------------------------
+struct RowsSmem {
+  uint64_t bar_load[1 + kMaxBandTiles];
+  uint64_t bar_s[2];
+  uint64_t bar_sg, bar_sgt, bar_p, bar_pv, bar_fin;
+  uint32_t tmem_base;
+  int abort;
+  int gc[kMaxGlobal];
+  float red[4][kMaxGlobal];
+  float red2[4][kMaxGlobal];
+};
+
+constexpr uint32_t kRowsDyn = kTileBytes * (1 + 2 * kMaxBandTiles) + 2 * kTileBytes +
+                              3 * kGTileBytes + 1024;
+
+__global__ void __launch_bounds__(kThreads, 1)
+    sc_rows_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
+                   const __grid_constant__ CUtensorMap mapV, const LayerParams p) {
+  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int n = __ldg(p.len + b);
+  if (qt * kTile >= n) return;
+  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  const int ngp = ng > 0 ? kMaxGlobal : 0;
+
+  extern __shared__ uint8_t dyn_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* Qs = base;
+  uint8_t* Ks = Qs + kTileBytes;                      // kMaxBandTiles tiles
+  uint8_t* Vs = Ks + kMaxBandTiles * kTileBytes;      // kMaxBandTiles tiles
+  uint8_t* Ps = Vs + kMaxBandTiles * kTileBytes;      // 32 KB (two 64-key halves)
+  uint8_t* KG = Ps + 2 * kTileBytes;
+  uint8_t* VG = KG + kGTileBytes;
+  uint8_t* QG = VG + kGTileBytes;
+  __shared__ RowsSmem sm;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int r0 = qt * kTile;
+  const int r1 = min(r0 + kTile - 1, n - 1);
+  const int kt_lo = max(0, r0 - p.w) / kTile;
+  const int kt_hi = min(n - 1, r1 + p.w) / kTile;
+  const int nb = kt_hi - kt_lo + 1;   // <= kMaxBandTiles (checked on the host)
+  const int ic = qt - kt_lo;          // index of the diagonal key tile
+
+  if (tid == 0) {
+    for (int i = 0; i < 1 + kMaxBandTiles; ++i) mbar_init(&sm.bar_load[i], 1);
+    mbar_init(&sm.bar_s[0], 1);
+    mbar_init(&sm.bar_s[1], 1);
+    mbar_init(&sm.bar_sg, 1);
+    mbar_init(&sm.bar_sgt, 1);
+    mbar_init(&sm.bar_p, 128);
+    mbar_init(&sm.bar_pv, 1);
+    mbar_init(&sm.bar_fin, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
+  if (warp == 5) tmem_alloc(&sm.tmem_base, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = sm.tmem_base;
+  const uint32_t tS0 = tm, tS1 = tm + 128, tO = tm + 256, tSG = tm + 320, tSGt = tm + 352;
+  volatile int* abort_flag = &sm.abort;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------- loads
+    if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[0], kTileBytes + 3 * ngp * 128);
+    __syncwarp();
+    load_tile(p, &mapQ, Qs, b, h, r0, n, &sm.bar_load[0], lane);
+    if (ngp) {
+      load_globals(p, &mapK, KG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
+      load_globals(p, &mapV, VG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
+      load_globals(p, &mapQ, QG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
+    }
+    for (int i = 0; i < nb; ++i) {
+      if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[1 + i], 2 * kTileBytes);
+      __syncwarp();
+      const int c0 = (kt_lo + i) * kTile;
+      load_tile(p, &mapK, Ks + i * kTileBytes, b, h, c0, n, &sm.bar_load[1 + i], lane);
+      load_tile(p, &mapV, Vs + i * kTileBytes, b, h, c0, n, &sm.bar_load[1 + i], lane);
+    }
+    if (lane == 0)
+      for (int i = 0; i <= nb; ++i) drain_wait(&sm.bar_load[i], 0);
+  } else if (warp == 5) {
+    // ------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      const uint32_t q_a = smem_u32(Qs), k_a = smem_u32(Ks), v_a = smem_u32(Vs);
+      const uint32_t p_a = smem_u32(Ps);
+      int p_use = 0;
+      bool ok = mbar_wait(&sm.bar_load[0], 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        if (ngp) {
+          mma_qk(tSG, q_a, smem_u32(KG), 16);
+          umma_commit(&sm.bar_sg);
+        }
+      }
+      for (int i = 0; ok && i < min(nb, 2); ++i) {
+        if (!(ok = mbar_wait(&sm.bar_load[1 + i], 0, abort_flag))) break;
+        tc_fence_after();
+        mma_qk(i ? tS1 : tS0, q_a, k_a + i * kTileBytes, 128);
+        umma_commit(&sm.bar_s[i & 1]);
+        if (ngp && i == ic) {
+          mma_qk(tSGt, k_a + i * kTileBytes, smem_u32(QG), 16);
+          umma_commit(&sm.bar_sgt);
+        }
+      }
+      if (ok && ngp) {
+        if ((ok = mbar_wait(&sm.bar_p, p_use & 1, abort_flag))) {
+          tc_fence_after();
+          mma_pv(tO, p_a, smem_u32(VG), kMaxGlobal / 16, false);
+          umma_commit(&sm.bar_pv);
+          ++p_use;
+        }
+      }
+      for (int i = 0; ok && i < nb; ++i) {
+        if (!(ok = mbar_wait(&sm.bar_p, p_use & 1, abort_flag))) break;
+        tc_fence_after();
+        mma_pv(tO, p_a, v_a + i * kTileBytes, kTile / 16, ngp > 0 || i > 0);
+        umma_commit(&sm.bar_pv);
+        ++p_use;
+        const int j = i + 2;
+        if (j < nb) {
+          if (!(ok = mbar_wait(&sm.bar_load[1 + j], 0, abort_flag))) break;
+          tc_fence_after();
+          mma_qk((j & 1) ? tS1 : tS0, q_a, k_a + j * kTileBytes, 128);
+          umma_commit(&sm.bar_s[j & 1]);
+          if (ngp && j == ic) {
+            mma_qk(tSGt, k_a + j * kTileBytes, smem_u32(QG), 16);
+            umma_commit(&sm.bar_sgt);
+          }
+        }
+      }
+      umma_commit(&sm.bar_fin);
+      drain_wait(&sm.bar_fin, 0);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------- softmax
+    const int r = tid;            // row inside the tile == TMEM lane
+    const int i = r0 + r;         // current index of this query row
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    bool row_global = false;
+    for (int g = 0; g < ng; ++g) row_global |= (sm.gc[g] == i);
+    const bool valid = (i < n) && !row_global;
+    // allowed band keys of this row (current index), inclusive
+    const int lo = valid ? max(0, i - p.w) : 0;
+    const int hi = valid ? min(n - 1, i + p.w) : n - 1;
+
+    float m_ref = -INFINITY, lsum = 0.f;
+    int p_use = 0;
+    bool ok = true;
+    bool o_written = false;
+    float x[128];
+
+    if (ngp) {
+      ok = warp_wait(&sm.bar_sg, 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        tmem_ld16(tSG + lane_off, x);
+        tmem_ld_wait();
+        float mx = -INFINITY;
+#pragma unroll
+        for (int g = 0; g < kMaxGlobal; ++g) {
+          const int cg = sm.gc[g];
+          const bool use = (g < ng) && (!valid || abs(i - cg) > p.w);
+          x[g] = use ? x[g] * kLogitScale2 : -INFINITY;
+          mx = fmaxf(mx, x[g]);
+        }
+        m_ref = mx;
+        const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
+        uint32_t pk[8];
+#pragma unroll
+        for (int g = 0; g < kMaxGlobal; g += 2) {
+          const float a = ex2(x[g] - ref), c = ex2(x[g + 1] - ref);
+          lsum += a + c;
+          pk[g / 2] = pack_bf16x2(a, c);
+        }
+        *reinterpret_cast<uint4*>(Ps + sw128_offset(r, 0)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        *reinterpret_cast<uint4*>(Ps + sw128_offset(r, 1)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(&sm.bar_p);
+        ++p_use;
+        o_written = true;
+      }
+    }
+
+    for (int t = 0; ok && t < nb; ++t) {
+      const int j0 = (kt_lo + t) * kTile;
+      if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
+      tc_fence_after();
+      const uint32_t ts = (t & 1) ? tS1 : tS0;
+#pragma unroll
+      for (int c = 0; c < 128; c += 32) tmem_ld32(ts + lane_off + c, x + c);
+      tmem_ld_wait();
+      const bool full = (lo <= j0) && (j0 + kTile - 1 <= hi);
+      float mx = -INFINITY;
+      if (__all_sync(0xffffffffu, full)) {
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          x[c] *= kLogitScale2;
+          mx = fmaxf(mx, x[c]);
+        }
+      } else {
+        const int a = lo - j0, e = hi - j0;
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          x[c] = (c >= a && c <= e) ? x[c] * kLogitScale2 : -INFINITY;
+          mx = fmaxf(mx, x[c]);
+        }
+      }
+      // lazy rescale: move the reference only when the tile max exceeds it by > 8 (2^8)
+      float scale = 1.f;
+      const bool bump = mx > m_ref + 8.f;
+      float new_ref = m_ref;
+      if (bump) {
+        new_ref = mx;
+        scale = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - new_ref);
+      }
+      const float ref = (new_ref == -INFINITY) ? 0.f : new_ref;
+      float ts_sum = 0.f;
+      uint32_t pk[64];
+#pragma unroll
+      for (int c = 0; c < 128; c += 2) {
+        const float a = ex2(x[c] - ref), d = ex2(x[c + 1] - ref);
+        ts_sum += a + d;
+        pk[c / 2] = pack_bf16x2(a, d);
+      }
+      lsum = lsum * scale + ts_sum;
+      m_ref = new_ref;
+      // the previous P V must be done before P is overwritten or O rescaled
+      if (p_use > 0) {
+        if (!(ok = warp_wait(&sm.bar_pv, (p_use - 1) & 1, abort_flag))) break;
+        tc_fence_after();
+      }
+      if (__any_sync(0xffffffffu, bump && o_written)) {
+        const float f = (bump && o_written) ? scale : 1.f;
+        float o[32];
+#pragma unroll
+        for (int c = 0; c < 64; c += 32) {
+          tmem_ld32(tO + lane_off + c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 32; ++k) o[k] *= f;
+          tmem_st32(tO + lane_off + c, o);
+        }
+        tmem_st_wait();
+      }
+#pragma unroll
+      for (int c = 0; c < 16; ++c)
+        *reinterpret_cast<uint4*>(Ps + (c >> 3) * 16384 + sw128_offset(r, c & 7)) =
+            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&sm.bar_p);
+      ++p_use;
+      o_written = true;
+    }
+
+    // ---- epilogue: O, LSE
+    float lse = INFINITY;
+    if (ok && (ok = warp_wait(&sm.bar_pv, (p_use - 1) & 1, abort_flag))) {
+      tc_fence_after();
+      const float inv = 1.f / lsum;
+      lse = valid ? m_ref + lg2(lsum) : INFINITY;
+      uint16_t* orow = p.O + ((static_cast<size_t>(b) * p.L + i) * p.H + h) * kHeadDim;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        float o[32];
+        tmem_ld32(tO + lane_off + c, o);
+        tmem_ld_wait();
+        if (valid) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 8) {
+            uint4 v = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
+                                 pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
+                                 pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
+                                 pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
+            *reinterpret_cast<uint4*>(orow + c + k) = v;
+          }
+        }
+      }
+    }
+    if (i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
+
+    if (ngp) {
+      // far-row column sums of the global keys: rows outside the key's band
+      float part[kMaxGlobal];
+      if (ok) {
+        tmem_ld16(tSG + lane_off, x);
+        tmem_ld_wait();
+      }
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        const int cg = sm.gc[g];
+        const bool use = ok && valid && (g < ng) && abs(i - cg) > p.w;
+        part[g] = use ? ex2(x[g] * kLogitScale2 - lse) : 0.f;
+        part[g] = warp_sum(part[g]);
+      }
+      if (lane == 0)
+        for (int g = 0; g < kMaxGlobal; ++g) sm.red[warp][g] = part[g];
+      // (max, sum) of each global row over this tile's keys j = 128 qt + r
+      bool ok2 = ok && warp_wait(&sm.bar_sgt, 0, abort_flag);
+      if (ok2) {
+        tc_fence_after();
+        tmem_ld16(tSGt + lane_off, x);
+        tmem_ld_wait();
+      }
+      const bool key_ok = ok2 && (r0 + r < n);
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        x[g] = key_ok ? x[g] * kLogitScale2 : -INFINITY;
+        part[g] = warp_max(x[g]);
+      }
+      if (lane == 0)
+        for (int g = 0; g < kMaxGlobal; ++g) sm.red2[warp][g] = part[g];
+      named_sync_softmax();
+      float gm[kMaxGlobal];
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        gm[g] = fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
+        const float e = (key_ok && gm[g] != -INFINITY) ? ex2(x[g] - gm[g]) : 0.f;
+        part[g] = warp_sum(e);
+      }
+      named_sync_softmax();
+      if (lane == 0)
+        for (int g = 0; g < kMaxGlobal; ++g) sm.red2[warp][g] = part[g];
+      named_sync_softmax();
+      if (tid < kMaxGlobal) {
+        const int g = tid;
+        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + g;
+        p.gpart[slot] = sm.red[0][g] + sm.red[1][g] + sm.red[2][g] + sm.red[3][g];
+        p.gstat[2 * slot] = gm[g];
+        p.gstat[2 * slot + 1] = sm.red2[0][g] + sm.red2[1][g] + sm.red2[2][g] + sm.red2[3][g];
+      }
+      if (qt == 0) {
+        float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
+        for (int k = tid; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
+  if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------------------
+// cols kernel
+// ---------------------------------------------------------------------------
+struct ColsSmem {
+  uint64_t bar_load[1 + kMaxBandTiles];
+  uint64_t bar_s[2], bar_sfree[2];
+  uint64_t bar_sg, bar_pg, bar_og, bar_fin;
+  uint32_t tmem_base;
+  int abort;
+  int gc[kMaxGlobal];
+  float lse_g[kMaxGlobal];
+  float lse[kMaxBandTiles * kTile];
+  int flag;
+  int scan[kThreads];
+  int gnew[kMaxGlobal];
+};
+
+constexpr uint32_t kColsDyn = kTileBytes * (2 + kMaxBandTiles) + kGTileBytes + 2 * kTileBytes + 1024;
+
+__device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm);
+
+__global__ void __launch_bounds__(kThreads, 1)
+    sc_cols_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
+                   const __grid_constant__ CUtensorMap mapV, const LayerParams p) {
+  const int kt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int n = __ldg(p.len + b);
+  if (n == 0) {
+    if (kt == 0 && h == 0 && threadIdx.x == 0) {
+      p.len_out[b] = 0;
+      p.ng_out[b] = 0;
+    }
+    return;
+  }
+  if (kt * kTile >= n) return;
+  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  const int ngp = ng > 0 ? kMaxGlobal : 0;
+  const int Tn = (n + kTile - 1) / kTile;
+
+  extern __shared__ uint8_t dyn_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* Ks = base;
+  uint8_t* Vs = Ks + kTileBytes;
+  uint8_t* Pg = Vs + kTileBytes;                  // 32 KB: A operand of the global-row P V
+  uint8_t* Qs = Pg + 2 * kTileBytes;              // kMaxBandTiles tiles
+  uint8_t* QG = Qs + kMaxBandTiles * kTileBytes;
+  __shared__ ColsSmem sm;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int j0 = kt * kTile;
+  const int j1 = min(j0 + kTile - 1, n - 1);
+  const int qt_lo = max(0, j0 - p.w) / kTile;
+  const int qt_hi = min(n - 1, j1 + p.w) / kTile;
+  const int nq = qt_hi - qt_lo + 1;
+
+  if (tid == 0) {
+    for (int i = 0; i < 1 + kMaxBandTiles; ++i) mbar_init(&sm.bar_load[i], 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.bar_s[i], 1);
+      mbar_init(&sm.bar_sfree[i], 128);
+    }
+    mbar_init(&sm.bar_sg, 1);
+    mbar_init(&sm.bar_pg, 128);
+    mbar_init(&sm.bar_og, 1);
+    mbar_init(&sm.bar_fin, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
+  if (warp == 5) tmem_alloc(&sm.tmem_base, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tm = sm.tmem_base;
+  const uint32_t tS0 = tm, tS1 = tm + 128, tSG = tm + 256, tOG = tm + 320;
+  volatile int* abort_flag = &sm.abort;
+
+  if (warp == 4) {
+    if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[0], 2 * kTileBytes + ngp * 128);
+    __syncwarp();
+    load_tile(p, &mapK, Ks, b, h, j0, n, &sm.bar_load[0], lane);
+    load_tile(p, &mapV, Vs, b, h, j0, n, &sm.bar_load[0], lane);
+    if (ngp) load_globals(p, &mapQ, QG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
+    for (int i = 0; i < nq; ++i) {
+      if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[1 + i], kTileBytes);
+      __syncwarp();
+      load_tile(p, &mapQ, Qs + i * kTileBytes, b, h, (qt_lo + i) * kTile, n,
+                &sm.bar_load[1 + i], lane);
+    }
+    if (lane == 0)
+      for (int i = 0; i <= nq; ++i) drain_wait(&sm.bar_load[i], 0);
+  } else if (warp == 5) {
+    if (lane == 0) {
+      const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs);
+      bool ok = mbar_wait(&sm.bar_load[0], 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        if (ngp) {
+          mma_qk(tSG, k_a, smem_u32(QG), 16);
+          umma_commit(&sm.bar_sg);
+        }
+      }
+      for (int i = 0; ok && i < min(nq, 2); ++i) {
+        if (!(ok = mbar_wait(&sm.bar_load[1 + i], 0, abort_flag))) break;
+        tc_fence_after();
+        mma_qk(i ? tS1 : tS0, k_a, q_a + i * kTileBytes, 128);
+        umma_commit(&sm.bar_s[i]);
+      }
+      for (int i = 0; ok && i + 2 < nq; ++i) {
+        const int j = i + 2;
+        if (!(ok = mbar_wait(&sm.bar_sfree[i & 1], (i >> 1) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait(&sm.bar_load[1 + j], 0, abort_flag))) break;
+        tc_fence_after();
+        mma_qk((j & 1) ? tS1 : tS0, k_a, q_a + j * kTileBytes, 128);
+        umma_commit(&sm.bar_s[j & 1]);
+      }
+      if (ok && ngp && (ok = mbar_wait(&sm.bar_pg, 0, abort_flag))) {
+        tc_fence_after();
+        mma_pv(tOG, smem_u32(Pg), smem_u32(Vs), kTile / 16, false);
+        umma_commit(&sm.bar_og);
+      }
+      umma_commit(&sm.bar_fin);
+      drain_wait(&sm.bar_fin, 0);
+    }
+    __syncwarp();
+  } else {
+    const int r = tid;
+    const int j = j0 + r;             // key column owned by this thread
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const float* lse_src = p.lse + (static_cast<size_t>(b) * p.H + h) * p.L;
+    for (int k = tid; k < nq * kTile; k += 128) {
+      const int row = qt_lo * kTile + k;
+      sm.lse[k] = row < n ? __ldcg(lse_src + row) : INFINITY;
+    }
+    if (ngp && warp == 0) {
+      // merge the per-tile (max, sum) of every global row into its LSE
+      for (int g = 0; g < ng; ++g) {
+        float m = -INFINITY, s = 0.f;
+        if (lane < Tn) {
+          const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + lane) * kMaxGlobal + g;
+          m = __ldcg(p.gstat + 2 * slot);
+          s = __ldcg(p.gstat + 2 * slot + 1);
+        }
+        const float M = warp_max(m);
+        const float part = (lane < Tn && m != -INFINITY) ? s * ex2(m - M) : 0.f;
+        const float S = warp_sum(part);
+        if (lane == 0) sm.lse_g[g] = M + lg2(S);
+      }
+    }
+    named_sync_softmax();
+
+    float acc = 0.f;
+    bool ok = true;
+    float x[128];
+    for (int t = 0; ok && t < nq; ++t) {
+      if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
+      tc_fence_after();
+      const uint32_t ts = (t & 1) ? tS1 : tS0;
+#pragma unroll
+      for (int c = 0; c < 128; c += 32) tmem_ld32(ts + lane_off + c, x + c);
+      tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(&sm.bar_sfree[t & 1]);
+      const int i0 = (qt_lo + t) * kTile;            // first query row of this tile
+      const float* lw = sm.lse + t * kTile;
+      const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
+      float s = 0.f;
+      if (__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
+#pragma unroll
+        for (int c = 0; c < 128; ++c) s += ex2(x[c] * kLogitScale2 - lw[c]);
+      } else {
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          const float v = ex2(x[c] * kLogitScale2 - lw[c]);
+          s += (c >= a && c <= e) ? v : 0.f;
+        }
+      }
+      acc += s;
+    }
+
+    if (ngp) {
+      bool ok2 = ok && warp_wait(&sm.bar_sg, 0, abort_flag);
+      if (ok2) {
+        tc_fence_after();
+        tmem_ld16(tSG + lane_off, x);
+        tmem_ld_wait();
+      }
+      uint16_t pb[kMaxGlobal];
+      float s = 0.f;
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        const float v = (ok2 && g < ng && j < n) ? ex2(x[g] * kLogitScale2 - sm.lse_g[g]) : 0.f;
+        s += v;
+        pb[g] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+      }
+      acc += s;
+      // P of the global rows, transposed into the A tile: row g, column (key) r
+      uint8_t* col = Pg + (r >> 6) * 16384;
+      const int ch = (r & 63) >> 3, wi = (r & 7) * 2;
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g)
+        *reinterpret_cast<uint16_t*>(col + sw128_offset(g, ch) + wi) = pb[g];
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&sm.bar_pg);
+      bool ok3 = ok2 && warp_wait(&sm.bar_og, 0, abort_flag);
+      if (warp == 0 && ok3) {
+        tc_fence_after();
+        float* og = p.og + ((static_cast<size_t>(b) * p.H + h) * kMaxGlobal) * kHeadDim;
+#pragma unroll
+        for (int c = 0; c < 64; c += 32) {
+          float o[32];
+          tmem_ld32(tOG + lane_off + c, o);
+          tmem_ld_wait();
+          if (lane < ng)
+            for (int k = 0; k < 32; ++k) atomicAdd(og + lane * kHeadDim + c + k, o[k]);
+        }
+      }
+    }
+    if (j < n) p.acc[(static_cast<size_t>(b) * p.H + h) * p.L + j] = acc;
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tm, 512);
+  }
+  if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
+
+  // ---- last head of this key tile: scores and keep flags (fixed head order)
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) sm.flag = (atomicAdd(p.cnt_tile + b * p.T + kt, 1u) == static_cast<uint32_t>(p.H - 1));
+  __syncthreads();
+  if (!sm.flag) return;
+  __threadfence();
+  if (tid < kTile && j0 + tid < n) {
+    const int jj = j0 + tid;
+    float a = 0.f;
+    for (int hh = 0; hh < p.H; ++hh) a += __ldcg(p.acc + (static_cast<size_t>(b) * p.H + hh) * p.L + jj);
+    for (int g = 0; g < ng; ++g) {
+      if (sm.gc[g] != jj) continue;
+      for (int hh = 0; hh < p.H; ++hh)
+        for (int q = 0; q < Tn; ++q)
+          a += __ldcg(p.gpart + ((static_cast<size_t>(b) * p.H + hh) * p.T + q) * kMaxGlobal + g);
+    }
+    const float s = a / static_cast<float>(p.H * n);
+    p.scores[static_cast<size_t>(b) * p.L + jj] = s;
+    const float theta = p.theta ? __ldg(p.theta + b) : p.alpha / static_cast<float>(n);
+    p.keep[static_cast<size_t>(b) * p.L + jj] = (jj == 0 || s >= theta) ? 1 : 0;
+  }
+  if (tid == 0) p.cnt_tile[b * p.T + kt] = 0u;
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) sm.flag = (atomicAdd(p.cnt_seq + b, 1u) == static_cast<uint32_t>(Tn - 1));
+  __syncthreads();
+  if (!sm.flag) return;
+  __threadfence();
+  finalize_sequence(p, b, n, sm);
+}
+
+// Order-preserving compaction of sequence b's kept tokens, the next layer's
+// global list, and the bf16 outputs of the global rows.  One CTA.
+__device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm) {
+  const int tid = threadIdx.x;
+  const int per = (n + kThreads - 1) / kThreads;
+  const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
+  const uint8_t* keep = p.keep + static_cast<size_t>(b) * p.L;
+  int cnt = 0;
+  for (int c = c0; c < c1; ++c) cnt += __ldcg(keep + c);
+  sm.scan[tid] = cnt;
+  __syncthreads();
+  // exclusive scan over kThreads counts (Hillis-Steele in shared memory)
+  for (int off = 1; off < kThreads; off <<= 1) {
+    const int v = tid >= off ? sm.scan[tid - off] : 0;
+    __syncthreads();
+    sm.scan[tid] += v;
+    __syncthreads();
+  }
+  int out = sm.scan[tid] - cnt;
+  const int total = sm.scan[kThreads - 1];
+  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  if (tid < kMaxGlobal) sm.gnew[tid] = -1;
+  __syncthreads();
+  const int32_t* pos = p.pos + static_cast<size_t>(b) * p.L;
+  int32_t* pos_out = p.pos_out + static_cast<size_t>(b) * p.L;
+  for (int c = c0; c < c1; ++c) {
+    if (!__ldcg(keep + c)) continue;
+    pos_out[out] = __ldg(pos + c);
+    for (int g = 0; g < ng; ++g)
+      if (sm.gc[g] == c) sm.gnew[g] = out;
+    ++out;
+  }
+  // bf16 outputs of the global rows
+  for (int k = tid; k < ng * p.H * kHeadDim; k += kThreads) {
+    const int g = k / (p.H * kHeadDim), hh = (k / kHeadDim) % p.H, dd = k % kHeadDim;
+    const float v = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
+    p.O[((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) * kHeadDim + dd] =
+        __bfloat16_as_ushort(__float2bfloat16_rn(v));
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int m = 0;
+    for (int g = 0; g < ng; ++g)
+      if (sm.gnew[g] >= 0) p.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
+    p.ng_out[b] = m;
+    p.len_out[b] = total;
+    p.cnt_seq[b] = 0u;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// prep kernel: padding removal (stack) or global-token lookup (single layer)
+// ---------------------------------------------------------------------------
+constexpr int kPrepThreads = 1024;
+
+__global__ void __launch_bounds__(kPrepThreads)
+    sc_prep_kernel(const PrepParams pp) {
+  const int b = blockIdx.x, tid = threadIdx.x;
+  __shared__ int scan[kPrepThreads];
+  __shared__ int spos[kMaxLen];
+  __shared__ int s_n;
+  int n;
+  if (pp.pos_in == nullptr) {
+    // stack mode: real tokens of the padded sequence, in order
+    const int L = pp.L;
+    const int per = (L + kPrepThreads - 1) / kPrepThreads;
+    const int c0 = min(L, tid * per), c1 = min(L, c0 + per);
+    int cnt = 0;
+    for (int c = c0; c < c1; ++c)
+      cnt += pp.pad_mask ? (pp.pad_mask[static_cast<size_t>(b) * L + c] != 0) : 1;
+    scan[tid] = cnt;
+    __syncthreads();
+    for (int off = 1; off < kPrepThreads; off <<= 1) {
+      const int v = tid >= off ? scan[tid - off] : 0;
+      __syncthreads();
+      scan[tid] += v;
+      __syncthreads();
+    }
+    int out = scan[tid] - cnt;
+    for (int c = c0; c < c1; ++c) {
+      if (pp.pad_mask && !pp.pad_mask[static_cast<size_t>(b) * L + c]) continue;
+      pp.pos_out[static_cast<size_t>(b) * L + out] = c;
+      spos[out] = c;
+      ++out;
+    }
+    if (tid == kPrepThreads - 1) {
+      s_n = scan[kPrepThreads - 1];
+      pp.len_out[b] = s_n;
+    }
+  } else {
+    if (tid == 0) s_n = pp.len_in[b];
+    __syncthreads();
+    for (int c = tid; c < s_n; c += kPrepThreads) spos[c] = pp.pos_in[static_cast<size_t>(b) * pp.L + c];
+  }
+  __syncthreads();
+  n = s_n;
+  if (tid == 0) {
+    // global positions are sorted and positions increase with the current
+    // index, so the matches come out in increasing current order
+    int m = 0;
+    for (int g = 0; g < pp.n_global; ++g) {
+      const int target = pp.global_pos[g];
+      int lo = 0, hi = n - 1;
+      while (lo <= hi) {
+        const int mid = (lo + hi) >> 1;
+        if (spos[mid] < target) lo = mid + 1;
+        else hi = mid - 1;
+      }
+      if (lo < n && spos[lo] == target) pp.gcur[b * kMaxGlobal + m++] = lo;
+    }
+    pp.ng[b] = m;
+  }
+}
+
+}  // namespace sc
+
+// ---------------------------------------------------------------------------
+// launch helpers used by the C ABI
+// ---------------------------------------------------------------------------
+namespace sc {
+
+cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st) {
+  sc_prep_kernel<<<pp.B, kPrepThreads, 0, st>>>(pp);
+  return cudaGetLastError();
+}
+
+cudaError_t configure_kernels() {
+  cudaError_t e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(kRowsDyn));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(sc_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(kColsDyn));
+}
+
+cudaError_t launch_layer(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
+                         const LayerParams& p, cudaStream_t st) {
+  dim3 grid(p.T, p.H, p.B);
+  sc_rows_kernel<<<grid, kThreads, kRowsDyn, st>>>(mq, mk, mv, p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  sc_cols_kernel<<<grid, kThreads, kColsDyn, st>>>(mq, mk, mv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace sc

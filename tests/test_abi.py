@@ -1,0 +1,112 @@
+"""The C ABI without a GPU: the library loads, exports every function that
+include/sparsecoder.h declares, and rejects bad arguments on the host before
+anything is launched (so these calls never reach the device)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2310_07109_gb300 import binding as bd
+from paper_2310_07109_gb300 import build as bld
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "sparsecoder.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    bld.build_library()
+    return bd.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:size_t|int|const char\*)\s+(sc_\w+)\s*\(", text, re.M)))
+
+
+def test_header_declares_the_documented_calls():
+    names = declared_functions()
+    assert set(bd.EXPORTED) <= set(names)
+    assert "sc_layer_forward" in names and "sc_stack_forward" in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    raw = ctypes.CDLL(bd.library_path())
+    for name in declared_functions():
+        assert hasattr(raw, name), name
+
+
+def test_status_strings(lib):
+    for code in range(6):
+        assert bd.status_string(code).startswith("SC_")
+    assert "unknown" in bd.status_string(99)
+
+
+def test_workspace_size(lib):
+    assert bd.workspace_size(2, 4096, 12) > 2 * 12 * 4096 * 8
+    assert bd.workspace_size(0, 10, 1) == 0
+    assert bd.workspace_size(1, 4097, 1) == 0
+    assert bd.workspace_size(1, 1, 1) % 256 == 0
+
+
+FAKE = 1 << 40  # host-side validation never dereferences device pointers
+
+
+def _layer_args(**kw):
+    g = (ctypes.c_int32 * 2)(0, 5)
+    a = dict(B=1, L=256, H=12, w=64, Q=FAKE, K=FAKE, V=FAKE, len=FAKE, pos=FAKE,
+             global_pos=ctypes.cast(g, ctypes.POINTER(ctypes.c_int32)), n_global=2, alpha=0.5,
+             theta=None, O=FAKE, scores=FAKE, pos_out=FAKE + 4096, len_out=FAKE + 8192)
+    a.update(kw)
+    return bd.LayerArgs(**a), g
+
+
+def _call_layer(lib, ws=FAKE, ws_bytes=1 << 30, **kw):
+    a, keep = _layer_args(**kw)
+    return lib.sc_layer_forward(ctypes.byref(a), ctypes.c_void_p(ws), ws_bytes, None)
+
+
+def test_layer_rejects_bad_arguments(lib):
+    assert lib.sc_layer_forward(None, None, 0, None) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, Q=None) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, B=0) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, w=-1) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, L=5000) == bd.SC_ERR_UNSUPPORTED
+    assert _call_layer(lib, L=2048, w=300) == bd.SC_ERR_UNSUPPORTED
+    assert _call_layer(lib, n_global=17) == bd.SC_ERR_UNSUPPORTED
+    assert _call_layer(lib, Q=FAKE + 8) == bd.SC_ERR_INVALID_ARG        # not 16-byte aligned
+    assert _call_layer(lib, pos_out=FAKE) == bd.SC_ERR_INVALID_ARG      # aliases pos
+    assert _call_layer(lib, ws=None) == bd.SC_ERR_WORKSPACE
+    assert _call_layer(lib, ws_bytes=16) == bd.SC_ERR_WORKSPACE
+    assert _call_layer(lib, ws=FAKE + 128) == bd.SC_ERR_WORKSPACE       # not 256-byte aligned
+    bad = (ctypes.c_int32 * 2)(5, 0)                                      # unsorted
+    assert _call_layer(lib, global_pos=ctypes.cast(bad, ctypes.POINTER(ctypes.c_int32))) \
+        == bd.SC_ERR_INVALID_ARG
+    dup = (ctypes.c_int32 * 2)(3, 3)
+    assert _call_layer(lib, global_pos=ctypes.cast(dup, ctypes.POINTER(ctypes.c_int32))) \
+        == bd.SC_ERR_INVALID_ARG
+    far = (ctypes.c_int32 * 2)(0, 256)                                    # outside [0, L)
+    assert _call_layer(lib, global_pos=ctypes.cast(far, ctypes.POINTER(ctypes.c_int32))) \
+        == bd.SC_ERR_INVALID_ARG
+
+
+def test_stack_rejects_bad_arguments(lib):
+    g = (ctypes.c_int32 * 1)(0)
+    al = (ctypes.c_float * 12)(*([0.5] * 12))
+
+    def call(**kw):
+        a = dict(n_layers=12, B=2, L=1024, H=12, w=256, Q=FAKE, K=FAKE, V=FAKE, pad_mask=None,
+                 global_pos=ctypes.cast(g, ctypes.POINTER(ctypes.c_int32)), n_global=1,
+                 alpha=ctypes.cast(al, ctypes.POINTER(ctypes.c_float)), O=FAKE, scores=FAKE,
+                 pos=FAKE, len=FAKE)
+        a.update(kw)
+        return lib.sc_stack_forward(ctypes.byref(bd.StackArgs(**a)), ctypes.c_void_p(FAKE),
+                                    1 << 30, None)
+
+    assert call(n_layers=0) == bd.SC_ERR_INVALID_ARG
+    assert call(alpha=None) == bd.SC_ERR_INVALID_ARG
+    assert call(O=None) == bd.SC_ERR_INVALID_ARG
+    assert call(V=FAKE + 2) == bd.SC_ERR_INVALID_ARG
+    assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
+    assert call(w=512) == bd.SC_ERR_UNSUPPORTED

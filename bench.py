@@ -1,0 +1,406 @@
+#!/usr/bin/env python
+"""Throughput of the SparseCoder hot path on GB300: kept tokens per second of the
+12-layer pruned sparse-attention stack at L = 4096 (and its roofline fraction).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
+                    [--workload cfg4|cfg2|cfg3|cfg5_L512|...|cfg5_L4096[_theta0]]
+
+One step = one call of sc_stack_forward over the whole workload: padding removal,
+then per layer the rows kernel (band + global attention, O, row LSE) and the
+cols kernel (column scores, threshold, compaction), 12 layers, inputs resident in
+HBM.  The default workload is the 12-layer stack B=2, L=4096, H=12, d=64, window
++-256, token 0 plus 8 seeded global positions, 5% salient keys x4, alpha 0.4->1.0.
+The inputs of one step (453 MB of Q/K/V) are larger than the 129 MB L2, so no
+flush is needed between steps.
+
+Metric: kept tokens/s = sum over layers and sequences of the tokens entering the
+layer (token-layers processed) / stack time.  Under torchrun each rank runs an
+independent replica (weak scaling, no collective on the data path); value is the
+sum over ranks divided by the slowest rank's time.
+
+--impl reference times the fp64 CPU oracle (the only reference this method has)
+on the host cores, each step a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as wk  # noqa: E402
+
+METRIC = "kept-tokens/sec per 12-layer pruned stack at L=4096; fraction of roofline"
+UNIT = "kept-tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+BYTES_PER_TOKEN = 6152      # Q,K,V read (3*12*64*2) + O write (12*64*2) + score (4) + position (4)
+FLOPS_PER_PAIR = 4 * 64 * 12  # QK^T and PV, multiply-add = 2 flops, 12 heads
+
+
+def pick_workload(name: str) -> wk.Workload:
+    if name in wk.CONFIGS:
+        return wk.CONFIGS[name]
+    if name.startswith("cfg5_L"):
+        rest = name[len("cfg5_L"):]
+        control = rest.endswith("_theta0")
+        return wk.cfg5(int(rest.replace("_theta0", "")), control=control)
+    raise SystemExit("unknown workload %s" % name)
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work of one (sequence, layer)
+# ---------------------------------------------------------------------------
+def nnz_allowed(n: int, w: int, gcur) -> int:
+    """Number of (query, key) pairs in the allowed sets of n current tokens."""
+    if n == 0:
+        return 0
+    i = np.arange(n)
+    band = np.minimum(n - 1, i + w) - np.maximum(0, i - w) + 1
+    isg = np.zeros(n, bool)
+    isg[list(gcur)] = True
+    total = int(band[~isg].sum())
+    for g in gcur:  # global keys outside the band of non-global rows
+        far = (~isg) & (np.abs(i - g) > w)
+        total += int(far.sum())
+    total += int(isg.sum()) * n  # global rows see every key
+    return total
+
+
+def layer_work(wl, inp, pos, lens):
+    """[n_layers] lists of (bytes, flops) summed over the batch, from the kept sets."""
+    gset = set(int(g) for g in inp["global_pos"])
+    out = []
+    for l in range(wl.n_layers):
+        B_, F_ = 0, 0
+        for b in range(wl.B):
+            n = int(lens[l, b])
+            gcur = [c for c in range(n) if int(pos[l, b, c]) in gset]
+            B_ += BYTES_PER_TOKEN * n
+            F_ += FLOPS_PER_PAIR * nnz_allowed(n, wl.w, gcur)
+        out.append((B_, F_))
+    return out
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (the reference arm and the cpu_baseline)
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, inp, b, n_layers, threads):
+    """Run the oracle stack on sequence b for the first n_layers layers; returns
+    (seconds, kept tokens processed, threads used)."""
+    import oracle
+    sl = slice(b, b + 1)
+    mask = None if inp["pad_mask"] is None else inp["pad_mask"][sl]
+    Q, K, V = (np.ascontiguousarray(inp[k][:n_layers, sl]) for k in ("Q", "K", "V"))
+    t0 = time.perf_counter()
+    res = oracle.stack(Q, K, V, mask, inp["global_pos"], wl.w, inp["alpha"][:n_layers],
+                       want_O=True, nthreads=threads)
+    dt = time.perf_counter() - t0
+    return dt, int(res["len"][:n_layers].sum()), min(threads, wl.H)
+
+
+def run_reference(args, wl):
+    import oracle
+    oracle.build()
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    inp = wk.make_inputs(wl)
+    threads = oracle.default_threads()
+    layers = max(1, min(wl.n_layers, args.ref_layers))
+    for s in range(args.warmup):
+        oracle_sample(wl, inp, s % wl.B, layers, threads)
+    tot_t, tot_tok = 0.0, 0
+    for s in range(args.steps):
+        dt, tok, cores = oracle_sample(wl, inp, s % wl.B, layers, threads)
+        tot_t += dt
+        tot_tok += tok
+    value = tot_tok / tot_t
+    sample = "one sequence of the workload, first %d layer(s), per step" % layers
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.describe(), "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# native arm
+# ---------------------------------------------------------------------------
+def run_native(args, wl):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2310_07109_gb300 import binding as sc
+    from paper_2310_07109_gb300 import build as sc_build
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    sc_build.build_library()
+    sc.load()
+
+    inp = wk.make_inputs(wl)
+    host = {k: torch.from_numpy(inp[k].view(np.int16)).view(torch.bfloat16).pin_memory()
+            for k in ("Q", "K", "V")}
+    dQKV = {k: host[k].to(dev) for k in host}
+    mask = None if inp["pad_mask"] is None else torch.from_numpy(inp["pad_mask"]).to(dev)
+    ws = sc.new_workspace(wl.B, wl.L, wl.H, dev)
+    out = None
+    alpha = [float(a) for a in inp["alpha"]]
+    gpos = [int(g) for g in inp["global_pos"]]
+
+    def step(events=None):
+        nonlocal out
+        out = sc.stack_forward(dQKV["Q"], dQKV["K"], dQKV["V"], mask, gpos, wl.w, alpha,
+                               out=out, workspace=ws, events=events)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    rc = sc.workspace_status(ws)
+    if rc != 0:
+        raise SystemExit("device status after warm-up: %s" % sc.status_string(rc))
+
+    # ---- timed region: K steps, inputs resident
+    stream = torch.cuda.current_stream()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device()) as clocks:
+        barrier()
+        t0.record(stream)
+        for _ in range(args.steps):
+            step()
+        t1.record(stream)
+        barrier()
+    ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_per_step = ms / args.steps
+    lens = out["len"].cpu().numpy()
+    pos = out["pos"].cpu().numpy()
+    kept_per_step = int(lens[:wl.n_layers].sum())
+    value = world * kept_per_step / (ms_per_step * 1e-3)
+
+    # ---- per-kernel times on the launching stream (same steps, events between kernels)
+    nev = 2 + 3 * wl.n_layers
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(nev)]
+    for e in evs:
+        e.record(stream)
+    torch.cuda.synchronize()
+    rows_ms = np.zeros(wl.n_layers)
+    cols_ms = np.zeros(wl.n_layers)
+    gath_ms = np.zeros(wl.n_layers)
+    prep_ms = 0.0
+    prof_steps = max(1, args.steps)
+    for _ in range(prof_steps):
+        step(evs)
+        torch.cuda.synchronize()
+        prep_ms += evs[0].elapsed_time(evs[1])
+        for l in range(wl.n_layers):
+            rows_ms[l] += evs[1 + 3 * l].elapsed_time(evs[2 + 3 * l])
+            cols_ms[l] += evs[2 + 3 * l].elapsed_time(evs[3 + 3 * l])
+            gath_ms[l] += evs[3 + 3 * l].elapsed_time(evs[4 + 3 * l])
+    rows_ms /= prof_steps
+    cols_ms /= prof_steps
+    gath_ms /= prof_steps
+    prep_ms /= prof_steps
+
+    peaks, peak_src = load_peaks()
+    work = layer_work(wl, inp, pos, lens)
+    bw = peaks["hbm_gbs"] * 1e9
+    fl = peaks["bf16_tflops"] * 1e12
+    t_roof = sum(max(Bb / bw, Ff / fl) for Bb, Ff in work)
+    t_meas = float((rows_ms + cols_ms).sum()) * 1e-3
+    bytes_alg = sum(Bb for Bb, _ in work)
+    flops_alg = sum(Ff for _, Ff in work)
+    hbm_bound = sum(Bb / bw for Bb, _ in work) >= sum(Ff / fl for _, Ff in work)
+    achieved = bytes_alg / t_meas / 1e9 if hbm_bound else flops_alg / t_meas / 1e12
+    l0 = work[0]
+    t_l0 = (rows_ms[0] + cols_ms[0]) * 1e-3
+    roofline = {
+        "bound": "hbm" if hbm_bound else "tensor",
+        "achieved": achieved,
+        "peak": peaks["hbm_gbs"] if hbm_bound else peaks["bf16_tflops"],
+        "unit": "GB/s" if hbm_bound else "TFLOP/s",
+        "frac": t_roof / t_meas,
+        "traffic": None,
+        "peak_source": peak_src,
+        "scope": "sc_rows_kernel + sc_cols_kernel of all layers of one step (the fused "
+                 "sparse-attention + LTP layer); algorithmic bytes 6152 B per token-layer, "
+                 "flops 3072 per allowed (query, key) pair; frac = sum_l max(F_l/peak_bf16, "
+                 "B_l/peak_hbm) / measured kernel time",
+        "layer0_frac": max(l0[0] / bw, l0[1] / fl) / t_l0,
+        "kernel_ms_per_step": {"sc_rows_kernel": float(rows_ms.sum()),
+                               "sc_cols_kernel": float(cols_ms.sum()),
+                               "sc_gather_kernel": float(gath_ms.sum()),
+                               "sc_prep_kernel": prep_ms},
+        "rows_ms_per_layer": [round(float(x), 5) for x in rows_ms],
+        "cols_ms_per_layer": [round(float(x), 5) for x in cols_ms],
+    }
+
+    # ---- end to end through the public API: pinned host inputs in, results out
+    hout = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in out.items()}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in hout.values())
+    e2e_steps = max(1, min(args.steps, 5))
+    barrier()
+    t0.record(stream)
+    for _ in range(e2e_steps):
+        for k in host:
+            dQKV[k].copy_(host[k], non_blocking=True)
+        step()
+        for k in out:
+            hout[k].copy_(out[k], non_blocking=True)
+    t1.record(stream)
+    barrier()
+    e2e_ms = t0.elapsed_time(t1) / e2e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e = {"value": world * kept_per_step / (e2e_ms * 1e-3), "unit": UNIT,
+           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+           "ms_per_step": e2e_ms}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": wl.describe(), "n_layers": wl.n_layers, "batch": wl.B,
+                       "seq_len": wl.L, "heads": wl.H, "head_dim": wl.d, "window": wl.w,
+                       "globals": len(gpos), "parallelism": "replicas" if world > 1 else "single",
+                       "l2": "inputs of one step (%.0f MB) exceed L2; no flush" % (
+                           3 * inp["Q"].nbytes / 1e6),
+                       "kept_tokens_per_step": kept_per_step,
+                       "input_tokens_per_step": int(lens[0].sum()),
+                       "survival": [round(float(x), 4) for x in
+                                    lens[:wl.n_layers + 1].sum(axis=1) / max(1, lens[0].sum())]},
+            "roofline": roofline,
+            "e2e": e2e,
+            "gpu_launches": args.steps * (1 + 3 * wl.n_layers - 1
+                                          + (1 if inp["pad_mask"] is not None else 0)),
+            "clocks": clocks.summary()}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        dt, tok, cores = oracle_sample(wl, inp, 0, wl.n_layers, oracle.default_threads())
+        line["cpu_baseline"] = {"value": tok / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": "sequence 0 of the workload, all %d layers (%d kept "
+                                          "token-layers, %.1f s)" % (wl.n_layers, tok, dt)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--workload", default="cfg4")
+    ap.add_argument("--ref-layers", type=int, default=2,
+                    help="layers of one sequence per reference step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    wl = pick_workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_native(args, wl)
+
+
+if __name__ == "__main__":
+    main()

@@ -145,6 +145,16 @@ int sc_layer_forward(const sc_layer_args* args, void* workspace, size_t workspac
 int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
                      void* stream);
 
+/* sc_stack_forward, plus CUDA events (cudaEvent_t passed as void*) recorded on
+ * `stream` around the kernels, for timing on the launching stream:
+ * events[0] before the first launch, events[1] after the padding-removal
+ * kernel, then for layer l: events[2+3l] after its rows kernel, events[3+3l]
+ * after its cols kernel (scores, threshold, compaction) and events[4+3l] after
+ * the gather of the next layer's rows.  n_events >= 2 + 3 * n_layers.  The
+ * events are caller-owned. */
+int sc_stack_forward_profiled(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
+                              void* stream, void** events, int n_events);
+
 /* Synchronises `stream`, returns SC_ERR_TIMEOUT if any kernel since the last
  * query recorded an expired wait (else SC_OK, or SC_ERR_CUDA), and clears
  * the status word. */
@@ -152,6 +162,11 @@ int sc_workspace_status(void* workspace, size_t workspace_bytes, void* stream);
 
 /* Static, human-readable name of a status code. */
 const char* sc_status_string(int status);
+
+/* Detail of the most recent SC_ERR_CUDA on the calling thread (which step
+ * failed and the CUDA error text); an empty string if none.  Valid until the
+ * next call on this thread. */
+const char* sc_last_error(void);
 
 #ifdef __cplusplus
 }

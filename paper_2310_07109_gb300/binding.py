@@ -52,8 +52,8 @@ class StackArgs(ctypes.Structure):
                 ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p)]
 
 
-EXPORTED = ["sc_layer_forward", "sc_stack_forward", "sc_workspace_size", "sc_workspace_status",
-            "sc_status_string"]
+EXPORTED = ["sc_layer_forward", "sc_stack_forward", "sc_stack_forward_profiled",
+            "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error"]
 
 
 def library_path() -> str:
@@ -82,10 +82,16 @@ def load(build_if_missing: bool = False):
         lib.sc_stack_forward.restype = ctypes.c_int
         lib.sc_stack_forward.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                          ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_stack_forward_profiled.restype = ctypes.c_int
+        lib.sc_stack_forward_profiled.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
+                                                  ctypes.c_size_t, ctypes.c_void_p,
+                                                  ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
         lib.sc_workspace_status.restype = ctypes.c_int
         lib.sc_workspace_status.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         lib.sc_status_string.restype = ctypes.c_char_p
         lib.sc_status_string.argtypes = [ctypes.c_int]
+        lib.sc_last_error.restype = ctypes.c_char_p
+        lib.sc_last_error.argtypes = []
         _lib = lib
         return lib
 
@@ -96,7 +102,10 @@ def status_string(code: int) -> str:
 
 def _check(code: int):
     if code != SC_OK:
-        raise SparseCoderError(code, status_string(code))
+        msg = status_string(code)
+        if code == SC_ERR_CUDA:
+            msg += " (" + load().sc_last_error().decode() + ")"
+        raise SparseCoderError(code, msg)
 
 
 def workspace_size(B: int, L: int, H: int) -> int:
@@ -150,11 +159,13 @@ def layer_forward(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *,
 
 
 def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
-                  stream=None):
+                  stream=None, events=None):
     """The pruned layer stack (``sc_stack_forward``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
     pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers].
+    events: optional list of >= 2 + 2 * n_layers torch.cuda.Event(enable_timing=True),
+    recorded around every kernel on the launching stream (sc_stack_forward_profiled).
     Returns a dict with O, scores, pos, len (device tensors).
     """
     nl, B, L, H, D = Q.shape
@@ -171,7 +182,13 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
                   _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]))
-    _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
+    if events is None:
+        _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
+                                       _stream_handle(stream)))
+    else:
+        handles = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+        _check(load().sc_stack_forward_profiled(ctypes.byref(a), _ptr(ws), ws.numel(),
+                                                _stream_handle(stream), handles, len(events)))
     return out
 
 

@@ -7,6 +7,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <cstdio>
 #include <cstring>
 #include <mutex>
 
@@ -16,8 +17,9 @@
 namespace sc {
 cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st);
 cudaError_t configure_kernels();
-cudaError_t launch_layer(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
-                         const LayerParams& p, cudaStream_t st);
+cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
+cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
+cudaError_t launch_gather(const GatherParams& g, cudaStream_t st);
 }  // namespace sc
 
 namespace {
@@ -26,10 +28,22 @@ using namespace sc;
 
 constexpr size_t kAlign = 256;
 
+// Detail of the most recent failure on this thread (sc_last_error()).
+thread_local char g_last_error[256] = "";
+
+int fail(int code, const char* what, const char* detail) {
+  snprintf(g_last_error, sizeof g_last_error, "%s: %s", what, detail ? detail : "");
+  return code;
+}
+
+int fail_cuda(const char* what, cudaError_t e) {
+  return fail(SC_ERR_CUDA, what, cudaGetErrorString(e));
+}
+
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
-  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, total;
+  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident, qkv, total;
 };
 
 bool ws_layout(int B, int L, int H, WsLayout* w) {
@@ -52,6 +66,9 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->cnt_seq = take(sizeof(uint32_t) * B);
   w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
   w->ng = take(sizeof(int32_t) * 2 * B);
+  w->ident = take(sizeof(int32_t) * 2 * B);
+  // compacted Q, K, V of the current layer (rows of the surviving tokens)
+  w->qkv = take(sizeof(uint16_t) * 3 * B * (size_t)L * H * kHeadDim);
   w->total = off;
   return true;
 }
@@ -72,28 +89,73 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encoder() {
   return fn;
 }
 
-// 2-D view [rows][64] of a bf16 tensor whose rows are (.., token, head); one
-// TMA box is a single 128-byte row, gathered four at a time.
+// Tile view: 3-D [tokens][H][64] of a bf16 tensor laid out (.., token, head,
+// 64); one TMA box is 128 consecutive tokens of one head (16 KB).
+bool encode_tiles(CUtensorMap* m, const void* base, long long tokens, int H) {
+  auto enc = get_encoder();
+  if (!enc) return fail(SC_ERR_CUDA, "tensor-map encoder", "cuTensorMapEncodeTiled unavailable"), false;
+  cuuint64_t gdim[3] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(H),
+                        static_cast<cuuint64_t>(tokens)};
+  cuuint64_t gstride[2] = {static_cast<cuuint64_t>(kHeadDim * 2),
+                           static_cast<cuuint64_t>(kHeadDim * 2) * H};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(kHeadDim), 1, static_cast<cuuint32_t>(kTile)};
+  cuuint32_t estride[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), gdim, gstride,
+                   box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char d[64];
+    snprintf(d, sizeof d, "CUresult %d", static_cast<int>(r));
+    fail(SC_ERR_CUDA, "encode 3-D tile map", d);
+  }
+  return r == CUDA_SUCCESS;
+}
+
+// Row view: 2-D [tokens * H][64]; one TMA box is a single 128-byte row,
+// gathered four at a time (the global tokens).
 bool encode_rows(CUtensorMap* m, const void* base, long long rows) {
   auto enc = get_encoder();
-  if (!enc) return false;
+  if (!enc) return fail(SC_ERR_CUDA, "tensor-map encoder", "cuTensorMapEncodeTiled unavailable"), false;
   cuuint64_t gdim[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
   cuuint64_t gstride[1] = {static_cast<cuuint64_t>(kHeadDim * 2)};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kHeadDim), 1};
   cuuint32_t estride[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride, box,
-             estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride,
+                   box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char d[64];
+    snprintf(d, sizeof d, "CUresult %d", static_cast<int>(r));
+    fail(SC_ERR_CUDA, "encode 2-D row map", d);
+  }
+  return r == CUDA_SUCCESS;
+}
+
+// Descriptors for the caller's Q, K, V (source 0, `tokens` tokens) and the
+// compacted copies in the workspace (source 1, B * L tokens).
+bool encode_maps(TensorMaps* m, const uint16_t* const src[3], long long tokens, uint16_t* const cmp[3],
+                 long long cmp_tokens, int H) {
+  for (int t = 0; t < 3; ++t) {
+    if (!encode_tiles(&m->tile[0][t], src[t], tokens, H) ||
+        !encode_rows(&m->row[0][t], src[t], tokens * H) ||
+        !encode_tiles(&m->tile[1][t], cmp[t], cmp_tokens, H) ||
+        !encode_rows(&m->row[1][t], cmp[t], cmp_tokens * H))
+      return false;
+  }
+  return true;
 }
 
 int ensure_configured() {
   static std::mutex mu;
   static bool done[256] = {false};
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return SC_ERR_CUDA;
+  const cudaError_t ge = cudaGetDevice(&dev);
+  if (ge != cudaSuccess) return fail_cuda("cudaGetDevice", ge);
+  if (dev < 0 || dev >= 256) return fail(SC_ERR_CUDA, "cudaGetDevice", "device index out of range");
   std::lock_guard<std::mutex> lock(mu);
   if (!done[dev]) {
-    if (configure_kernels() != cudaSuccess) return SC_ERR_CUDA;
+    const cudaError_t e = configure_kernels();
+    if (e != cudaSuccess) return fail_cuda("kernel attributes", e);
     done[dev] = true;
   }
   return SC_OK;
@@ -126,17 +188,26 @@ void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->cnt_seq = reinterpret_cast<uint32_t*>(ws + lay.cnt_seq);
   int32_t* gcur = reinterpret_cast<int32_t*>(ws + lay.gcur);
   int32_t* ng = reinterpret_cast<int32_t*>(ws + lay.ng);
+  int32_t* ident = reinterpret_cast<int32_t*>(ws + lay.ident);
   p->gcur = gcur + slot * p->B * kMaxGlobal;
   p->gcur_out = gcur + (1 - slot) * p->B * kMaxGlobal;
   p->ng = ng + slot * p->B;
   p->ng_out = ng + (1 - slot) * p->B;
+  p->ident = ident + slot * p->B;
+  p->ident_out = ident + (1 - slot) * p->B;
+}
+
+void compacted_qkv(char* ws, const WsLayout& lay, int B, int L, int H, uint16_t* out[3]) {
+  const size_t per = static_cast<size_t>(B) * L * H * kHeadDim;
+  uint16_t* base = reinterpret_cast<uint16_t*>(ws + lay.qkv);
+  for (int t = 0; t < 3; ++t) out[t] = base + t * per;
 }
 
 int reset_counters(char* ws, const WsLayout& lay, cudaStream_t st) {
   // the counters reset themselves after each layer; clearing them per call
   // keeps a call independent of any earlier call that was cut short
-  if (cudaMemsetAsync(ws + lay.cnt_tile, 0, lay.gcur - lay.cnt_tile, st) != cudaSuccess)
-    return SC_ERR_CUDA;
+  const cudaError_t e = cudaMemsetAsync(ws + lay.cnt_tile, 0, lay.gcur - lay.cnt_tile, st);
+  if (e != cudaSuccess) return fail_cuda("counter reset", e);
   return SC_OK;
 }
 
@@ -149,6 +220,8 @@ size_t sc_workspace_size(int B, int L, int H) {
   if (!ws_layout(B, L, H, &lay)) return 0;
   return lay.total;
 }
+
+const char* sc_last_error(void) { return g_last_error; }
 
 const char* sc_status_string(int status) {
   switch (status) {
@@ -180,18 +253,18 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
 
-  const long long rows = static_cast<long long>(a->B) * a->L * a->H;
-  CUtensorMap mq, mk, mv;
-  if (!encode_rows(&mq, a->Q, rows) || !encode_rows(&mk, a->K, rows) ||
-      !encode_rows(&mv, a->V, rows))
-    return SC_ERR_CUDA;
+  TensorMaps maps;
+  uint16_t* cmp[3];
+  compacted_qkv(ws, lay, a->B, a->L, a->H, cmp);
+  const uint16_t* src[3] = {a->Q, a->K, a->V};
+  const long long tokens = static_cast<long long>(a->B) * a->L;
+  if (!encode_maps(&maps, src, tokens, cmp, tokens, a->H)) return SC_ERR_CUDA;
   if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
 
   LayerParams p{};
   p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
   p.T = (a->L + kTile - 1) / kTile;
-  p.gather = 0;
-  p.row_base = 0;
+  p.src_base = 0;
   p.len = a->len;
   p.pos = a->pos;
   p.O = a->O;
@@ -208,14 +281,18 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   pp.len_in = a->len;
   pp.gcur = const_cast<int32_t*>(p.gcur);
   pp.ng = const_cast<int32_t*>(p.ng);
+  pp.ident = const_cast<int32_t*>(p.ident);
   pp.n_global = a->n_global;
   for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
-  if (launch_prep(pp, st) != cudaSuccess) return SC_ERR_CUDA;
-  if (launch_layer(mq, mk, mv, p, st) != cudaSuccess) return SC_ERR_CUDA;
+  cudaError_t e;
+  if ((e = launch_prep(pp, st)) != cudaSuccess) return fail_cuda("launch prep kernel", e);
+  if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
+  if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
   return SC_OK;
 }
 
-int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
+static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
+                              void* stream, void** events, int n_events) {
   if (!a) return SC_ERR_INVALID_ARG;
   if (a->n_layers < 1) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
@@ -234,17 +311,18 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
 
-  CUtensorMap mq, mk, mv;
-  if (!encode_rows(&mq, a->Q, rows) || !encode_rows(&mk, a->K, rows) ||
-      !encode_rows(&mv, a->V, rows))
-    return SC_ERR_CUDA;
+  TensorMaps maps;
+  uint16_t* cmp[3];
+  compacted_qkv(ws, lay, a->B, a->L, a->H, cmp);
+  const uint16_t* src[3] = {a->Q, a->K, a->V};
+  const long long BLt = static_cast<long long>(a->B) * a->L;
+  if (!encode_maps(&maps, src, a->n_layers * BLt, cmp, BLt, a->H)) return SC_ERR_CUDA;
   if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
 
   const size_t BL = static_cast<size_t>(a->B) * a->L;
   LayerParams p{};
   p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
   p.T = (a->L + kTile - 1) / kTile;
-  p.gather = 1;
   p.theta = nullptr;
   fill_workspace(&p, ws, lay, 0);
 
@@ -255,13 +333,28 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
   pp.len_out = a->len;
   pp.gcur = const_cast<int32_t*>(p.gcur);
   pp.ng = const_cast<int32_t*>(p.ng);
+  pp.ident = const_cast<int32_t*>(p.ident);
   pp.n_global = a->n_global;
   for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
-  if (launch_prep(pp, st) != cudaSuccess) return SC_ERR_CUDA;
-
+  auto mark = [&](int k) {
+    return events == nullptr ||
+           cudaEventRecord(static_cast<cudaEvent_t>(events[k]), st) == cudaSuccess;
+  };
+  cudaError_t e;
+  if (!mark(0)) return fail(SC_ERR_CUDA, "event record", "");
+  if ((e = launch_prep(pp, st)) != cudaSuccess) return fail_cuda("launch prep kernel", e);
+  if (!mark(1)) return fail(SC_ERR_CUDA, "event record", "");
+  // layer 0 reads the caller's rows in place when no padding was removed; the
+  // gather kernel copies the survivors' rows for every later layer
+  GatherParams gp{};
+  gp.B = a->B; gp.L = a->L; gp.H = a->H;
+  for (int t = 0; t < 3; ++t) {
+    gp.src[t] = src[t];
+    gp.dst[t] = cmp[t];
+  }
   for (int l = 0; l < a->n_layers; ++l) {
     fill_workspace(&p, ws, lay, l & 1);
-    p.row_base = static_cast<long long>(l) * a->B * a->L * a->H;
+    p.src_base = static_cast<long long>(l) * BLt;
     p.len = a->len + static_cast<size_t>(l) * a->B;
     p.len_out = a->len + static_cast<size_t>(l + 1) * a->B;
     p.pos = a->pos + static_cast<size_t>(l) * BL;
@@ -269,9 +362,40 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
     p.O = a->O + static_cast<size_t>(l) * BL * a->H * kHeadDim;
     p.scores = a->scores + static_cast<size_t>(l) * BL;
     p.alpha = a->alpha[l];
-    if (launch_layer(mq, mk, mv, p, st) != cudaSuccess) return SC_ERR_CUDA;
+    if (l == 0 && a->pad_mask != nullptr) {
+      // padding removal may have moved rows: compact layer 0 as well
+      gp.src_base = 0;
+      gp.len = p.len;
+      gp.pos = p.pos;
+      gp.ident = p.ident;
+      if ((e = launch_gather(gp, st)) != cudaSuccess) return fail_cuda("launch gather kernel", e);
+    }
+    if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
+    if (!mark(2 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");
+    if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
+    if (!mark(3 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");
+    if (l + 1 < a->n_layers) {
+      gp.src_base = static_cast<long long>(l + 1) * BLt;
+      gp.len = p.len_out;
+      gp.pos = p.pos_out;
+      gp.ident = p.ident_out;
+      if ((e = launch_gather(gp, st)) != cudaSuccess) return fail_cuda("launch gather kernel", e);
+    }
+    if (!mark(4 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");
   }
   return SC_OK;
+}
+
+int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
+  return stack_forward_impl(a, workspace, ws_bytes, stream, nullptr, 0);
+}
+
+int sc_stack_forward_profiled(const sc_stack_args* a, void* workspace, size_t ws_bytes,
+                              void* stream, void** events, int n_events) {
+  if (!a || !events || a->n_layers < 1 || n_events < 2 + 3 * a->n_layers) return SC_ERR_INVALID_ARG;
+  for (int k = 0; k < 2 + 3 * a->n_layers; ++k)
+    if (!events[k]) return SC_ERR_INVALID_ARG;
+  return stack_forward_impl(a, workspace, ws_bytes, stream, events, n_events);
 }
 
 int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {

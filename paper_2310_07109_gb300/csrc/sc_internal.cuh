@@ -23,11 +23,23 @@ constexpr int kStatusTimeout = 1;
 // log2(e) / sqrt(64): logits are kept in base-2 units, x = (q.k) * kLogitScale2.
 constexpr float kLogitScale2 = 0.125f * 1.4426950408889634f;
 
+// TMA descriptors of Q, K, V (index 0, 1, 2) for both row sources: [0] the
+// caller's tensors, [1] the compacted copies.  tile: 3-D [tokens][H][64] with a
+// 128-token x 1-head box; row: 2-D [tokens*H][64] with a one-row box (gather4).
+struct TensorMaps {
+  CUtensorMap tile[2][3];
+  CUtensorMap row[2][3];
+};
+
 struct LayerParams {
   int B, L, H, w;
   int T;                 // tiles per padded sequence = ceil(L / 128)
-  int gather;            // 1: row of current token c is at original position pos[b][c]
-  long long row_base;    // first tensor-map row of this layer's [B][L][H] block
+  // Where the current rows of sequence b live: when ident[b] != 0 (the current
+  // tokens are original positions 0..n-1) row c is token (src_base + b*L + c)
+  // of the "source" tensors; otherwise it is token (b*L + c) of the compacted
+  // copies written by the gather kernel.
+  long long src_base;    // token offset of this layer's [B][L] block in the source tensors
+  const int32_t* ident;  // [B]
   const int32_t* len;    // [B] current lengths
   const int32_t* pos;    // [B][L] original positions of current tokens
   const int32_t* gcur;   // [B][kMaxGlobal] current indices of global tokens (increasing)
@@ -38,6 +50,7 @@ struct LayerParams {
   int32_t* len_out;      // [B] out
   int32_t* gcur_out;     // [B][kMaxGlobal] out (next layer)
   int32_t* ng_out;       // [B] out
+  int32_t* ident_out;    // [B] out (next layer)
   float alpha;           // theta_b = alpha / n_b unless theta != nullptr
   const float* theta;    // [B] absolute thresholds or nullptr
   // workspace
@@ -52,6 +65,18 @@ struct LayerParams {
   int* status;
 };
 
+// Copies the rows of the kept tokens (at their original positions) of one
+// layer's Q, K, V into compacted [B][L][H][64] buffers.
+struct GatherParams {
+  int B, L, H;
+  long long src_base;          // token offset of the layer's [B][L] block in the sources
+  const int32_t* len;          // [B]
+  const int32_t* pos;          // [B][L]
+  const int32_t* ident;        // [B]: sequences whose rows need no copy
+  const uint16_t* src[3];      // Q, K, V sources [.., B, L, H, 64]
+  uint16_t* dst[3];            // compacted Q, K, V [B][L][H][64]
+};
+
 struct PrepParams {
   int B, L;
   const uint8_t* pad_mask;   // [B][L] or nullptr (stack mode)
@@ -61,6 +86,7 @@ struct PrepParams {
   int32_t* len_out;          // [B] (stack mode)
   int32_t* gcur;             // [B][kMaxGlobal]
   int32_t* ng;               // [B]
+  int32_t* ident;            // [B]
   int n_global;
   int global_pos[kMaxGlobal];
 };

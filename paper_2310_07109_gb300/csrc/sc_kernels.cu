@@ -65,42 +65,38 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 
-// Tensor-map row of (sequence b, row src of that sequence, head h).
-__device__ __forceinline__ int tmap_row(const LayerParams& p, int b, int src, int h) {
-  return static_cast<int>(p.row_base + (static_cast<long long>(b) * p.L + src) * p.H + h);
+// Which source holds the current rows of sequence b, and the token index of
+// its current row 0 in that source.
+struct RowSource {
+  int s;
+  long long tok_b;
+};
+
+__device__ __forceinline__ RowSource row_source(const LayerParams& p, int b) {
+  const bool id = __ldg(p.ident + b) != 0;
+  return {id ? 0 : 1, (id ? p.src_base : 0) + static_cast<long long>(b) * p.L};
 }
 
-__device__ __forceinline__ int src_row(const LayerParams& p, int b, int c) {
-  return p.gather ? __ldg(p.pos + static_cast<size_t>(b) * p.L + c) : c;
+// One 128-token tile (current rows c0 .. c0+127) of tensor t (0 Q, 1 K, 2 V)
+// for head h: a single TMA copy.  Rows past the sequence are read but masked.
+__device__ __forceinline__ void load_tile(const TensorMaps& m, int t, const RowSource& rs, int h,
+                                          int c0, uint8_t* dst, uint64_t* bar) {
+  tma_load_3d(dst, &m.tile[rs.s][t], 0, h, static_cast<int>(rs.tok_b + c0), bar);
 }
 
-// The load warp gathers a 128-row tile (rows first_c .. first_c+127 of the
-// current sequence, clamped to n-1) of one tensor into `dst`; each lane moves
-// four rows with one gather4.
-__device__ __forceinline__ void load_tile(const LayerParams& p, const CUtensorMap* map,
-                                          uint8_t* dst, int b, int h, int first_c, int n,
-                                          uint64_t* bar, int lane) {
-  int r[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    int c = min(first_c + 4 * lane + k, n - 1);
-    r[k] = tmap_row(p, b, src_row(p, b, c), h);
-  }
-  tma_gather4(dst + 512 * lane, map, 0, r[0], r[1], r[2], r[3], bar);
-}
-
-// The 16 global rows (current indices gc[0..ng-1], the last repeated).
-__device__ __forceinline__ void load_globals(const LayerParams& p, const CUtensorMap* map,
-                                             uint8_t* dst, int b, int h, const int* gc, int ng,
+// The 16 global rows (current indices gc[0..ng-1], the last repeated): lanes
+// 0..3 gather four rows each.
+__device__ __forceinline__ void load_globals(const TensorMaps& m, int t, const RowSource& rs, int h,
+                                             int H, const int* gc, int ng, uint8_t* dst,
                                              uint64_t* bar, int lane) {
   if (lane < 4) {
     int r[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      int g = min(4 * lane + k, ng - 1);
-      r[k] = tmap_row(p, b, src_row(p, b, gc[g]), h);
+      const int g = min(4 * lane + k, ng - 1);
+      r[k] = static_cast<int>((rs.tok_b + gc[g]) * H + h);
     }
-    tma_gather4(dst + 512 * lane, map, 0, r[0], r[1], r[2], r[3], bar);
+    tma_gather4(dst + 512 * lane, &m.row[rs.s][t], 0, r[0], r[1], r[2], r[3], bar);
   }
 }
 
@@ -137,15 +133,17 @@ struct RowsSmem {
   int gc[kMaxGlobal];
   float red[4][kMaxGlobal];
   float red2[4][kMaxGlobal];
+  float red3[4][kMaxGlobal];
 };
 
 constexpr uint32_t kRowsDyn = kTileBytes * (1 + 2 * kMaxBandTiles) + 2 * kTileBytes +
                               3 * kGTileBytes + 1024;
 
 __global__ void __launch_bounds__(kThreads, 1)
-    sc_rows_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                   const __grid_constant__ CUtensorMap mapV, const LayerParams p) {
-  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    sc_rows_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
+  // grid: x = (sequence, head), y = query tile, so that low tiles (the ones
+  // every sequence has) are dispatched first
+  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, qt = blockIdx.y;
   const int n = __ldg(p.len + b);
   if (qt * kTile >= n) return;
   const int ng = min(__ldg(p.ng + b), kMaxGlobal);
@@ -194,23 +192,26 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 4) {
     // ------------------------------------------------------------- loads
-    if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[0], kTileBytes + 3 * ngp * 128);
+    const RowSource rs = row_source(p, b);
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&sm.bar_load[0], kTileBytes + 3 * ngp * 128);
+      load_tile(maps, 0, rs, h, r0, Qs, &sm.bar_load[0]);
+    }
     __syncwarp();
-    load_tile(p, &mapQ, Qs, b, h, r0, n, &sm.bar_load[0], lane);
     if (ngp) {
-      load_globals(p, &mapK, KG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
-      load_globals(p, &mapV, VG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
-      load_globals(p, &mapQ, QG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
+      load_globals(maps, 1, rs, h, p.H, sm.gc, ng, KG, &sm.bar_load[0], lane);
+      load_globals(maps, 2, rs, h, p.H, sm.gc, ng, VG, &sm.bar_load[0], lane);
+      load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_load[0], lane);
     }
-    for (int i = 0; i < nb; ++i) {
-      if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[1 + i], 2 * kTileBytes);
-      __syncwarp();
-      const int c0 = (kt_lo + i) * kTile;
-      load_tile(p, &mapK, Ks + i * kTileBytes, b, h, c0, n, &sm.bar_load[1 + i], lane);
-      load_tile(p, &mapV, Vs + i * kTileBytes, b, h, c0, n, &sm.bar_load[1 + i], lane);
-    }
-    if (lane == 0)
+    if (lane == 0) {
+      // key tiles in the order the MMA consumes them
+      for (int i = 0; i < nb; ++i) {
+        mbar_arrive_expect_tx(&sm.bar_load[1 + i], 2 * kTileBytes);
+        load_tile(maps, 1, rs, h, (kt_lo + i) * kTile, Ks + i * kTileBytes, &sm.bar_load[1 + i]);
+        load_tile(maps, 2, rs, h, (kt_lo + i) * kTile, Vs + i * kTileBytes, &sm.bar_load[1 + i]);
+      }
       for (int i = 0; i <= nb; ++i) drain_wait(&sm.bar_load[i], 0);
+    }
   } else if (warp == 5) {
     // ------------------------------------------------------------- MMA issue
     if (lane == 0) {
@@ -273,9 +274,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool row_global = false;
     for (int g = 0; g < ng; ++g) row_global |= (sm.gc[g] == i);
     const bool valid = (i < n) && !row_global;
-    // allowed band keys of this row (current index), inclusive
-    const int lo = valid ? max(0, i - p.w) : 0;
-    const int hi = valid ? min(n - 1, i + p.w) : n - 1;
+    // allowed band keys of this row, inclusive (current index); the same band
+    // is used for rows whose results are discarded (global rows, rows >= n)
+    const int lo = max(0, i - p.w);
+    const int hi = min(n - 1, i + p.w);
+    // union of the band over this warp's 32 rows: chunks outside it are skipped
+    const int wlo = max(0, r0 + 32 * warp - p.w);
+    const int whi = min(n - 1, r0 + 32 * warp + 31 + p.w);
 
     float m_ref = -INFINITY, lsum = 0.f;
     int p_use = 0;
@@ -293,16 +298,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; ++g) {
           const int cg = sm.gc[g];
-          const bool use = (g < ng) && (!valid || abs(i - cg) > p.w);
-          x[g] = use ? x[g] * kLogitScale2 : -INFINITY;
+          const bool use = (g < ng) && abs(i - cg) > p.w;
+          x[g] = use ? x[g] : -INFINITY;
           mx = fmaxf(mx, x[g]);
         }
-        m_ref = mx;
+        m_ref = mx * kLogitScale2;
         const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
         uint32_t pk[8];
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; g += 2) {
-          const float a = ex2(x[g] - ref), c = ex2(x[g + 1] - ref);
+          const float a = ex2(fmaf(x[g], kLogitScale2, -ref));
+          const float c = ex2(fmaf(x[g + 1], kLogitScale2, -ref));
           lsum += a + c;
           pk[g / 2] = pack_bf16x2(a, c);
         }
@@ -318,28 +324,36 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     for (int t = 0; ok && t < nb; ++t) {
       const int j0 = (kt_lo + t) * kTile;
+      // 32-column chunks of this tile that intersect the warp's band
+      const int clo = max(0, wlo - j0), chi = min(kTile - 1, whi - j0);
+      const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
       if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
       tc_fence_after();
       const uint32_t ts = (t & 1) ? tS1 : tS0;
 #pragma unroll
-      for (int c = 0; c < 128; c += 32) tmem_ld32(ts + lane_off + c, x + c);
+      for (int ch = 0; ch < 4; ++ch)
+        if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(ts + lane_off + 32 * ch, x + 32 * ch);
       tmem_ld_wait();
-      const bool full = (lo <= j0) && (j0 + kTile - 1 <= hi);
-      float mx = -INFINITY;
-      if (__all_sync(0xffffffffu, full)) {
+      const int a = lo - j0, e = hi - j0;
+      // eight independent partial maxima: no long dependency chain
+      float pm[8];
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          x[c] *= kLogitScale2;
-          mx = fmaxf(mx, x[c]);
-        }
-      } else {
-        const int a = lo - j0, e = hi - j0;
+      for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          x[c] = (c >= a && c <= e) ? x[c] * kLogitScale2 : -INFINITY;
-          mx = fmaxf(mx, x[c]);
+      for (int ch = 0; ch < 4; ++ch) {
+        if (ch < ch_lo || ch > ch_hi) continue;
+        if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const int c = 32 * ch + k;
+            x[c] = (c >= a && c <= e) ? x[c] : -INFINITY;
+          }
         }
+#pragma unroll
+        for (int k = 0; k < 32; ++k) pm[k & 7] = fmaxf(pm[k & 7], x[32 * ch + k]);
       }
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * kLogitScale2;
       // lazy rescale: move the reference only when the tile max exceeds it by > 8 (2^8)
       float scale = 1.f;
       const bool bump = mx > m_ref + 8.f;
@@ -348,17 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         new_ref = mx;
         scale = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - new_ref);
       }
-      const float ref = (new_ref == -INFINITY) ? 0.f : new_ref;
-      float ts_sum = 0.f;
-      uint32_t pk[64];
-#pragma unroll
-      for (int c = 0; c < 128; c += 2) {
-        const float a = ex2(x[c] - ref), d = ex2(x[c + 1] - ref);
-        ts_sum += a + d;
-        pk[c / 2] = pack_bf16x2(a, d);
-      }
-      lsum = lsum * scale + ts_sum;
-      m_ref = new_ref;
+      const float nref = (new_ref == -INFINITY) ? 0.f : -new_ref;
       // the previous P V must be done before P is overwritten or O rescaled
       if (p_use > 0) {
         if (!(ok = warp_wait(&sm.bar_pv, (p_use - 1) & 1, abort_flag))) break;
@@ -377,10 +381,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st_wait();
       }
+      // P = exp2(x - ref) in bf16, written chunk by chunk into the swizzled A tile;
+      // the row sum is kept in eight independent partial sums
+      float ps[8];
 #pragma unroll
-      for (int c = 0; c < 16; ++c)
-        *reinterpret_cast<uint4*>(Ps + (c >> 3) * 16384 + sw128_offset(r, c & 7)) =
-            make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) {
+        uint8_t* prow = Ps + (ch >> 1) * 16384;
+        if (ch >= ch_lo && ch <= ch_hi) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t w4[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int c = 32 * ch + 8 * q + 2 * k;
+              const float u = ex2(fmaf(x[c], kLogitScale2, nref));
+              const float v = ex2(fmaf(x[c + 1], kLogitScale2, nref));
+              ps[2 * k] += u;
+              ps[2 * k + 1] += v;
+              w4[k] = pack_bf16x2(u, v);
+            }
+            *reinterpret_cast<uint4*>(prow + sw128_offset(r, (ch & 1) * 4 + q)) =
+                make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(prow + sw128_offset(r, (ch & 1) * 4 + q)) =
+                make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+      const float ts_sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      lsum = lsum * scale + ts_sum;
+      m_ref = new_ref;
       fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(&sm.bar_p);
@@ -425,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int g = 0; g < kMaxGlobal; ++g) {
         const int cg = sm.gc[g];
         const bool use = ok && valid && (g < ng) && abs(i - cg) > p.w;
-        part[g] = use ? ex2(x[g] * kLogitScale2 - lse) : 0.f;
+        part[g] = use ? ex2(fmaf(x[g], kLogitScale2, -lse)) : 0.f;
         part[g] = warp_sum(part[g]);
       }
       if (lane == 0)
@@ -446,23 +480,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0)
         for (int g = 0; g < kMaxGlobal; ++g) sm.red2[warp][g] = part[g];
       named_sync_softmax();
-      float gm[kMaxGlobal];
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        gm[g] = fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
-        const float e = (key_ok && gm[g] != -INFINITY) ? ex2(x[g] - gm[g]) : 0.f;
+        const float gm =
+            fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
+        const float e = (key_ok && gm != -INFINITY) ? ex2(x[g] - gm) : 0.f;
         part[g] = warp_sum(e);
       }
-      named_sync_softmax();
       if (lane == 0)
-        for (int g = 0; g < kMaxGlobal; ++g) sm.red2[warp][g] = part[g];
+        for (int g = 0; g < kMaxGlobal; ++g) sm.red3[warp][g] = part[g];
       named_sync_softmax();
       if (tid < kMaxGlobal) {
         const int g = tid;
         const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + g;
         p.gpart[slot] = sm.red[0][g] + sm.red[1][g] + sm.red[2][g] + sm.red[3][g];
-        p.gstat[2 * slot] = gm[g];
-        p.gstat[2 * slot + 1] = sm.red2[0][g] + sm.red2[1][g] + sm.red2[2][g] + sm.red2[3][g];
+        p.gstat[2 * slot] =
+            fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
+        p.gstat[2 * slot + 1] = sm.red3[0][g] + sm.red3[1][g] + sm.red3[2][g] + sm.red3[3][g];
       }
       if (qt == 0) {
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
@@ -491,7 +525,8 @@ struct ColsSmem {
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  float lse[kMaxBandTiles * kTile];
+  alignas(16) float lse[kMaxBandTiles * kTile];  // read as float4
+  float gsum[kMaxGlobal];
   int flag;
   int scan[kThreads];
   int gnew[kMaxGlobal];
@@ -502,14 +537,14 @@ constexpr uint32_t kColsDyn = kTileBytes * (2 + kMaxBandTiles) + kGTileBytes + 2
 __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm);
 
 __global__ void __launch_bounds__(kThreads, 1)
-    sc_cols_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                   const __grid_constant__ CUtensorMap mapV, const LayerParams p) {
-  const int kt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    sc_cols_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
+  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, kt = blockIdx.y;
   const int n = __ldg(p.len + b);
   if (n == 0) {
     if (kt == 0 && h == 0 && threadIdx.x == 0) {
       p.len_out[b] = 0;
       p.ng_out[b] = 0;
+      p.ident_out[b] = 1;
     }
     return;
   }
@@ -558,19 +593,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = &sm.abort;
 
   if (warp == 4) {
-    if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[0], 2 * kTileBytes + ngp * 128);
-    __syncwarp();
-    load_tile(p, &mapK, Ks, b, h, j0, n, &sm.bar_load[0], lane);
-    load_tile(p, &mapV, Vs, b, h, j0, n, &sm.bar_load[0], lane);
-    if (ngp) load_globals(p, &mapQ, QG, b, h, sm.gc, ng, &sm.bar_load[0], lane);
-    for (int i = 0; i < nq; ++i) {
-      if (lane == 0) mbar_arrive_expect_tx(&sm.bar_load[1 + i], kTileBytes);
-      __syncwarp();
-      load_tile(p, &mapQ, Qs + i * kTileBytes, b, h, (qt_lo + i) * kTile, n,
-                &sm.bar_load[1 + i], lane);
+    const RowSource rs = row_source(p, b);
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&sm.bar_load[0], 2 * kTileBytes + ngp * 128);
+      load_tile(maps, 1, rs, h, j0, Ks, &sm.bar_load[0]);
+      load_tile(maps, 2, rs, h, j0, Vs, &sm.bar_load[0]);
     }
-    if (lane == 0)
+    __syncwarp();
+    if (ngp) load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_load[0], lane);
+    if (lane == 0) {
+      for (int i = 0; i < nq; ++i) {
+        mbar_arrive_expect_tx(&sm.bar_load[1 + i], kTileBytes);
+        load_tile(maps, 0, rs, h, (qt_lo + i) * kTile, Qs + i * kTileBytes, &sm.bar_load[1 + i]);
+      }
       for (int i = 0; i <= nq; ++i) drain_wait(&sm.bar_load[i], 0);
+    }
   } else if (warp == 5) {
     if (lane == 0) {
       const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs);
@@ -615,49 +652,80 @@ __global__ void __launch_bounds__(kThreads, 1)
       sm.lse[k] = row < n ? __ldcg(lse_src + row) : INFINITY;
     }
     if (ngp && warp == 0) {
-      // merge the per-tile (max, sum) of every global row into its LSE
-      for (int g = 0; g < ng; ++g) {
-        float m = -INFINITY, s = 0.f;
-        if (lane < Tn) {
-          const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + lane) * kMaxGlobal + g;
-          m = __ldcg(p.gstat + 2 * slot);
-          s = __ldcg(p.gstat + 2 * slot + 1);
-        }
-        const float M = warp_max(m);
-        const float part = (lane < Tn && m != -INFINITY) ? s * ex2(m - M) : 0.f;
+      // merge the per-tile (max, sum) of every global row into its LSE; lane = key tile,
+      // all loads issued before any reduction
+      float m[kMaxGlobal], sm_[kMaxGlobal];
+      const size_t base_slot = ((static_cast<size_t>(b) * p.H + h) * p.T + lane) * kMaxGlobal;
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        const bool use = lane < Tn && g < ng;
+        m[g] = use ? __ldcg(p.gstat + 2 * (base_slot + g)) : -INFINITY;
+        sm_[g] = use ? __ldcg(p.gstat + 2 * (base_slot + g) + 1) : 0.f;
+      }
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        const float M = warp_max(m[g]);
+        const float part = (m[g] != -INFINITY) ? sm_[g] * ex2(m[g] - M) : 0.f;
         const float S = warp_sum(part);
-        if (lane == 0) sm.lse_g[g] = M + lg2(S);
+        if (lane == 0 && g < ng) sm.lse_g[g] = M + lg2(S);
       }
     }
     named_sync_softmax();
 
+    // union of the band over this warp's 32 key columns
+    const int wlo = max(0, j0 + 32 * warp - p.w);
+    const int whi = min(n - 1, j0 + 32 * warp + 31 + p.w);
     float acc = 0.f;
     bool ok = true;
     float x[128];
     for (int t = 0; ok && t < nq; ++t) {
+      const int i0 = (qt_lo + t) * kTile;            // first query row of this tile
+      const int clo = max(0, wlo - i0), chi = min(kTile - 1, whi - i0);
+      const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
       if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
       tc_fence_after();
       const uint32_t ts = (t & 1) ? tS1 : tS0;
 #pragma unroll
-      for (int c = 0; c < 128; c += 32) tmem_ld32(ts + lane_off + c, x + c);
+      for (int ch = 0; ch < 4; ++ch)
+        if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(ts + lane_off + 32 * ch, x + 32 * ch);
       tmem_ld_wait();
       tc_fence_before();
       mbar_arrive(&sm.bar_sfree[t & 1]);
-      const int i0 = (qt_lo + t) * kTile;            // first query row of this tile
       const float* lw = sm.lse + t * kTile;
       const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
-      float s = 0.f;
-      if (__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
+      // eight independent partial sums per tile
+      float ps[8];
 #pragma unroll
-        for (int c = 0; c < 128; ++c) s += ex2(x[c] * kLogitScale2 - lw[c]);
-      } else {
+      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          const float v = ex2(x[c] * kLogitScale2 - lw[c]);
-          s += (c >= a && c <= e) ? v : 0.f;
+      for (int ch = 0; ch < 4; ++ch) {
+        if (ch < ch_lo || ch > ch_hi) continue;
+        if (__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
+            const int u = (k >> 2) & 1;
+            ps[4 * u] += ex2(fmaf(x[32 * ch + k], kLogitScale2, -l4.x));
+            ps[4 * u + 1] += ex2(fmaf(x[32 * ch + k + 1], kLogitScale2, -l4.y));
+            ps[4 * u + 2] += ex2(fmaf(x[32 * ch + k + 2], kLogitScale2, -l4.z));
+            ps[4 * u + 3] += ex2(fmaf(x[32 * ch + k + 3], kLogitScale2, -l4.w));
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; k += 4) {
+            const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
+            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
+            const int u = (k >> 2) & 1;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int c = 32 * ch + k + q;
+              const float v = ex2(fmaf(x[c], kLogitScale2, -lv[q]));
+              ps[4 * u + q] += (c >= a && c <= e) ? v : 0.f;
+            }
+          }
         }
       }
-      acc += s;
+      acc += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
     }
 
     if (ngp) {
@@ -671,7 +739,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float s = 0.f;
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const float v = (ok2 && g < ng && j < n) ? ex2(x[g] * kLogitScale2 - sm.lse_g[g]) : 0.f;
+        const float v = (ok2 && g < ng && j < n) ? ex2(fmaf(x[g], kLogitScale2, -sm.lse_g[g])) : 0.f;
         s += v;
         pb[g] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
       }
@@ -717,16 +785,43 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (!sm.flag) return;
   __threadfence();
+  // far-row partial sums of the global keys that lie in this tile: one warp per
+  // global key, summed over heads and query tiles in a fixed order
+  if (warp < 4) {
+    for (int g = warp; g < ng; g += 4) {
+      const int cg = sm.gc[g];
+      float v = 0.f;
+      if (cg >= j0 && cg < j0 + kTile) {
+        const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * kMaxGlobal + g;
+#pragma unroll 4
+        for (int k = lane; k < p.H * Tn; k += 32) {
+          const int hh = k / Tn, q = k - hh * Tn;
+          v += __ldcg(gp + (static_cast<size_t>(hh) * p.T + q) * kMaxGlobal);
+        }
+        v = warp_sum(v);
+      }
+      if (lane == 0) sm.gsum[g] = v;
+    }
+  }
+  __syncthreads();
   if (tid < kTile && j0 + tid < n) {
     const int jj = j0 + tid;
+    const float* ap = p.acc + static_cast<size_t>(b) * p.H * p.L + jj;
     float a = 0.f;
-    for (int hh = 0; hh < p.H; ++hh) a += __ldcg(p.acc + (static_cast<size_t>(b) * p.H + hh) * p.L + jj);
-    for (int g = 0; g < ng; ++g) {
-      if (sm.gc[g] != jj) continue;
-      for (int hh = 0; hh < p.H; ++hh)
-        for (int q = 0; q < Tn; ++q)
-          a += __ldcg(p.gpart + ((static_cast<size_t>(b) * p.H + hh) * p.T + q) * kMaxGlobal + g);
+    int hh = 0;
+    for (; hh + 4 <= p.H; hh += 4) {
+      const float v0 = __ldcg(ap + static_cast<size_t>(hh) * p.L);
+      const float v1 = __ldcg(ap + static_cast<size_t>(hh + 1) * p.L);
+      const float v2 = __ldcg(ap + static_cast<size_t>(hh + 2) * p.L);
+      const float v3 = __ldcg(ap + static_cast<size_t>(hh + 3) * p.L);
+      a += v0;
+      a += v1;
+      a += v2;
+      a += v3;
     }
+    for (; hh < p.H; ++hh) a += __ldcg(ap + static_cast<size_t>(hh) * p.L);
+    for (int g = 0; g < ng; ++g)
+      if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
     p.scores[static_cast<size_t>(b) * p.L + jj] = s;
     const float theta = p.theta ? __ldg(p.theta + b) : p.alpha / static_cast<float>(n);
@@ -750,6 +845,7 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
   const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
   const uint8_t* keep = p.keep + static_cast<size_t>(b) * p.L;
   int cnt = 0;
+#pragma unroll 8
   for (int c = c0; c < c1; ++c) cnt += __ldcg(keep + c);
   sm.scan[tid] = cnt;
   __syncthreads();
@@ -775,6 +871,7 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
     ++out;
   }
   // bf16 outputs of the global rows
+#pragma unroll 4
   for (int k = tid; k < ng * p.H * kHeadDim; k += kThreads) {
     const int g = k / (p.H * kHeadDim), hh = (k / kHeadDim) % p.H, dd = k % kHeadDim;
     const float v = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
@@ -788,7 +885,40 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
       if (sm.gnew[g] >= 0) p.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
     p.ng_out[b] = m;
     p.len_out[b] = total;
+    // the survivors are original positions 0..total-1 exactly when the last one is total-1
+    p.ident_out[b] = (total == 0 || pos_out[total - 1] == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// gather kernel: the next layer's Q, K, V rows of the kept tokens, compacted
+// ---------------------------------------------------------------------------
+constexpr int kGatherTokens = 32;
+constexpr int kGatherThreads = 256;
+
+__global__ void __launch_bounds__(kGatherThreads)
+    sc_gather_kernel(const GatherParams g) {
+  const int b = blockIdx.y;
+  const int n = __ldg(g.len + b);
+  const int c0 = blockIdx.x * kGatherTokens;
+  if (__ldg(g.ident + b) != 0 || c0 >= n) return;
+  const int cnt = min(kGatherTokens, n - c0);
+  __shared__ long long src_tok[kGatherTokens];
+  if (threadIdx.x < cnt)
+    src_tok[threadIdx.x] =
+        g.src_base + static_cast<long long>(b) * g.L + __ldg(g.pos + static_cast<size_t>(b) * g.L + c0 + threadIdx.x);
+  __syncthreads();
+  const int vec = g.H * kHeadDim / 8;  // 16-byte vectors per token row
+  const long long dst_tok0 = static_cast<long long>(b) * g.L + c0;
+  for (int t = 0; t < 3; ++t) {
+    const uint4* src = reinterpret_cast<const uint4*>(g.src[t]);
+    uint4* dst = reinterpret_cast<uint4*>(g.dst[t]);
+#pragma unroll 4
+    for (int k = threadIdx.x; k < cnt * vec; k += kGatherThreads) {
+      const int tk = k / vec, v = k - tk * vec;
+      dst[(dst_tok0 + tk) * vec + v] = __ldg(src + src_tok[tk] * vec + v);
+    }
   }
 }
 
@@ -853,6 +983,8 @@ __global__ void __launch_bounds__(kPrepThreads)
       if (lo < n && spos[lo] == target) pp.gcur[b * kMaxGlobal + m++] = lo;
     }
     pp.ng[b] = m;
+    // single-layer calls read their (already current-order) inputs in place
+    pp.ident[b] = (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1) ? 1 : 0;
   }
 }
 
@@ -876,13 +1008,21 @@ cudaError_t configure_kernels() {
                               static_cast<int>(kColsDyn));
 }
 
-cudaError_t launch_layer(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv,
-                         const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.T, p.H, p.B);
-  sc_rows_kernel<<<grid, kThreads, kRowsDyn, st>>>(mq, mk, mv, p);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  sc_cols_kernel<<<grid, kThreads, kColsDyn, st>>>(mq, mk, mv, p);
+cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
+  dim3 grid(p.B * p.H, p.T);
+  sc_rows_kernel<<<grid, kThreads, kRowsDyn, st>>>(m, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
+  dim3 grid(p.B * p.H, p.T);
+  sc_cols_kernel<<<grid, kThreads, kColsDyn, st>>>(m, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {
+  dim3 grid((g.L + kGatherTokens - 1) / kGatherTokens, g.B);
+  sc_gather_kernel<<<grid, kGatherThreads, 0, st>>>(g);
   return cudaGetLastError();
 }
 

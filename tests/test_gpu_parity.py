@@ -131,3 +131,18 @@ def test_stack_huge_theta_keeps_only_first(sc):
     got = _run_stack(sc, wl, inp)
     assert (got["len"][1:] == 1).all()
     assert (got["pos"][1:, :, 0] == 0).all()
+
+
+def test_stack_scattered_padding_uses_compacted_rows(sc):
+    """Padding in the middle of sequences: every layer reads compacted rows."""
+    import oracle
+    wl = wk.Workload("holes", n_layers=3, B=2, L=400, w=64, n_extra_global=2,
+                     alpha_first=0.0, alpha_last=0.0, seed=8)
+    inp = wk.make_inputs(wl)
+    rng = np.random.default_rng(8)
+    mask = (rng.random((wl.B, wl.L)) < 0.8).astype(np.uint8)
+    mask[:, 0] = 1
+    mask[:, inp["global_pos"]] = 1
+    inp["pad_mask"] = mask
+    res = oracle.stack(inp["Q"], inp["K"], inp["V"], mask, inp["global_pos"], wl.w, inp["alpha"])
+    _check_stack(wl, res, _run_stack(sc, wl, inp))

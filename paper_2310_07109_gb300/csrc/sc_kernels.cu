@@ -3,23 +3,27 @@
 //
 // Per layer, per sequence b (n current tokens, original positions pos[b][*]):
 //
-//   rows kernel   (one CTA per (128-query-row tile, head, sequence))
-//     S = Q K^T over the band key tiles and one 16-wide tile of global keys,
-//     tensor cores (tcgen05, bf16 -> fp32 in tensor memory), operands gathered
-//     by TMA (gather4) straight from the original-position rows.  Row softmax
-//     in fp32 (base-2, lazily rescaled running max), P (bf16) V accumulated in
-//     tensor memory.  Writes O, the row log-sum-exp LSE_i, the far-row column
-//     sums of the global keys, and (max, sum) of the global rows over this
-//     tile's keys.
+//   rows kernel   (one CTA per (128-query-row tile, head, sequence); two CTAs
+//                 per SM)
+//     S = Q K^T over the band key tiles and one 16-wide tile of global keys on
+//     the tensor cores (tcgen05, bf16 -> fp32 in tensor memory); each 16 KB
+//     operand tile is one TMA copy.  Row softmax in fp32 (base 2, lazily
+//     rescaled running max); P (bf16) goes back to tensor memory and P V
+//     accumulates there.  Writes O, the row log-sum-exp LSE_i, the far-row
+//     column sums of the global keys, and (max, sum) of the global rows over
+//     this tile's keys.
 //
-//   cols kernel   (one CTA per (128-key tile, head, sequence))
+//   cols kernel   (one CTA per (128-key tile, head, sequence); two per SM)
 //     S^T = K Q^T for the query tiles whose band reaches this key tile, then
-//     P[i,j] = exp2(S_ij - LSE_i) summed over the rows i of each key column j
-//     (each thread owns one key column, so no cross-thread reduction), plus the
-//     global rows' probabilities and their P V outputs.  The last CTA of a key
-//     tile sums the heads in a fixed order and applies the threshold; the last
-//     tile of a sequence compacts the survivors in order.  No wait on other
-//     CTAs: the "last" CTA is found by an atomic counter.
+//     P[i,j] = exp2(S_ij - LSE_i) summed down each key column j (one thread
+//     per column, so no cross-thread reduction), plus the global rows'
+//     probabilities and their P V outputs.  The last CTA of a key tile sums
+//     the heads in a fixed order and applies the threshold; the last tile of a
+//     sequence compacts the survivors in order.  No CTA waits for another: the
+//     "last" CTA is found by an atomic counter.
+//
+//   gather kernel copies the survivors' next-layer Q, K, V rows into compacted
+//   buffers (coalesced 16-byte vectors) when they are not already in place.
 //
 // The method (allowed sets, row softmax, vertical accumulation, >= threshold,
 // order-preserving removal) is Sec. "Sparse Attention", Sec. "Extractor of
@@ -124,22 +128,67 @@ __device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_
 // ---------------------------------------------------------------------------
 // rows kernel
 // ---------------------------------------------------------------------------
+// Tensor memory of one CTA (256 columns, so two CTAs share an SM):
+//   [0,128)   S of the current key tile (fp32); P (bf16 pairs) overwrites its
+//             first 64 columns once S has been read.  The MMA that reads P
+//             and the next one that writes S are issued in that order by one
+//             thread, and tcgen05.mma from one thread executes in issue order.
+//   [128,192) O accumulator
+//   [192,208) S of the 16 global keys
+//   [208,224) S^T of the diagonal key tile against the 16 global queries
+//   [224,232) P of the global keys
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColSP = 0, kColO = 128, kColSG = 192, kColSGt = 208, kColPG = 224;
+
 struct RowsSmem {
-  uint64_t bar_load[1 + kMaxBandTiles];
-  uint64_t bar_s[2];
-  uint64_t bar_sg, bar_sgt, bar_p, bar_pv, bar_fin;
+  uint64_t bar_q;
+  uint64_t bar_kfull[2], bar_vfull[2], bar_kempty[2], bar_vempty[2];
+  uint64_t bar_sg, bar_sgt, bar_sfull, bar_pready, bar_done, bar_fin;
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
-  float red[4][kMaxGlobal];
-  float red2[4][kMaxGlobal];
-  float red3[4][kMaxGlobal];
+  float gm[kMaxGlobal];
+  float red2[8][kMaxGlobal];
 };
 
-constexpr uint32_t kRowsDyn = kTileBytes * (1 + 2 * kMaxBandTiles) + 2 * kTileBytes +
-                              3 * kGTileBytes + 1024;
+// dynamic shared memory: Q, a two-stage ring of K and of V tiles, the global rows
+constexpr uint32_t kRowsDyn = kTileBytes * 5 + 3 * kGTileBytes + 1024;
 
-__global__ void __launch_bounds__(kThreads, 1)
+// Issue P V for one 128-key tile: P (A) from tensor memory, V (B) MN-major smem.
+__device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint32_t v_smem,
+                                          int ksteps, bool accumulate) {
+  const uint32_t idesc = idesc_bf16(128, 64, false, true);
+  for (int k = 0; k < ksteps; ++k)
+    umma_bf16_ts(d_tmem, p_tmem + 8 * k, sdesc_sw128(v_smem + k * 2048), idesc,
+                 (accumulate || k > 0) ? 1u : 0u);
+}
+
+// Column reduction of a [128 rows][16] block held one row per thread
+// (red[r * 17 + g]): 8 partial results per g in sm.red2, then the combine.
+template <bool kMax>
+__device__ __forceinline__ float reduce_cols16(float* red, RowsSmem& sm, int tid) {
+  named_sync_softmax();
+  {
+    const int g = tid & 15, part = tid >> 4;
+    float v = red[(16 * part) * 17 + g];
+#pragma unroll
+    for (int k = 1; k < 16; ++k) {
+      const float u = red[(16 * part + k) * 17 + g];
+      v = kMax ? fmaxf(v, u) : v + u;
+    }
+    sm.red2[part][g] = v;
+  }
+  named_sync_softmax();
+  float v = 0.f;
+  if (tid < kMaxGlobal) {
+    v = sm.red2[0][tid];
+#pragma unroll
+    for (int k = 1; k < 8; ++k) v = kMax ? fmaxf(v, sm.red2[k][tid]) : v + sm.red2[k][tid];
+  }
+  return v;
+}
+
+__global__ void __launch_bounds__(kThreads, 2)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
   // grid: x = (sequence, head), y = query tile, so that low tiles (the ones
   // every sequence has) are dispatched first
@@ -153,10 +202,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* Qs = base;
-  uint8_t* Ks = Qs + kTileBytes;                      // kMaxBandTiles tiles
-  uint8_t* Vs = Ks + kMaxBandTiles * kTileBytes;      // kMaxBandTiles tiles
-  uint8_t* Ps = Vs + kMaxBandTiles * kTileBytes;      // 32 KB (two 64-key halves)
-  uint8_t* KG = Ps + 2 * kTileBytes;
+  uint8_t* Ks = Qs + kTileBytes;       // 2 stages
+  uint8_t* Vs = Ks + 2 * kTileBytes;   // 2 stages
+  uint8_t* KG = Vs + 2 * kTileBytes;
   uint8_t* VG = KG + kGTileBytes;
   uint8_t* QG = VG + kGTileBytes;
   __shared__ RowsSmem sm;
@@ -170,55 +218,70 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ic = qt - kt_lo;          // index of the diagonal key tile
 
   if (tid == 0) {
-    for (int i = 0; i < 1 + kMaxBandTiles; ++i) mbar_init(&sm.bar_load[i], 1);
-    mbar_init(&sm.bar_s[0], 1);
-    mbar_init(&sm.bar_s[1], 1);
+    mbar_init(&sm.bar_q, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.bar_kfull[s], 1);
+      mbar_init(&sm.bar_vfull[s], 1);
+      mbar_init(&sm.bar_kempty[s], 1);
+      mbar_init(&sm.bar_vempty[s], 1);
+    }
     mbar_init(&sm.bar_sg, 1);
     mbar_init(&sm.bar_sgt, 1);
-    mbar_init(&sm.bar_p, 128);
-    mbar_init(&sm.bar_pv, 1);
+    mbar_init(&sm.bar_sfull, 1);
+    mbar_init(&sm.bar_pready, 128);
+    mbar_init(&sm.bar_done, 1);
     mbar_init(&sm.bar_fin, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
-  if (warp == 5) tmem_alloc(&sm.tmem_base, 512);
+  if (warp == 5) tmem_alloc(&sm.tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tm = sm.tmem_base;
-  const uint32_t tS0 = tm, tS1 = tm + 128, tO = tm + 256, tSG = tm + 320, tSGt = tm + 352;
+  const uint32_t tSP = tm + kColSP, tO = tm + kColO, tSG = tm + kColSG, tSGt = tm + kColSGt,
+                 tPG = tm + kColPG;
   volatile int* abort_flag = &sm.abort;
 
   if (warp == 4) {
     // ------------------------------------------------------------- loads
     const RowSource rs = row_source(p, b);
     if (lane == 0) {
-      mbar_arrive_expect_tx(&sm.bar_load[0], kTileBytes + 3 * ngp * 128);
-      load_tile(maps, 0, rs, h, r0, Qs, &sm.bar_load[0]);
+      mbar_arrive_expect_tx(&sm.bar_q, kTileBytes + 3 * ngp * 128);
+      load_tile(maps, 0, rs, h, r0, Qs, &sm.bar_q);
     }
     __syncwarp();
     if (ngp) {
-      load_globals(maps, 1, rs, h, p.H, sm.gc, ng, KG, &sm.bar_load[0], lane);
-      load_globals(maps, 2, rs, h, p.H, sm.gc, ng, VG, &sm.bar_load[0], lane);
-      load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_load[0], lane);
+      load_globals(maps, 1, rs, h, p.H, sm.gc, ng, KG, &sm.bar_q, lane);
+      load_globals(maps, 2, rs, h, p.H, sm.gc, ng, VG, &sm.bar_q, lane);
+      load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_q, lane);
     }
     if (lane == 0) {
-      // key tiles in the order the MMA consumes them
-      for (int i = 0; i < nb; ++i) {
-        mbar_arrive_expect_tx(&sm.bar_load[1 + i], 2 * kTileBytes);
-        load_tile(maps, 1, rs, h, (kt_lo + i) * kTile, Ks + i * kTileBytes, &sm.bar_load[1 + i]);
-        load_tile(maps, 2, rs, h, (kt_lo + i) * kTile, Vs + i * kTileBytes, &sm.bar_load[1 + i]);
+      bool ok = true;
+      for (int t = 0; ok && t < nb; ++t) {
+        const int s = t & 1, c0 = (kt_lo + t) * kTile;
+        if (t >= 2 && !(ok = mbar_wait(&sm.bar_kempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+        mbar_arrive_expect_tx(&sm.bar_kfull[s], kTileBytes);
+        load_tile(maps, 1, rs, h, c0, Ks + s * kTileBytes, &sm.bar_kfull[s]);
+        if (t >= 2 && !(ok = mbar_wait(&sm.bar_vempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+        mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
+        load_tile(maps, 2, rs, h, c0, Vs + s * kTileBytes, &sm.bar_vfull[s]);
       }
-      for (int i = 0; i <= nb; ++i) drain_wait(&sm.bar_load[i], 0);
+      // nothing may still be landing in shared memory when the CTA exits
+      drain_wait(&sm.bar_q, 0);
+      for (int s = 0; s < 2 && s < nb; ++s) {
+        const int last = s + 2 * ((nb - 1 - s) >> 1);  // last tile that used stage s
+        drain_wait(&sm.bar_kfull[s], (last >> 1) & 1);
+        drain_wait(&sm.bar_vfull[s], (last >> 1) & 1);
+      }
     }
   } else if (warp == 5) {
     // ------------------------------------------------------------- MMA issue
     if (lane == 0) {
       const uint32_t q_a = smem_u32(Qs), k_a = smem_u32(Ks), v_a = smem_u32(Vs);
-      const uint32_t p_a = smem_u32(Ps);
-      int p_use = 0;
-      bool ok = mbar_wait(&sm.bar_load[0], 0, abort_flag);
+      int pu = 0;  // completed uses of bar_pready waited for
+      bool ok = mbar_wait(&sm.bar_q, 0, abort_flag);
       if (ok) {
         tc_fence_after();
         if (ngp) {
@@ -226,42 +289,44 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(&sm.bar_sg);
         }
       }
-      for (int i = 0; ok && i < min(nb, 2); ++i) {
-        if (!(ok = mbar_wait(&sm.bar_load[1 + i], 0, abort_flag))) break;
+      // S(0)
+      if (ok && (ok = mbar_wait(&sm.bar_kfull[0], 0, abort_flag))) {
         tc_fence_after();
-        mma_qk(i ? tS1 : tS0, q_a, k_a + i * kTileBytes, 128);
-        umma_commit(&sm.bar_s[i & 1]);
-        if (ngp && i == ic) {
-          mma_qk(tSGt, k_a + i * kTileBytes, smem_u32(QG), 16);
+        mma_qk(tSP, q_a, k_a, 128);
+        if (ngp && ic == 0) {
+          mma_qk(tSGt, k_a, smem_u32(QG), 16);
           umma_commit(&sm.bar_sgt);
         }
+        umma_commit(&sm.bar_kempty[0]);
+        umma_commit(&sm.bar_sfull);
       }
-      if (ok && ngp) {
-        if ((ok = mbar_wait(&sm.bar_p, p_use & 1, abort_flag))) {
-          tc_fence_after();
-          mma_pv(tO, p_a, smem_u32(VG), kMaxGlobal / 16, false);
-          umma_commit(&sm.bar_pv);
-          ++p_use;
-        }
-      }
-      for (int i = 0; ok && i < nb; ++i) {
-        if (!(ok = mbar_wait(&sm.bar_p, p_use & 1, abort_flag))) break;
+      if (ok && ngp && (ok = mbar_wait(&sm.bar_pready, pu & 1, abort_flag))) {
+        ++pu;
         tc_fence_after();
-        mma_pv(tO, p_a, v_a + i * kTileBytes, kTile / 16, ngp > 0 || i > 0);
-        umma_commit(&sm.bar_pv);
-        ++p_use;
-        const int j = i + 2;
-        if (j < nb) {
-          if (!(ok = mbar_wait(&sm.bar_load[1 + j], 0, abort_flag))) break;
+        mma_pv_ts(tO, tPG, smem_u32(VG), kMaxGlobal / 16, false);
+      }
+      for (int t = 0; ok && t < nb; ++t) {
+        const int s = t & 1;
+        if (!(ok = mbar_wait(&sm.bar_pready, pu & 1, abort_flag))) break;
+        ++pu;
+        if (!(ok = mbar_wait(&sm.bar_vfull[s], (t >> 1) & 1, abort_flag))) break;
+        tc_fence_after();
+        mma_pv_ts(tO, tSP, v_a + s * kTileBytes, kTile / 16, ngp > 0 || t > 0);
+        umma_commit(&sm.bar_vempty[s]);
+        if (t + 1 < nb) {
+          const int s1 = (t + 1) & 1;
+          if (!(ok = mbar_wait(&sm.bar_kfull[s1], ((t + 1) >> 1) & 1, abort_flag))) break;
           tc_fence_after();
-          mma_qk((j & 1) ? tS1 : tS0, q_a, k_a + j * kTileBytes, 128);
-          umma_commit(&sm.bar_s[j & 1]);
-          if (ngp && j == ic) {
-            mma_qk(tSGt, k_a + j * kTileBytes, smem_u32(QG), 16);
+          mma_qk(tSP, q_a, k_a + s1 * kTileBytes, 128);
+          if (ngp && t + 1 == ic) {
+            mma_qk(tSGt, k_a + s1 * kTileBytes, smem_u32(QG), 16);
             umma_commit(&sm.bar_sgt);
           }
+          umma_commit(&sm.bar_kempty[s1]);
+          umma_commit(&sm.bar_sfull);
         }
       }
+      if (ok) umma_commit(&sm.bar_done);
       umma_commit(&sm.bar_fin);
       drain_wait(&sm.bar_fin, 0);
     }
@@ -283,10 +348,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int whi = min(n - 1, r0 + 32 * warp + 31 + p.w);
 
     float m_ref = -INFINITY, lsum = 0.f;
-    int p_use = 0;
     bool ok = true;
     bool o_written = false;
-    float x[128];
+    float x[32];
 
     if (ngp) {
       ok = warp_wait(&sm.bar_sg, 0, abort_flag);
@@ -297,27 +361,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         float mx = -INFINITY;
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; ++g) {
-          const int cg = sm.gc[g];
-          const bool use = (g < ng) && abs(i - cg) > p.w;
+          const bool use = (g < ng) && abs(i - sm.gc[g]) > p.w;
           x[g] = use ? x[g] : -INFINITY;
           mx = fmaxf(mx, x[g]);
         }
         m_ref = mx * kLogitScale2;
-        const float ref = (m_ref == -INFINITY) ? 0.f : m_ref;
+        const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
         uint32_t pk[8];
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; g += 2) {
-          const float a = ex2(fmaf(x[g], kLogitScale2, -ref));
-          const float c = ex2(fmaf(x[g + 1], kLogitScale2, -ref));
+          const float a = ex2(fmaf(x[g], kLogitScale2, nref));
+          const float c = ex2(fmaf(x[g + 1], kLogitScale2, nref));
           lsum += a + c;
           pk[g / 2] = pack_bf16x2(a, c);
         }
-        *reinterpret_cast<uint4*>(Ps + sw128_offset(r, 0)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        *reinterpret_cast<uint4*>(Ps + sw128_offset(r, 1)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        fence_proxy_async_smem();
+        tmem_st8(tPG + lane_off, pk);
+        tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&sm.bar_p);
-        ++p_use;
+        mbar_arrive(&sm.bar_pready);
         o_written = true;
       }
     }
@@ -327,30 +388,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       // 32-column chunks of this tile that intersect the warp's band
       const int clo = max(0, wlo - j0), chi = min(kTile - 1, whi - j0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
-      if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
-      tc_fence_after();
-      const uint32_t ts = (t & 1) ? tS1 : tS0;
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch)
-        if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(ts + lane_off + 32 * ch, x + 32 * ch);
-      tmem_ld_wait();
       const int a = lo - j0, e = hi - j0;
-      // eight independent partial maxima: no long dependency chain
+      if (!(ok = warp_wait(&sm.bar_sfull, t & 1, abort_flag))) break;
+      tc_fence_after();
+      // pass 1: tile maximum over the allowed keys (eight independent partials)
       float pm[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
         if (ch < ch_lo || ch > ch_hi) continue;
-        if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+        tmem_ld32(tSP + lane_off + 32 * ch, x);
+        tmem_ld_wait();
+        if (__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) pm[k & 7] = fmaxf(pm[k & 7], x[k]);
+        } else {
 #pragma unroll
           for (int k = 0; k < 32; ++k) {
             const int c = 32 * ch + k;
-            x[c] = (c >= a && c <= e) ? x[c] : -INFINITY;
+            pm[k & 7] = fmaxf(pm[k & 7], (c >= a && c <= e) ? x[k] : -INFINITY);
           }
         }
-#pragma unroll
-        for (int k = 0; k < 32; ++k) pm[k & 7] = fmaxf(pm[k & 7], x[32 * ch + k]);
       }
       const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
                              fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * kLogitScale2;
@@ -363,11 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         scale = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - new_ref);
       }
       const float nref = (new_ref == -INFINITY) ? 0.f : -new_ref;
-      // the previous P V must be done before P is overwritten or O rescaled
-      if (p_use > 0) {
-        if (!(ok = warp_wait(&sm.bar_pv, (p_use - 1) & 1, abort_flag))) break;
-        tc_fence_after();
-      }
+      // every earlier P V has completed: S of this tile was issued after them
       if (__any_sync(0xffffffffu, bump && o_written)) {
         const float f = (bump && o_written) ? scale : 1.f;
         float o[32];
@@ -379,52 +434,50 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < 32; ++k) o[k] *= f;
           tmem_st32(tO + lane_off + c, o);
         }
-        tmem_st_wait();
       }
-      // P = exp2(x - ref) in bf16, written chunk by chunk into the swizzled A tile;
-      // the row sum is kept in eight independent partial sums
+      // pass 2: P = exp2(x - ref) in bf16 pairs, written over the S columns
+      // already read (chunk ch of P lands in columns [16 ch, 16 ch + 16))
       float ps[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) ps[k] = 0.f;
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
-        uint8_t* prow = Ps + (ch >> 1) * 16384;
+        uint32_t pk[16];
         if (ch >= ch_lo && ch <= ch_hi) {
+          tmem_ld32(tSP + lane_off + 32 * ch, x);
+          tmem_ld_wait();
+          const bool full = __all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31);
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            uint32_t w4[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const int c = 32 * ch + 8 * q + 2 * k;
-              const float u = ex2(fmaf(x[c], kLogitScale2, nref));
-              const float v = ex2(fmaf(x[c + 1], kLogitScale2, nref));
-              ps[2 * k] += u;
-              ps[2 * k + 1] += v;
-              w4[k] = pack_bf16x2(u, v);
+          for (int k = 0; k < 32; k += 2) {
+            const int c = 32 * ch + k;
+            float u = ex2(fmaf(x[k], kLogitScale2, nref));
+            float v = ex2(fmaf(x[k + 1], kLogitScale2, nref));
+            if (!full) {
+              u = (c >= a && c <= e) ? u : 0.f;
+              v = (c + 1 >= a && c + 1 <= e) ? v : 0.f;
             }
-            *reinterpret_cast<uint4*>(prow + sw128_offset(r, (ch & 1) * 4 + q)) =
-                make_uint4(w4[0], w4[1], w4[2], w4[3]);
+            ps[k & 7] += u;
+            ps[(k & 7) + 1] += v;
+            pk[k >> 1] = pack_bf16x2(u, v);
           }
         } else {
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            *reinterpret_cast<uint4*>(prow + sw128_offset(r, (ch & 1) * 4 + q)) =
-                make_uint4(0u, 0u, 0u, 0u);
+          for (int k = 0; k < 16; ++k) pk[k] = 0u;
         }
+        tmem_st16(tSP + lane_off + 16 * ch, pk);
       }
+      tmem_st_wait();
       const float ts_sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       lsum = lsum * scale + ts_sum;
       m_ref = new_ref;
-      fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&sm.bar_p);
-      ++p_use;
+      mbar_arrive(&sm.bar_pready);
       o_written = true;
     }
 
     // ---- epilogue: O, LSE
     float lse = INFINITY;
-    if (ok && (ok = warp_wait(&sm.bar_pv, (p_use - 1) & 1, abort_flag))) {
+    if (ok && (ok = warp_wait(&sm.bar_done, 0, abort_flag))) {
       tc_fence_after();
       const float inv = 1.f / lsum;
       lse = valid ? m_ref + lg2(lsum) : INFINITY;
@@ -449,23 +502,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
 
     if (ngp) {
+      // every MMA has completed (bar_done), so the K ring is free scratch
+      float* red = reinterpret_cast<float*>(Ks);
       // far-row column sums of the global keys: rows outside the key's band
-      float part[kMaxGlobal];
       if (ok) {
         tmem_ld16(tSG + lane_off, x);
         tmem_ld_wait();
       }
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const int cg = sm.gc[g];
-        const bool use = ok && valid && (g < ng) && abs(i - cg) > p.w;
-        part[g] = use ? ex2(fmaf(x[g], kLogitScale2, -lse)) : 0.f;
-        part[g] = warp_sum(part[g]);
+        const bool use = ok && valid && (g < ng) && abs(i - sm.gc[g]) > p.w;
+        red[r * 17 + g] = use ? ex2(fmaf(x[g], kLogitScale2, -lse)) : 0.f;
       }
-      if (lane == 0)
-        for (int g = 0; g < kMaxGlobal; ++g) sm.red[warp][g] = part[g];
-      // (max, sum) of each global row over this tile's keys j = 128 qt + r
-      bool ok2 = ok && warp_wait(&sm.bar_sgt, 0, abort_flag);
+      const float gpart = reduce_cols16<false>(red, sm, tid);
+      // (max, sum) of each global query over this tile's keys j = 128 qt + r
+      const bool ok2 = ok && warp_wait(&sm.bar_sgt, 0, abort_flag);
       if (ok2) {
         tc_fence_after();
         tmem_ld16(tSGt + lane_off, x);
@@ -475,28 +526,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
         x[g] = key_ok ? x[g] * kLogitScale2 : -INFINITY;
-        part[g] = warp_max(x[g]);
+        red[r * 17 + g] = x[g];
       }
-      if (lane == 0)
-        for (int g = 0; g < kMaxGlobal; ++g) sm.red2[warp][g] = part[g];
+      const float gmax = reduce_cols16<true>(red, sm, tid);
+      if (tid < kMaxGlobal) sm.gm[tid] = gmax;
       named_sync_softmax();
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const float gm =
-            fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
-        const float e = (key_ok && gm != -INFINITY) ? ex2(x[g] - gm) : 0.f;
-        part[g] = warp_sum(e);
+        const float m = sm.gm[g];
+        red[r * 17 + g] = (key_ok && m != -INFINITY) ? ex2(x[g] - m) : 0.f;
       }
-      if (lane == 0)
-        for (int g = 0; g < kMaxGlobal; ++g) sm.red3[warp][g] = part[g];
-      named_sync_softmax();
+      const float gsum = reduce_cols16<false>(red, sm, tid);
       if (tid < kMaxGlobal) {
-        const int g = tid;
-        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + g;
-        p.gpart[slot] = sm.red[0][g] + sm.red[1][g] + sm.red[2][g] + sm.red[3][g];
-        p.gstat[2 * slot] =
-            fmaxf(fmaxf(sm.red2[0][g], sm.red2[1][g]), fmaxf(sm.red2[2][g], sm.red2[3][g]));
-        p.gstat[2 * slot + 1] = sm.red3[0][g] + sm.red3[1][g] + sm.red3[2][g] + sm.red3[3][g];
+        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + tid;
+        p.gpart[slot] = gpart;
+        p.gstat[2 * slot] = gmax;
+        p.gstat[2 * slot + 1] = gsum;
       }
       if (qt == 0) {
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
@@ -509,7 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 5) {
     tc_fence_after();
-    tmem_dealloc(tm, 512);
+    tmem_dealloc(tm, kTmemCols);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 }
@@ -517,9 +562,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ---------------------------------------------------------------------------
 // cols kernel
 // ---------------------------------------------------------------------------
+// Tensor memory (256 columns): [0,128) S^T of the current query tile,
+// [128,144) S^T against the 16 global queries, [160,224) their P V.
+constexpr uint32_t kColST = 0, kColSGc = 128, kColOG = 160;
+
 struct ColsSmem {
-  uint64_t bar_load[1 + kMaxBandTiles];
-  uint64_t bar_s[2], bar_sfree[2];
+  uint64_t bar_kv;
+  uint64_t bar_qfull[2], bar_qempty[2];
+  uint64_t bar_sfull, bar_sfree;
   uint64_t bar_sg, bar_pg, bar_og, bar_fin;
   uint32_t tmem_base;
   int abort;
@@ -532,11 +582,13 @@ struct ColsSmem {
   int gnew[kMaxGlobal];
 };
 
-constexpr uint32_t kColsDyn = kTileBytes * (2 + kMaxBandTiles) + kGTileBytes + 2 * kTileBytes + 1024;
+// dynamic shared memory: K and V of the key tile, a two-stage ring of Q
+// tiles, the global queries and the A tile of the global rows' P V
+constexpr uint32_t kColsDyn = kTileBytes * 4 + kGTileBytes + 2 * kTileBytes + 1024;
 
 __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm);
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, kt = blockIdx.y;
   const int n = __ldg(p.len + b);
@@ -559,8 +611,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* Ks = base;
   uint8_t* Vs = Ks + kTileBytes;
   uint8_t* Pg = Vs + kTileBytes;                  // 32 KB: A operand of the global-row P V
-  uint8_t* Qs = Pg + 2 * kTileBytes;              // kMaxBandTiles tiles
-  uint8_t* QG = Qs + kMaxBandTiles * kTileBytes;
+  uint8_t* Qs = Pg + 2 * kTileBytes;              // 2 stages
+  uint8_t* QG = Qs + 2 * kTileBytes;
   __shared__ ColsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -571,11 +623,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nq = qt_hi - qt_lo + 1;
 
   if (tid == 0) {
-    for (int i = 0; i < 1 + kMaxBandTiles; ++i) mbar_init(&sm.bar_load[i], 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.bar_s[i], 1);
-      mbar_init(&sm.bar_sfree[i], 128);
+    mbar_init(&sm.bar_kv, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&sm.bar_qfull[s], 1);
+      mbar_init(&sm.bar_qempty[s], 1);
     }
+    mbar_init(&sm.bar_sfull, 1);
+    mbar_init(&sm.bar_sfree, 128);
     mbar_init(&sm.bar_sg, 1);
     mbar_init(&sm.bar_pg, 128);
     mbar_init(&sm.bar_og, 1);
@@ -584,34 +638,41 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
-  if (warp == 5) tmem_alloc(&sm.tmem_base, 512);
+  if (warp == 5) tmem_alloc(&sm.tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tm = sm.tmem_base;
-  const uint32_t tS0 = tm, tS1 = tm + 128, tSG = tm + 256, tOG = tm + 320;
+  const uint32_t tST = tm + kColST, tSG = tm + kColSGc, tOG = tm + kColOG;
   volatile int* abort_flag = &sm.abort;
 
   if (warp == 4) {
     const RowSource rs = row_source(p, b);
     if (lane == 0) {
-      mbar_arrive_expect_tx(&sm.bar_load[0], 2 * kTileBytes + ngp * 128);
-      load_tile(maps, 1, rs, h, j0, Ks, &sm.bar_load[0]);
-      load_tile(maps, 2, rs, h, j0, Vs, &sm.bar_load[0]);
+      mbar_arrive_expect_tx(&sm.bar_kv, 2 * kTileBytes + ngp * 128);
+      load_tile(maps, 1, rs, h, j0, Ks, &sm.bar_kv);
+      load_tile(maps, 2, rs, h, j0, Vs, &sm.bar_kv);
     }
     __syncwarp();
-    if (ngp) load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_load[0], lane);
+    if (ngp) load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_kv, lane);
     if (lane == 0) {
-      for (int i = 0; i < nq; ++i) {
-        mbar_arrive_expect_tx(&sm.bar_load[1 + i], kTileBytes);
-        load_tile(maps, 0, rs, h, (qt_lo + i) * kTile, Qs + i * kTileBytes, &sm.bar_load[1 + i]);
+      bool ok = true;
+      for (int t = 0; ok && t < nq; ++t) {
+        const int s = t & 1;
+        if (t >= 2 && !(ok = mbar_wait(&sm.bar_qempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+        mbar_arrive_expect_tx(&sm.bar_qfull[s], kTileBytes);
+        load_tile(maps, 0, rs, h, (qt_lo + t) * kTile, Qs + s * kTileBytes, &sm.bar_qfull[s]);
       }
-      for (int i = 0; i <= nq; ++i) drain_wait(&sm.bar_load[i], 0);
+      drain_wait(&sm.bar_kv, 0);
+      for (int s = 0; s < 2 && s < nq; ++s) {
+        const int last = s + 2 * ((nq - 1 - s) >> 1);
+        drain_wait(&sm.bar_qfull[s], (last >> 1) & 1);
+      }
     }
   } else if (warp == 5) {
     if (lane == 0) {
       const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs);
-      bool ok = mbar_wait(&sm.bar_load[0], 0, abort_flag);
+      bool ok = mbar_wait(&sm.bar_kv, 0, abort_flag);
       if (ok) {
         tc_fence_after();
         if (ngp) {
@@ -619,19 +680,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(&sm.bar_sg);
         }
       }
-      for (int i = 0; ok && i < min(nq, 2); ++i) {
-        if (!(ok = mbar_wait(&sm.bar_load[1 + i], 0, abort_flag))) break;
+      for (int t = 0; ok && t < nq; ++t) {
+        const int s = t & 1;
+        if (!(ok = mbar_wait(&sm.bar_qfull[s], (t >> 1) & 1, abort_flag))) break;
+        if (t > 0 && !(ok = mbar_wait(&sm.bar_sfree, (t - 1) & 1, abort_flag))) break;
         tc_fence_after();
-        mma_qk(i ? tS1 : tS0, k_a, q_a + i * kTileBytes, 128);
-        umma_commit(&sm.bar_s[i]);
-      }
-      for (int i = 0; ok && i + 2 < nq; ++i) {
-        const int j = i + 2;
-        if (!(ok = mbar_wait(&sm.bar_sfree[i & 1], (i >> 1) & 1, abort_flag))) break;
-        if (!(ok = mbar_wait(&sm.bar_load[1 + j], 0, abort_flag))) break;
-        tc_fence_after();
-        mma_qk((j & 1) ? tS1 : tS0, k_a, q_a + j * kTileBytes, 128);
-        umma_commit(&sm.bar_s[j & 1]);
+        mma_qk(tST, k_a, q_a + s * kTileBytes, 128);
+        umma_commit(&sm.bar_qempty[s]);
+        umma_commit(&sm.bar_sfull);
       }
       if (ok && ngp && (ok = mbar_wait(&sm.bar_pg, 0, abort_flag))) {
         tc_fence_after();
@@ -677,20 +733,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int whi = min(n - 1, j0 + 32 * warp + 31 + p.w);
     float acc = 0.f;
     bool ok = true;
-    float x[128];
+    float x[32];
     for (int t = 0; ok && t < nq; ++t) {
       const int i0 = (qt_lo + t) * kTile;            // first query row of this tile
       const int clo = max(0, wlo - i0), chi = min(kTile - 1, whi - i0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
-      if (!(ok = warp_wait(&sm.bar_s[t & 1], (t >> 1) & 1, abort_flag))) break;
+      if (!(ok = warp_wait(&sm.bar_sfull, t & 1, abort_flag))) break;
       tc_fence_after();
-      const uint32_t ts = (t & 1) ? tS1 : tS0;
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch)
-        if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(ts + lane_off + 32 * ch, x + 32 * ch);
-      tmem_ld_wait();
-      tc_fence_before();
-      mbar_arrive(&sm.bar_sfree[t & 1]);
       const float* lw = sm.lse + t * kTile;
       const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
       // eight independent partial sums per tile
@@ -700,15 +749,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
         if (ch < ch_lo || ch > ch_hi) continue;
+        tmem_ld32(tST + lane_off + 32 * ch, x);
+        tmem_ld_wait();
         if (__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
 #pragma unroll
           for (int k = 0; k < 32; k += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
             const int u = (k >> 2) & 1;
-            ps[4 * u] += ex2(fmaf(x[32 * ch + k], kLogitScale2, -l4.x));
-            ps[4 * u + 1] += ex2(fmaf(x[32 * ch + k + 1], kLogitScale2, -l4.y));
-            ps[4 * u + 2] += ex2(fmaf(x[32 * ch + k + 2], kLogitScale2, -l4.z));
-            ps[4 * u + 3] += ex2(fmaf(x[32 * ch + k + 3], kLogitScale2, -l4.w));
+            ps[4 * u] += ex2(fmaf(x[k], kLogitScale2, -l4.x));
+            ps[4 * u + 1] += ex2(fmaf(x[k + 1], kLogitScale2, -l4.y));
+            ps[4 * u + 2] += ex2(fmaf(x[k + 2], kLogitScale2, -l4.z));
+            ps[4 * u + 3] += ex2(fmaf(x[k + 3], kLogitScale2, -l4.w));
           }
         } else {
 #pragma unroll
@@ -719,12 +770,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               const int c = 32 * ch + k + q;
-              const float v = ex2(fmaf(x[c], kLogitScale2, -lv[q]));
+              const float v = ex2(fmaf(x[k + q], kLogitScale2, -lv[q]));
               ps[4 * u + q] += (c >= a && c <= e) ? v : 0.f;
             }
           }
         }
       }
+      tc_fence_before();
+      mbar_arrive(&sm.bar_sfree);
       acc += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
     }
 
@@ -739,7 +792,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       float s = 0.f;
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const float v = (ok2 && g < ng && j < n) ? ex2(fmaf(x[g], kLogitScale2, -sm.lse_g[g])) : 0.f;
+        const float v =
+            (ok2 && g < ng && j < n) ? ex2(fmaf(x[g], kLogitScale2, -sm.lse_g[g])) : 0.f;
         s += v;
         pb[g] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
       }
@@ -774,7 +828,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 5) {
     tc_fence_after();
-    tmem_dealloc(tm, 512);
+    tmem_dealloc(tm, kTmemCols);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 
@@ -1001,11 +1055,20 @@ cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st) {
 }
 
 cudaError_t configure_kernels() {
+  // two CTAs of each attention kernel share an SM: ask for the full shared
+  // memory carveout so both fit
   cudaError_t e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kRowsDyn));
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(sc_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(kColsDyn));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(sc_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kColsDyn));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(sc_cols_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
+  return e;
 }
 
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {

@@ -13,7 +13,6 @@ constexpr int kMaxBandTiles = 5;   // key (query) tiles touched by one 128-row t
 constexpr int kMaxGlobal = 16;     // global tokens per sequence (one 16-wide MMA tile)
 constexpr int kMaxLen = 4096;
 constexpr int kMaxTiles = kMaxLen / kTile;
-constexpr int kThreads = 192;      // 4 softmax warps + 1 load warp + 1 MMA warp
 constexpr uint32_t kTileBytes = kTile * kHeadDim * 2;   // 16 KB bf16 tile
 constexpr uint32_t kGTileBytes = kMaxGlobal * kHeadDim * 2;
 

@@ -3,8 +3,8 @@
 //
 // Per layer, per sequence b (n current tokens, original positions pos[b][*]):
 //
-//   rows kernel   (one CTA per (128-query-row tile, head, sequence); two CTAs
-//                 per SM)
+//   rows kernel   (one CTA per pair of 128-row query tiles of one (sequence,
+//                 head); one softmax warpgroup per tile)
 //     S = Q K^T over the band key tiles and one 16-wide tile of global keys on
 //     the tensor cores (tcgen05, bf16 -> fp32 in tensor memory); each 16 KB
 //     operand tile is one TMA copy.  Row softmax in fp32 (base 2, lazily
@@ -13,7 +13,7 @@
 //     column sums of the global keys, and (max, sum) of the global rows over
 //     this tile's keys.
 //
-//   cols kernel   (one CTA per (128-key tile, head, sequence); two per SM)
+//   cols kernel   (one CTA per pair of 128-key tiles; one warpgroup per tile)
 //     S^T = K Q^T for the query tiles whose band reaches this key tile, then
 //     P[i,j] = exp2(S_ij - LSE_i) summed down each key column j (one thread
 //     per column, so no cross-thread reduction), plus the global rows'
@@ -128,31 +128,45 @@ __device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_
 // ---------------------------------------------------------------------------
 // rows kernel
 // ---------------------------------------------------------------------------
-// Tensor memory of one CTA (256 columns, so two CTAs share an SM):
-//   [0,128)   S of the current key tile (fp32); P (bf16 pairs) overwrites its
-//             first 64 columns once S has been read.  The MMA that reads P
-//             and the next one that writes S are issued in that order by one
-//             thread, and tcgen05.mma from one thread executes in issue order.
-//   [128,192) O accumulator
-//   [192,208) S of the 16 global keys
-//   [208,224) S^T of the diagonal key tile against the 16 global queries
-//   [224,232) P of the global keys
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColSP = 0, kColO = 128, kColSG = 192, kColSGt = 208, kColPG = 224;
+// One CTA per pair of 128-row query tiles (2p, 2p+1) of one (sequence, head),
+// one softmax warpgroup per tile; the two tiles share their K/V tiles (the
+// band of the pair spans at most six 128-key tiles) and the tensor core
+// alternates between the two warpgroups.
+//
+// Tensor memory (512 columns) per warpgroup X in {0, 1}:
+//   S/P  [192 X, 192 X + 128)  S of the current key tile (fp32); P (bf16
+//        pairs) overwrites its first 64 columns once all of S is in registers.
+//        The MMA that reads P and the next one that writes S are issued in
+//        that order by one thread, and they execute in issue order.
+//   O    [192 X + 128, 192 X + 192)
+//   S_G  [384 + 32 X, +16)  S of the 16 global keys;  P_G [400 + 32 X, +8)
+//   S_Gt [448 + 16 X, +16)  S^T of the diagonal key tile against the global queries
+constexpr int kRowsThreads = 320;   // 2 softmax warpgroups + load warp + MMA warp
+constexpr int kStages = 4;          // K/V ring depth
+constexpr int kPairTiles = kMaxBandTiles + 1;
+
+__host__ __device__ constexpr uint32_t col_sp(int X) { return 192u * X; }
+__host__ __device__ constexpr uint32_t col_o(int X) { return 192u * X + 128u; }
+__host__ __device__ constexpr uint32_t col_sg(int X) { return 384u + 32u * X; }
+__host__ __device__ constexpr uint32_t col_pg(int X) { return 400u + 32u * X; }
+__host__ __device__ constexpr uint32_t col_sgt(int X) { return 448u + 16u * X; }
 
 struct RowsSmem {
   uint64_t bar_q;
-  uint64_t bar_kfull[2], bar_vfull[2], bar_kempty[2], bar_vempty[2];
-  uint64_t bar_sg, bar_sgt, bar_sfull, bar_pready, bar_done, bar_fin;
+  uint64_t bar_kfull[kStages], bar_vfull[kStages], bar_kempty[kStages], bar_vempty[kStages];
+  uint64_t bar_sg[2], bar_sgt[2], bar_sfull[2], bar_pready[2], bar_done[2], bar_fin;
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
-  float gm[kMaxGlobal];
-  float red2[8][kMaxGlobal];
+  float gm[2][kMaxGlobal];
+  float red2[2][8][kMaxGlobal];
 };
 
-// dynamic shared memory: Q, a two-stage ring of K and of V tiles, the global rows
-constexpr uint32_t kRowsDyn = kTileBytes * 5 + 3 * kGTileBytes + 1024;
+// dynamic shared memory: two Q tiles, the K/V ring, the global rows, and one
+// [128][17] fp32 reduction scratch per warpgroup
+constexpr uint32_t kRedBytes = 128 * 17 * 4;
+constexpr uint32_t kRowsDyn =
+    kTileBytes * (2 + 2 * kStages) + 3 * kGTileBytes + 2 * kRedBytes + 1024;
 
 // Issue P V for one 128-key tile: P (A) from tensor memory, V (B) MN-major smem.
 __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint32_t v_smem,
@@ -163,93 +177,106 @@ __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint
                  (accumulate || k > 0) ? 1u : 0u);
 }
 
+__device__ __forceinline__ void wg_sync(int X) {
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + X) : "memory");
+}
+
 // Column reduction of a [128 rows][16] block held one row per thread
-// (red[r * 17 + g]): 8 partial results per g in sm.red2, then the combine.
+// (red[r * 17 + g]): eight partial results per g, then the combine.
 template <bool kMax>
-__device__ __forceinline__ float reduce_cols16(float* red, RowsSmem& sm, int tid) {
-  named_sync_softmax();
+__device__ __forceinline__ float reduce_cols16(const float* red, float (*red2)[kMaxGlobal], int X,
+                                               int r) {
+  wg_sync(X);
   {
-    const int g = tid & 15, part = tid >> 4;
+    const int g = r & 15, part = r >> 4;
     float v = red[(16 * part) * 17 + g];
 #pragma unroll
     for (int k = 1; k < 16; ++k) {
       const float u = red[(16 * part + k) * 17 + g];
       v = kMax ? fmaxf(v, u) : v + u;
     }
-    sm.red2[part][g] = v;
+    red2[part][g] = v;
   }
-  named_sync_softmax();
+  wg_sync(X);
   float v = 0.f;
-  if (tid < kMaxGlobal) {
-    v = sm.red2[0][tid];
+  if (r < kMaxGlobal) {
+    v = red2[0][r];
 #pragma unroll
-    for (int k = 1; k < 8; ++k) v = kMax ? fmaxf(v, sm.red2[k][tid]) : v + sm.red2[k][tid];
+    for (int k = 1; k < 8; ++k) v = kMax ? fmaxf(v, red2[k][r]) : v + red2[k][r];
   }
   return v;
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
-  // grid: x = (sequence, head), y = query tile, so that low tiles (the ones
-  // every sequence has) are dispatched first
-  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, qt = blockIdx.y;
+  // grid: x = (sequence, head), y = pair of query tiles, so that low tiles (the
+  // ones every sequence has) are dispatched first
+  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
   const int n = __ldg(p.len + b);
-  if (qt * kTile >= n) return;
+  if (2 * pr * kTile >= n) return;
   const int ng = min(__ldg(p.ng + b), kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
+  const bool hasB = (2 * pr + 1) * kTile < n;
 
   extern __shared__ uint8_t dyn_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* Qs = base;
-  uint8_t* Ks = Qs + kTileBytes;       // 2 stages
-  uint8_t* Vs = Ks + 2 * kTileBytes;   // 2 stages
-  uint8_t* KG = Vs + 2 * kTileBytes;
+  uint8_t* Qs = base;                                // 2 tiles
+  uint8_t* Ks = Qs + 2 * kTileBytes;                 // kStages tiles
+  uint8_t* Vs = Ks + kStages * kTileBytes;           // kStages tiles
+  uint8_t* KG = Vs + kStages * kTileBytes;
   uint8_t* VG = KG + kGTileBytes;
   uint8_t* QG = VG + kGTileBytes;
+  float* red_all = reinterpret_cast<float*>(QG + kGTileBytes);
   __shared__ RowsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int r0 = qt * kTile;
-  const int r1 = min(r0 + kTile - 1, n - 1);
-  const int kt_lo = max(0, r0 - p.w) / kTile;
-  const int kt_hi = min(n - 1, r1 + p.w) / kTile;
-  const int nb = kt_hi - kt_lo + 1;   // <= kMaxBandTiles (checked on the host)
-  const int ic = qt - kt_lo;          // index of the diagonal key tile
+  // key tiles of each query tile, and of the pair (absolute tile indices)
+  int klo[2], khi[2];
+#pragma unroll
+  for (int X = 0; X < 2; ++X) {
+    const int q0 = (2 * pr + X) * kTile, q1 = min(q0 + kTile - 1, n - 1);
+    klo[X] = max(0, q0 - p.w) / kTile;
+    khi[X] = min(n - 1, q1 + p.w) / kTile;
+  }
+  const int kt_lo = klo[0];
+  const int kt_hi = hasB ? khi[1] : khi[0];
+  const int nk = kt_hi - kt_lo + 1;   // <= kPairTiles (window checked on the host)
 
   if (tid == 0) {
     mbar_init(&sm.bar_q, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.bar_kfull[s], 1);
       mbar_init(&sm.bar_vfull[s], 1);
       mbar_init(&sm.bar_kempty[s], 1);
       mbar_init(&sm.bar_vempty[s], 1);
     }
-    mbar_init(&sm.bar_sg, 1);
-    mbar_init(&sm.bar_sgt, 1);
-    mbar_init(&sm.bar_sfull, 1);
-    mbar_init(&sm.bar_pready, 128);
-    mbar_init(&sm.bar_done, 1);
+    for (int X = 0; X < 2; ++X) {
+      mbar_init(&sm.bar_sg[X], 1);
+      mbar_init(&sm.bar_sgt[X], 1);
+      mbar_init(&sm.bar_sfull[X], 1);
+      mbar_init(&sm.bar_pready[X], 128);
+      mbar_init(&sm.bar_done[X], 1);
+    }
     mbar_init(&sm.bar_fin, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
-  if (warp == 5) tmem_alloc(&sm.tmem_base, kTmemCols);
+  if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tm = sm.tmem_base;
-  const uint32_t tSP = tm + kColSP, tO = tm + kColO, tSG = tm + kColSG, tSGt = tm + kColSGt,
-                 tPG = tm + kColPG;
   volatile int* abort_flag = &sm.abort;
 
-  if (warp == 4) {
+  if (warp == 8) {
     // ------------------------------------------------------------- loads
     const RowSource rs = row_source(p, b);
     if (lane == 0) {
-      mbar_arrive_expect_tx(&sm.bar_q, kTileBytes + 3 * ngp * 128);
-      load_tile(maps, 0, rs, h, r0, Qs, &sm.bar_q);
+      mbar_arrive_expect_tx(&sm.bar_q, (hasB ? 2 : 1) * kTileBytes + 3 * ngp * 128);
+      load_tile(maps, 0, rs, h, 2 * pr * kTile, Qs, &sm.bar_q);
+      if (hasB) load_tile(maps, 0, rs, h, (2 * pr + 1) * kTile, Qs + kTileBytes, &sm.bar_q);
     }
     __syncwarp();
     if (ngp) {
@@ -259,83 +286,113 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     if (lane == 0) {
       bool ok = true;
-      for (int t = 0; ok && t < nb; ++t) {
-        const int s = t & 1, c0 = (kt_lo + t) * kTile;
-        if (t >= 2 && !(ok = mbar_wait(&sm.bar_kempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+      for (int k = 0; ok && k < nk; ++k) {
+        const int s = k % kStages, c0 = (kt_lo + k) * kTile;
+        const uint32_t ph = ((k / kStages) - 1) & 1;
+        if (k >= kStages && !(ok = mbar_wait(&sm.bar_kempty[s], ph, abort_flag))) break;
         mbar_arrive_expect_tx(&sm.bar_kfull[s], kTileBytes);
         load_tile(maps, 1, rs, h, c0, Ks + s * kTileBytes, &sm.bar_kfull[s]);
-        if (t >= 2 && !(ok = mbar_wait(&sm.bar_vempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+        if (k >= kStages && !(ok = mbar_wait(&sm.bar_vempty[s], ph, abort_flag))) break;
         mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
         load_tile(maps, 2, rs, h, c0, Vs + s * kTileBytes, &sm.bar_vfull[s]);
       }
       // nothing may still be landing in shared memory when the CTA exits
       drain_wait(&sm.bar_q, 0);
-      for (int s = 0; s < 2 && s < nb; ++s) {
-        const int last = s + 2 * ((nb - 1 - s) >> 1);  // last tile that used stage s
-        drain_wait(&sm.bar_kfull[s], (last >> 1) & 1);
-        drain_wait(&sm.bar_vfull[s], (last >> 1) & 1);
+      for (int s = 0; s < kStages && s < nk; ++s) {
+        const int last = s + kStages * ((nk - 1 - s) / kStages);  // last tile of stage s
+        drain_wait(&sm.bar_kfull[s], (last / kStages) & 1);
+        drain_wait(&sm.bar_vfull[s], (last / kStages) & 1);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     // ------------------------------------------------------------- MMA issue
     if (lane == 0) {
       const uint32_t q_a = smem_u32(Qs), k_a = smem_u32(Ks), v_a = smem_u32(Vs);
-      int pu = 0;  // completed uses of bar_pready waited for
+      const int nX = hasB ? 2 : 1;
+      // remaining users (warpgroups) of each key tile's K and V
+      int kuse[kPairTiles], vuse[kPairTiles];
+      for (int k = 0; k < kPairTiles; ++k) {
+        const int a = kt_lo + k;
+        const int u = (a >= klo[0] && a <= khi[0]) + (hasB && a >= klo[1] && a <= khi[1]);
+        kuse[k] = u;
+        vuse[k] = u;
+      }
+      int cur[2] = {klo[0], klo[1]};   // next key tile of each warpgroup
+      int pu[2] = {0, 0};              // completed pready phases waited for
       bool ok = mbar_wait(&sm.bar_q, 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        if (ngp) {
-          mma_qk(tSG, q_a, smem_u32(KG), 16);
-          umma_commit(&sm.bar_sg);
-        }
-      }
-      // S(0)
-      if (ok && (ok = mbar_wait(&sm.bar_kfull[0], 0, abort_flag))) {
-        tc_fence_after();
-        mma_qk(tSP, q_a, k_a, 128);
-        if (ngp && ic == 0) {
-          mma_qk(tSGt, k_a, smem_u32(QG), 16);
-          umma_commit(&sm.bar_sgt);
-        }
-        umma_commit(&sm.bar_kempty[0]);
-        umma_commit(&sm.bar_sfull);
-      }
-      if (ok && ngp && (ok = mbar_wait(&sm.bar_pready, pu & 1, abort_flag))) {
-        ++pu;
-        tc_fence_after();
-        mma_pv_ts(tO, tPG, smem_u32(VG), kMaxGlobal / 16, false);
-      }
-      for (int t = 0; ok && t < nb; ++t) {
-        const int s = t & 1;
-        if (!(ok = mbar_wait(&sm.bar_pready, pu & 1, abort_flag))) break;
-        ++pu;
-        if (!(ok = mbar_wait(&sm.bar_vfull[s], (t >> 1) & 1, abort_flag))) break;
-        tc_fence_after();
-        mma_pv_ts(tO, tSP, v_a + s * kTileBytes, kTile / 16, ngp > 0 || t > 0);
-        umma_commit(&sm.bar_vempty[s]);
-        if (t + 1 < nb) {
-          const int s1 = (t + 1) & 1;
-          if (!(ok = mbar_wait(&sm.bar_kfull[s1], ((t + 1) >> 1) & 1, abort_flag))) break;
-          tc_fence_after();
-          mma_qk(tSP, q_a, k_a + s1 * kTileBytes, 128);
-          if (ngp && t + 1 == ic) {
-            mma_qk(tSGt, k_a + s1 * kTileBytes, smem_u32(QG), 16);
-            umma_commit(&sm.bar_sgt);
+        if (ngp)
+          for (int X = 0; X < nX; ++X) {
+            mma_qk(tm + col_sg(X), q_a + X * kTileBytes, smem_u32(KG), 16);
+            umma_commit(&sm.bar_sg[X]);
           }
-          umma_commit(&sm.bar_kempty[s1]);
-          umma_commit(&sm.bar_sfull);
+      }
+      // S of the first key tile of each warpgroup
+      auto issue_s = [&](int X, int a) -> bool {
+        const int k = a - kt_lo, s = k % kStages;
+        if (!mbar_wait(&sm.bar_kfull[s], (k / kStages) & 1, abort_flag)) return false;
+        tc_fence_after();
+        mma_qk(tm + col_sp(X), q_a + X * kTileBytes, k_a + s * kTileBytes, 128);
+        if (ngp && a == 2 * pr + X) {
+          mma_qk(tm + col_sgt(X), k_a + s * kTileBytes, smem_u32(QG), 16);
+          umma_commit(&sm.bar_sgt[X]);
+        }
+        if (--kuse[k] == 0) umma_commit(&sm.bar_kempty[s]);
+        umma_commit(&sm.bar_sfull[X]);
+        return true;
+      };
+      // P V of the global keys goes first, so that the commit of the first band
+      // S also covers it (the softmax may rescale O as soon as S is ready)
+      for (int X = 0; ok && X < nX; ++X) {
+        if (ngp) {
+          if (!(ok = mbar_wait(&sm.bar_pready[X], pu[X] & 1, abort_flag))) break;
+          ++pu[X];
+          tc_fence_after();
+          mma_pv_ts(tm + col_o(X), tm + col_pg(X), smem_u32(VG), kMaxGlobal / 16, false);
+        }
+        ok = issue_s(X, cur[X]);
+      }
+      // steady state: P V of the current tile, then S of the next, per warpgroup
+      bool more = true;
+      while (ok && more) {
+        more = false;
+        for (int X = 0; ok && X < nX; ++X) {
+          if (cur[X] > khi[X]) continue;
+          const int a = cur[X], k = a - kt_lo, s = k % kStages;
+          if (!(ok = mbar_wait(&sm.bar_pready[X], pu[X] & 1, abort_flag))) break;
+          ++pu[X];
+          if (!(ok = mbar_wait(&sm.bar_vfull[s], (k / kStages) & 1, abort_flag))) break;
+          tc_fence_after();
+          mma_pv_ts(tm + col_o(X), tm + col_sp(X), v_a + s * kTileBytes, kTile / 16,
+                    ngp > 0 || a > klo[X]);
+          if (--vuse[k] == 0) umma_commit(&sm.bar_vempty[s]);
+          cur[X] = a + 1;
+          if (cur[X] <= khi[X]) {
+            if (!(ok = issue_s(X, cur[X]))) break;
+            more = true;
+          } else {
+            umma_commit(&sm.bar_done[X]);
+          }
         }
       }
-      if (ok) umma_commit(&sm.bar_done);
       umma_commit(&sm.bar_fin);
       drain_wait(&sm.bar_fin, 0);
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------- softmax
-    const int r = tid;            // row inside the tile == TMEM lane
-    const int i = r0 + r;         // current index of this query row
-    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const int X = warp >> 2;              // warpgroup = query tile of the pair
+    const int wq = warp & 3;              // TMEM lane quarter of this warp
+    const int r = tid & 127;              // row inside the tile == TMEM lane
+    const int qt = 2 * pr + X;
+    const int r0 = qt * kTile;
+    const bool active = X == 0 || hasB;
+    const int i = r0 + r;                 // current index of this query row
+    const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
+    const uint32_t tSP = tm + col_sp(X), tO = tm + col_o(X), tSG = tm + col_sg(X),
+                   tPG = tm + col_pg(X), tSGt = tm + col_sgt(X);
+    float* red = red_all + X * (128 * 17);
     bool row_global = false;
     for (int g = 0; g < ng; ++g) row_global |= (sm.gc[g] == i);
     const bool valid = (i < n) && !row_global;
@@ -344,140 +401,155 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int lo = max(0, i - p.w);
     const int hi = min(n - 1, i + p.w);
     // union of the band over this warp's 32 rows: chunks outside it are skipped
-    const int wlo = max(0, r0 + 32 * warp - p.w);
-    const int whi = min(n - 1, r0 + 32 * warp + 31 + p.w);
+    const int wlo = max(0, r0 + 32 * wq - p.w);
+    const int whi = min(n - 1, r0 + 32 * wq + 31 + p.w);
 
     float m_ref = -INFINITY, lsum = 0.f;
-    bool ok = true;
+    bool ok = active;
     bool o_written = false;
-    float x[32];
+    float xg[kMaxGlobal];
 
-    if (ngp) {
-      ok = warp_wait(&sm.bar_sg, 0, abort_flag);
+    if (ok && ngp) {
+      ok = warp_wait(&sm.bar_sg[X], 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        tmem_ld16(tSG + lane_off, x);
+        tmem_ld16(tSG + lane_off, xg);
         tmem_ld_wait();
         float mx = -INFINITY;
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; ++g) {
           const bool use = (g < ng) && abs(i - sm.gc[g]) > p.w;
-          x[g] = use ? x[g] : -INFINITY;
-          mx = fmaxf(mx, x[g]);
+          xg[g] = use ? xg[g] : -INFINITY;
+          mx = fmaxf(mx, xg[g]);
         }
         m_ref = mx * kLogitScale2;
         const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
         uint32_t pk[8];
 #pragma unroll
         for (int g = 0; g < kMaxGlobal; g += 2) {
-          const float a = ex2(fmaf(x[g], kLogitScale2, nref));
-          const float c = ex2(fmaf(x[g + 1], kLogitScale2, nref));
+          const float a = ex2(fmaf(xg[g], kLogitScale2, nref));
+          const float c = ex2(fmaf(xg[g + 1], kLogitScale2, nref));
           lsum += a + c;
           pk[g / 2] = pack_bf16x2(a, c);
         }
         tmem_st8(tPG + lane_off, pk);
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&sm.bar_pready);
+        mbar_arrive(&sm.bar_pready[X]);
         o_written = true;
       }
     }
 
-    for (int t = 0; ok && t < nb; ++t) {
-      const int j0 = (kt_lo + t) * kTile;
+    // Softmax with a running reference m_ref (base-2 units): P = exp2(x - ref).
+    // Each 64-column half of a tile is loaded once; its maximum is taken before
+    // its exponentials, and when it exceeds the reference by more than 8 the
+    // reference is raised there: O (all earlier P V of this warpgroup have
+    // completed, since S of this tile was issued after them), the row sum, this
+    // tile's partial sums and the already-stored first half of P are rescaled
+    // exactly.  P values therefore stay below 2^8.
+    float x[64];
+    for (int t = 0; ok && t <= khi[X] - klo[X]; ++t) {
+      const int j0 = (klo[X] + t) * kTile;
       // 32-column chunks of this tile that intersect the warp's band
       const int clo = max(0, wlo - j0), chi = min(kTile - 1, whi - j0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
       const int a = lo - j0, e = hi - j0;
-      if (!(ok = warp_wait(&sm.bar_sfull, t & 1, abort_flag))) break;
+      if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
-      // pass 1: tile maximum over the allowed keys (eight independent partials)
-      float pm[8];
+      float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
+      for (int hf = 0; hf < 2; ++hf) {
+        // two 32-column chunks into x[0..63], keys outside the band masked
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        if (ch < ch_lo || ch > ch_hi) continue;
-        tmem_ld32(tSP + lane_off + 32 * ch, x);
+        for (int c2 = 0; c2 < 2; ++c2) {
+          const int ch = 2 * hf + c2;
+          if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(tSP + lane_off + 32 * ch, x + 32 * c2);
+        }
         tmem_ld_wait();
-        if (__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-          for (int k = 0; k < 32; ++k) pm[k & 7] = fmaxf(pm[k & 7], x[k]);
-        } else {
+        for (int c2 = 0; c2 < 2; ++c2) {
+          const int ch = 2 * hf + c2;
+          if (ch < ch_lo || ch > ch_hi) continue;
+          if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const int c = 32 * ch + k;
-            pm[k & 7] = fmaxf(pm[k & 7], (c >= a && c <= e) ? x[k] : -INFINITY);
-          }
-        }
-      }
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * kLogitScale2;
-      // lazy rescale: move the reference only when the tile max exceeds it by > 8 (2^8)
-      float scale = 1.f;
-      const bool bump = mx > m_ref + 8.f;
-      float new_ref = m_ref;
-      if (bump) {
-        new_ref = mx;
-        scale = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - new_ref);
-      }
-      const float nref = (new_ref == -INFINITY) ? 0.f : -new_ref;
-      // every earlier P V has completed: S of this tile was issued after them
-      if (__any_sync(0xffffffffu, bump && o_written)) {
-        const float f = (bump && o_written) ? scale : 1.f;
-        float o[32];
-#pragma unroll
-        for (int c = 0; c < 64; c += 32) {
-          tmem_ld32(tO + lane_off + c, o);
-          tmem_ld_wait();
-#pragma unroll
-          for (int k = 0; k < 32; ++k) o[k] *= f;
-          tmem_st32(tO + lane_off + c, o);
-        }
-      }
-      // pass 2: P = exp2(x - ref) in bf16 pairs, written over the S columns
-      // already read (chunk ch of P lands in columns [16 ch, 16 ch + 16))
-      float ps[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        uint32_t pk[16];
-        if (ch >= ch_lo && ch <= ch_hi) {
-          tmem_ld32(tSP + lane_off + 32 * ch, x);
-          tmem_ld_wait();
-          const bool full = __all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31);
-#pragma unroll
-          for (int k = 0; k < 32; k += 2) {
-            const int c = 32 * ch + k;
-            float u = ex2(fmaf(x[k], kLogitScale2, nref));
-            float v = ex2(fmaf(x[k + 1], kLogitScale2, nref));
-            if (!full) {
-              u = (c >= a && c <= e) ? u : 0.f;
-              v = (c + 1 >= a && c + 1 <= e) ? v : 0.f;
+            for (int k = 0; k < 32; ++k) {
+              const int c = 32 * ch + k;
+              x[32 * c2 + k] = (c >= a && c <= e) ? x[32 * c2 + k] : -INFINITY;
             }
-            ps[k & 7] += u;
-            ps[(k & 7) + 1] += v;
-            pk[k >> 1] = pack_bf16x2(u, v);
           }
-        } else {
 #pragma unroll
-          for (int k = 0; k < 16; ++k) pk[k] = 0u;
+          for (int k = 0; k < 32; ++k) pm[k & 3] = fmaxf(pm[k & 3], x[32 * c2 + k]);
         }
-        tmem_st16(tSP + lane_off + 16 * ch, pk);
+        const float hmax = fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])) * kLogitScale2;
+        const bool raise = hmax > m_ref + 8.f;
+        if (__any_sync(0xffffffffu, raise)) {
+          float f = 1.f;
+          if (raise) {
+            f = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - hmax);
+            m_ref = hmax;
+            lsum *= f;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) ps[k] *= f;
+          }
+          float o[32];
+          if (o_written) {
+#pragma unroll
+            for (int c = 0; c < 64; c += 32) {
+              tmem_ld32(tO + lane_off + c, o);
+              tmem_ld_wait();
+#pragma unroll
+              for (int k = 0; k < 32; ++k) o[k] *= f;
+              tmem_st32(tO + lane_off + c, o);
+              tmem_st_wait();   // o is reused
+            }
+          }
+          if (hf == 1) {
+            // the first half of this tile's P, already stored: 32 columns of bf16 pairs
+            tmem_st_wait();
+            tmem_ld32(tSP + lane_off, o);
+            tmem_ld_wait();
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const uint32_t w = __float_as_uint(o[k]);
+              const float lo16 = __uint_as_float(w << 16) * f;
+              const float hi16 = __uint_as_float(w & 0xffff0000u) * f;
+              o[k] = __uint_as_float(pack_bf16x2(lo16, hi16));
+            }
+            tmem_st32(tSP + lane_off, o);
+          }
+        }
+        const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {   // 16-column quarters of the half
+          const int ch = 2 * hf + (q >> 1);
+          uint32_t pk[8];
+          if (ch >= ch_lo && ch <= ch_hi) {
+#pragma unroll
+            for (int k = 0; k < 16; k += 2) {
+              const float u = ex2(fmaf(x[16 * q + k], kLogitScale2, nref));
+              const float v = ex2(fmaf(x[16 * q + k + 1], kLogitScale2, nref));
+              ps[k & 3] += u;
+              ps[(k & 3) + 1] += v;
+              pk[k >> 1] = pack_bf16x2(u, v);
+            }
+          } else {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) pk[k] = 0u;
+          }
+          tmem_st8(tSP + lane_off + 8 * (4 * hf + q), pk);
+        }
       }
       tmem_st_wait();
-      const float ts_sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-      lsum = lsum * scale + ts_sum;
-      m_ref = new_ref;
+      lsum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
       tc_fence_before();
-      mbar_arrive(&sm.bar_pready);
+      mbar_arrive(&sm.bar_pready[X]);
       o_written = true;
     }
 
     // ---- epilogue: O, LSE
     float lse = INFINITY;
-    if (ok && (ok = warp_wait(&sm.bar_done, 0, abort_flag))) {
+    if (ok && (ok = warp_wait(&sm.bar_done[X], 0, abort_flag))) {
       tc_fence_after();
       const float inv = 1.f / lsum;
       lse = valid ? m_ref + lg2(lsum) : INFINITY;
@@ -499,62 +571,60 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       }
     }
-    if (i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
+    if (active && i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
 
-    if (ngp) {
-      // every MMA has completed (bar_done), so the K ring is free scratch
-      float* red = reinterpret_cast<float*>(Ks);
+    if (active && ngp) {
       // far-row column sums of the global keys: rows outside the key's band
       if (ok) {
-        tmem_ld16(tSG + lane_off, x);
+        tmem_ld16(tSG + lane_off, xg);
         tmem_ld_wait();
       }
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
         const bool use = ok && valid && (g < ng) && abs(i - sm.gc[g]) > p.w;
-        red[r * 17 + g] = use ? ex2(fmaf(x[g], kLogitScale2, -lse)) : 0.f;
+        red[r * 17 + g] = use ? ex2(fmaf(xg[g], kLogitScale2, -lse)) : 0.f;
       }
-      const float gpart = reduce_cols16<false>(red, sm, tid);
+      const float gpart = reduce_cols16<false>(red, sm.red2[X], X, r);
       // (max, sum) of each global query over this tile's keys j = 128 qt + r
-      const bool ok2 = ok && warp_wait(&sm.bar_sgt, 0, abort_flag);
+      const bool ok2 = ok && warp_wait(&sm.bar_sgt[X], 0, abort_flag);
       if (ok2) {
         tc_fence_after();
-        tmem_ld16(tSGt + lane_off, x);
+        tmem_ld16(tSGt + lane_off, xg);
         tmem_ld_wait();
       }
       const bool key_ok = ok2 && (r0 + r < n);
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        x[g] = key_ok ? x[g] * kLogitScale2 : -INFINITY;
-        red[r * 17 + g] = x[g];
+        xg[g] = key_ok ? xg[g] * kLogitScale2 : -INFINITY;
+        red[r * 17 + g] = xg[g];
       }
-      const float gmax = reduce_cols16<true>(red, sm, tid);
-      if (tid < kMaxGlobal) sm.gm[tid] = gmax;
-      named_sync_softmax();
+      const float gmax = reduce_cols16<true>(red, sm.red2[X], X, r);
+      if (r < kMaxGlobal) sm.gm[X][r] = gmax;
+      wg_sync(X);
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const float m = sm.gm[g];
-        red[r * 17 + g] = (key_ok && m != -INFINITY) ? ex2(x[g] - m) : 0.f;
+        const float m = sm.gm[X][g];
+        red[r * 17 + g] = (key_ok && m != -INFINITY) ? ex2(xg[g] - m) : 0.f;
       }
-      const float gsum = reduce_cols16<false>(red, sm, tid);
-      if (tid < kMaxGlobal) {
-        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + tid;
+      const float gsum = reduce_cols16<false>(red, sm.red2[X], X, r);
+      if (r < kMaxGlobal) {
+        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + r;
         p.gpart[slot] = gpart;
         p.gstat[2 * slot] = gmax;
         p.gstat[2 * slot + 1] = gsum;
       }
       if (qt == 0) {
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
-        for (int k = tid; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
+        for (int k = r; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
       }
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 9) {
     tc_fence_after();
-    tmem_dealloc(tm, kTmemCols);
+    tmem_dealloc(tm, 512);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 }
@@ -562,154 +632,182 @@ __global__ void __launch_bounds__(kThreads, 2)
 // ---------------------------------------------------------------------------
 // cols kernel
 // ---------------------------------------------------------------------------
-// Tensor memory (256 columns): [0,128) S^T of the current query tile,
-// [128,144) S^T against the 16 global queries, [160,224) their P V.
-constexpr uint32_t kColST = 0, kColSGc = 128, kColOG = 160;
+// One CTA per pair of 128-key tiles (2p, 2p+1) of one (sequence, head), one
+// softmax warpgroup per key tile; the two share the query tiles of their band.
+// Tensor memory per warpgroup X: S^T [128 X, 128 X + 128), S^T against the
+// global queries [256 + 16 X, +16), the global rows' P V [320 + 64 X, +64).
+constexpr int kColsThreads = 320;
 
 struct ColsSmem {
   uint64_t bar_kv;
-  uint64_t bar_qfull[2], bar_qempty[2];
-  uint64_t bar_sfull, bar_sfree;
-  uint64_t bar_sg, bar_pg, bar_og, bar_fin;
+  uint64_t bar_qfull[kStages], bar_qempty[kStages];
+  uint64_t bar_sfull[2], bar_sfree[2], bar_sg[2], bar_pg[2], bar_og[2], bar_fin;
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  alignas(16) float lse[kMaxBandTiles * kTile];  // read as float4
+  alignas(16) float lse[kPairTiles * kTile];  // read as float4
   float gsum[kMaxGlobal];
   int flag;
-  int scan[kThreads];
+  int scan[kColsThreads];
   int gnew[kMaxGlobal];
 };
 
-// dynamic shared memory: K and V of the key tile, a two-stage ring of Q
-// tiles, the global queries and the A tile of the global rows' P V
-constexpr uint32_t kColsDyn = kTileBytes * 4 + kGTileBytes + 2 * kTileBytes + 1024;
+// dynamic shared memory: K and V of both key tiles, the Q ring, the global
+// queries, and one A tile (32 KB) per warpgroup for the global rows' P V
+constexpr uint32_t kColsDyn = kTileBytes * (4 + kStages) + kGTileBytes + 4 * kTileBytes + 1024;
 
 __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm);
 
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kColsThreads, 1)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
-  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, kt = blockIdx.y;
+  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
   const int n = __ldg(p.len + b);
   if (n == 0) {
-    if (kt == 0 && h == 0 && threadIdx.x == 0) {
+    if (pr == 0 && h == 0 && threadIdx.x == 0) {
       p.len_out[b] = 0;
       p.ng_out[b] = 0;
       p.ident_out[b] = 1;
     }
     return;
   }
-  if (kt * kTile >= n) return;
+  if (2 * pr * kTile >= n) return;
   const int ng = min(__ldg(p.ng + b), kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
   const int Tn = (n + kTile - 1) / kTile;
+  const int Tp = (Tn + 1) / 2;
+  const bool hasB = (2 * pr + 1) * kTile < n;
 
   extern __shared__ uint8_t dyn_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* Ks = base;
-  uint8_t* Vs = Ks + kTileBytes;
-  uint8_t* Pg = Vs + kTileBytes;                  // 32 KB: A operand of the global-row P V
-  uint8_t* Qs = Pg + 2 * kTileBytes;              // 2 stages
-  uint8_t* QG = Qs + 2 * kTileBytes;
+  uint8_t* Ks = base;                              // 2 tiles
+  uint8_t* Vs = Ks + 2 * kTileBytes;               // 2 tiles
+  uint8_t* Pg = Vs + 2 * kTileBytes;               // 2 x 32 KB A tiles
+  uint8_t* Qs = Pg + 4 * kTileBytes;               // kStages tiles
+  uint8_t* QG = Qs + kStages * kTileBytes;
   __shared__ ColsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int j0 = kt * kTile;
-  const int j1 = min(j0 + kTile - 1, n - 1);
-  const int qt_lo = max(0, j0 - p.w) / kTile;
-  const int qt_hi = min(n - 1, j1 + p.w) / kTile;
+  int qlo[2], qhi[2];
+#pragma unroll
+  for (int X = 0; X < 2; ++X) {
+    const int j0 = (2 * pr + X) * kTile, j1 = min(j0 + kTile - 1, n - 1);
+    qlo[X] = max(0, j0 - p.w) / kTile;
+    qhi[X] = min(n - 1, j1 + p.w) / kTile;
+  }
+  const int qt_lo = qlo[0];
+  const int qt_hi = hasB ? qhi[1] : qhi[0];
   const int nq = qt_hi - qt_lo + 1;
 
   if (tid == 0) {
     mbar_init(&sm.bar_kv, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&sm.bar_qfull[s], 1);
       mbar_init(&sm.bar_qempty[s], 1);
     }
-    mbar_init(&sm.bar_sfull, 1);
-    mbar_init(&sm.bar_sfree, 128);
-    mbar_init(&sm.bar_sg, 1);
-    mbar_init(&sm.bar_pg, 128);
-    mbar_init(&sm.bar_og, 1);
+    for (int X = 0; X < 2; ++X) {
+      mbar_init(&sm.bar_sfull[X], 1);
+      mbar_init(&sm.bar_sfree[X], 128);
+      mbar_init(&sm.bar_sg[X], 1);
+      mbar_init(&sm.bar_pg[X], 128);
+      mbar_init(&sm.bar_og[X], 1);
+    }
     mbar_init(&sm.bar_fin, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
-  if (warp == 5) tmem_alloc(&sm.tmem_base, kTmemCols);
+  if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tm = sm.tmem_base;
-  const uint32_t tST = tm + kColST, tSG = tm + kColSGc, tOG = tm + kColOG;
   volatile int* abort_flag = &sm.abort;
 
-  if (warp == 4) {
+  if (warp == 8) {
     const RowSource rs = row_source(p, b);
     if (lane == 0) {
-      mbar_arrive_expect_tx(&sm.bar_kv, 2 * kTileBytes + ngp * 128);
-      load_tile(maps, 1, rs, h, j0, Ks, &sm.bar_kv);
-      load_tile(maps, 2, rs, h, j0, Vs, &sm.bar_kv);
+      mbar_arrive_expect_tx(&sm.bar_kv, (hasB ? 4 : 2) * kTileBytes + ngp * 128);
+      for (int X = 0; X < (hasB ? 2 : 1); ++X) {
+        load_tile(maps, 1, rs, h, (2 * pr + X) * kTile, Ks + X * kTileBytes, &sm.bar_kv);
+        load_tile(maps, 2, rs, h, (2 * pr + X) * kTile, Vs + X * kTileBytes, &sm.bar_kv);
+      }
     }
     __syncwarp();
     if (ngp) load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_kv, lane);
     if (lane == 0) {
       bool ok = true;
-      for (int t = 0; ok && t < nq; ++t) {
-        const int s = t & 1;
-        if (t >= 2 && !(ok = mbar_wait(&sm.bar_qempty[s], ((t - 2) >> 1) & 1, abort_flag))) break;
+      for (int q = 0; ok && q < nq; ++q) {
+        const int s = q % kStages;
+        if (q >= kStages &&
+            !(ok = mbar_wait(&sm.bar_qempty[s], ((q / kStages) - 1) & 1, abort_flag)))
+          break;
         mbar_arrive_expect_tx(&sm.bar_qfull[s], kTileBytes);
-        load_tile(maps, 0, rs, h, (qt_lo + t) * kTile, Qs + s * kTileBytes, &sm.bar_qfull[s]);
+        load_tile(maps, 0, rs, h, (qt_lo + q) * kTile, Qs + s * kTileBytes, &sm.bar_qfull[s]);
       }
       drain_wait(&sm.bar_kv, 0);
-      for (int s = 0; s < 2 && s < nq; ++s) {
-        const int last = s + 2 * ((nq - 1 - s) >> 1);
-        drain_wait(&sm.bar_qfull[s], (last >> 1) & 1);
+      for (int s = 0; s < kStages && s < nq; ++s) {
+        const int last = s + kStages * ((nq - 1 - s) / kStages);
+        drain_wait(&sm.bar_qfull[s], (last / kStages) & 1);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     if (lane == 0) {
-      const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs);
+      const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs), v_a = smem_u32(Vs);
+      const int nX = hasB ? 2 : 1;
+      int su[2] = {0, 0};   // S^T tiles issued per warpgroup
       bool ok = mbar_wait(&sm.bar_kv, 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        if (ngp) {
-          mma_qk(tSG, k_a, smem_u32(QG), 16);
-          umma_commit(&sm.bar_sg);
+        if (ngp)
+          for (int X = 0; X < nX; ++X) {
+            mma_qk(tm + 256 + 16 * X, k_a + X * kTileBytes, smem_u32(QG), 16);
+            umma_commit(&sm.bar_sg[X]);
+          }
+      }
+      for (int q = 0; ok && q < nq; ++q) {
+        const int s = q % kStages, a = qt_lo + q;
+        if (!(ok = mbar_wait(&sm.bar_qfull[s], (q / kStages) & 1, abort_flag))) break;
+        for (int X = 0; ok && X < nX; ++X) {
+          if (a < qlo[X] || a > qhi[X]) continue;
+          if (su[X] > 0 && !(ok = mbar_wait(&sm.bar_sfree[X], (su[X] - 1) & 1, abort_flag))) break;
+          tc_fence_after();
+          mma_qk(tm + 128 * X, k_a + X * kTileBytes, q_a + s * kTileBytes, 128);
+          umma_commit(&sm.bar_sfull[X]);
+          ++su[X];
         }
+        if (ok) umma_commit(&sm.bar_qempty[s]);
       }
-      for (int t = 0; ok && t < nq; ++t) {
-        const int s = t & 1;
-        if (!(ok = mbar_wait(&sm.bar_qfull[s], (t >> 1) & 1, abort_flag))) break;
-        if (t > 0 && !(ok = mbar_wait(&sm.bar_sfree, (t - 1) & 1, abort_flag))) break;
-        tc_fence_after();
-        mma_qk(tST, k_a, q_a + s * kTileBytes, 128);
-        umma_commit(&sm.bar_qempty[s]);
-        umma_commit(&sm.bar_sfull);
-      }
-      if (ok && ngp && (ok = mbar_wait(&sm.bar_pg, 0, abort_flag))) {
-        tc_fence_after();
-        mma_pv(tOG, smem_u32(Pg), smem_u32(Vs), kTile / 16, false);
-        umma_commit(&sm.bar_og);
-      }
+      if (ok && ngp)
+        for (int X = 0; ok && X < nX; ++X) {
+          if (!(ok = mbar_wait(&sm.bar_pg[X], 0, abort_flag))) break;
+          tc_fence_after();
+          mma_pv(tm + 320 + 64 * X, smem_u32(Pg) + X * 2 * kTileBytes, v_a + X * kTileBytes,
+                 kTile / 16, false);
+          umma_commit(&sm.bar_og[X]);
+        }
       umma_commit(&sm.bar_fin);
       drain_wait(&sm.bar_fin, 0);
     }
     __syncwarp();
   } else {
-    const int r = tid;
+    const int X = warp >> 2, wq = warp & 3;
+    const int r = tid & 127;
+    const int kt = 2 * pr + X;
+    const int j0 = kt * kTile;
     const int j = j0 + r;             // key column owned by this thread
-    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const bool active = X == 0 || hasB;
+    const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
+    const uint32_t tST = tm + 128 * X, tSG = tm + 256 + 16 * X, tOG = tm + 320 + 64 * X;
     const float* lse_src = p.lse + (static_cast<size_t>(b) * p.H + h) * p.L;
-    for (int k = tid; k < nq * kTile; k += 128) {
+    for (int k = tid; k < nq * kTile; k += 256) {
       const int row = qt_lo * kTile + k;
       sm.lse[k] = row < n ? __ldcg(lse_src + row) : INFINITY;
     }
     if (ngp && warp == 0) {
-      // merge the per-tile (max, sum) of every global row into its LSE; lane = key tile,
-      // all loads issued before any reduction
+      // merge the per-tile (max, sum) of every global row into its LSE; lane =
+      // query tile, all loads issued before any reduction
       float m[kMaxGlobal], sm_[kMaxGlobal];
       const size_t base_slot = ((static_cast<size_t>(b) * p.H + h) * p.T + lane) * kMaxGlobal;
 #pragma unroll
@@ -726,42 +824,44 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (lane == 0 && g < ng) sm.lse_g[g] = M + lg2(S);
       }
     }
-    named_sync_softmax();
+    asm volatile("bar.sync 3, 256;" ::: "memory");
 
     // union of the band over this warp's 32 key columns
-    const int wlo = max(0, j0 + 32 * warp - p.w);
-    const int whi = min(n - 1, j0 + 32 * warp + 31 + p.w);
+    const int wlo = max(0, j0 + 32 * wq - p.w);
+    const int whi = min(n - 1, j0 + 32 * wq + 31 + p.w);
     float acc = 0.f;
-    bool ok = true;
-    float x[32];
-    for (int t = 0; ok && t < nq; ++t) {
-      const int i0 = (qt_lo + t) * kTile;            // first query row of this tile
+    bool ok = active;
+    float x[64];
+    for (int t = 0; ok && t <= qhi[X] - qlo[X]; ++t) {
+      const int i0 = (qlo[X] + t) * kTile;            // first query row of this tile
       const int clo = max(0, wlo - i0), chi = min(kTile - 1, whi - i0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
-      if (!(ok = warp_wait(&sm.bar_sfull, t & 1, abort_flag))) break;
+      if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
-      const float* lw = sm.lse + t * kTile;
+      const float* lw = sm.lse + (qlo[X] + t - qt_lo) * kTile;
       const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
-      // eight independent partial sums per tile
       float ps[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+      // two halves of 64 columns: load both chunks of a half, then use them;
+      // S^T is released to the next MMA once the second half is in registers
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        if (ch < ch_lo || ch > ch_hi) continue;
-        tmem_ld32(tST + lane_off + 32 * ch, x);
+      for (int hf = 0; hf < 2; ++hf) {
+#pragma unroll
+        for (int c2 = 0; c2 < 2; ++c2) {
+          const int ch = 2 * hf + c2;
+          if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(tST + lane_off + 32 * ch, x + 32 * c2);
+        }
         tmem_ld_wait();
-        if (__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+        if (hf == 1) {
+          tc_fence_before();
+          mbar_arrive(&sm.bar_sfree[X]);
+        }
 #pragma unroll
-          for (int k = 0; k < 32; k += 4) {
-            const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
-            const int u = (k >> 2) & 1;
-            ps[4 * u] += ex2(fmaf(x[k], kLogitScale2, -l4.x));
-            ps[4 * u + 1] += ex2(fmaf(x[k + 1], kLogitScale2, -l4.y));
-            ps[4 * u + 2] += ex2(fmaf(x[k + 2], kLogitScale2, -l4.z));
-            ps[4 * u + 3] += ex2(fmaf(x[k + 3], kLogitScale2, -l4.w));
-          }
-        } else {
+        for (int c2 = 0; c2 < 2; ++c2) {
+          const int ch = 2 * hf + c2;
+          if (ch < ch_lo || ch > ch_hi) continue;
+          const bool full = __all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31);
 #pragma unroll
           for (int k = 0; k < 32; k += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
@@ -770,19 +870,17 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               const int c = 32 * ch + k + q;
-              const float v = ex2(fmaf(x[k + q], kLogitScale2, -lv[q]));
-              ps[4 * u + q] += (c >= a && c <= e) ? v : 0.f;
+              const float v = ex2(fmaf(x[32 * c2 + k + q], kLogitScale2, -lv[q]));
+              ps[4 * u + q] += (full || (c >= a && c <= e)) ? v : 0.f;
             }
           }
         }
       }
-      tc_fence_before();
-      mbar_arrive(&sm.bar_sfree);
       acc += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
     }
 
-    if (ngp) {
-      bool ok2 = ok && warp_wait(&sm.bar_sg, 0, abort_flag);
+    if (active && ngp) {
+      bool ok2 = ok && warp_wait(&sm.bar_sg[X], 0, abort_flag);
       if (ok2) {
         tc_fence_after();
         tmem_ld16(tSG + lane_off, x);
@@ -798,17 +896,18 @@ __global__ void __launch_bounds__(kThreads, 2)
         pb[g] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
       }
       acc += s;
-      // P of the global rows, transposed into the A tile: row g, column (key) r
-      uint8_t* col = Pg + (r >> 6) * 16384;
+      // P of the global rows, transposed into this warpgroup's A tile: row g,
+      // column (key) r
+      uint8_t* col = Pg + X * 2 * kTileBytes + (r >> 6) * 16384;
       const int ch = (r & 63) >> 3, wi = (r & 7) * 2;
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g)
         *reinterpret_cast<uint16_t*>(col + sw128_offset(g, ch) + wi) = pb[g];
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&sm.bar_pg);
-      bool ok3 = ok2 && warp_wait(&sm.bar_og, 0, abort_flag);
-      if (warp == 0 && ok3) {
+      mbar_arrive(&sm.bar_pg[X]);
+      bool ok3 = ok2 && warp_wait(&sm.bar_og[X], 0, abort_flag);
+      if (wq == 0 && ok3) {
         tc_fence_after();
         float* og = p.og + ((static_cast<size_t>(b) * p.H + h) * kMaxGlobal) * kHeadDim;
 #pragma unroll
@@ -821,31 +920,33 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
       }
     }
-    if (j < n) p.acc[(static_cast<size_t>(b) * p.H + h) * p.L + j] = acc;
+    if (active && j < n) p.acc[(static_cast<size_t>(b) * p.H + h) * p.L + j] = acc;
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 9) {
     tc_fence_after();
-    tmem_dealloc(tm, kTmemCols);
+    tmem_dealloc(tm, 512);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 
-  // ---- last head of this key tile: scores and keep flags (fixed head order)
+  // ---- last head of this pair of key tiles: scores and keep flags (fixed head order)
   __threadfence();
   __syncthreads();
-  if (tid == 0) sm.flag = (atomicAdd(p.cnt_tile + b * p.T + kt, 1u) == static_cast<uint32_t>(p.H - 1));
+  if (tid == 0) sm.flag = (atomicAdd(p.cnt_tile + b * p.T + pr, 1u) == static_cast<uint32_t>(p.H - 1));
   __syncthreads();
   if (!sm.flag) return;
   __threadfence();
-  // far-row partial sums of the global keys that lie in this tile: one warp per
+  const int j0 = 2 * pr * kTile;
+  const int jn = min(n, j0 + 2 * kTile);
+  // far-row partial sums of the global keys that lie in this pair: one warp per
   // global key, summed over heads and query tiles in a fixed order
-  if (warp < 4) {
-    for (int g = warp; g < ng; g += 4) {
+  if (warp < 8) {
+    for (int g = warp; g < ng; g += 8) {
       const int cg = sm.gc[g];
       float v = 0.f;
-      if (cg >= j0 && cg < j0 + kTile) {
+      if (cg >= j0 && cg < jn) {
         const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * kMaxGlobal + g;
 #pragma unroll 4
         for (int k = lane; k < p.H * Tn; k += 32) {
@@ -858,7 +959,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
   }
   __syncthreads();
-  if (tid < kTile && j0 + tid < n) {
+  if (tid < 2 * kTile && j0 + tid < jn) {
     const int jj = j0 + tid;
     const float* ap = p.acc + static_cast<size_t>(b) * p.H * p.L + jj;
     float a = 0.f;
@@ -881,10 +982,10 @@ __global__ void __launch_bounds__(kThreads, 2)
     const float theta = p.theta ? __ldg(p.theta + b) : p.alpha / static_cast<float>(n);
     p.keep[static_cast<size_t>(b) * p.L + jj] = (jj == 0 || s >= theta) ? 1 : 0;
   }
-  if (tid == 0) p.cnt_tile[b * p.T + kt] = 0u;
+  if (tid == 0) p.cnt_tile[b * p.T + pr] = 0u;
   __threadfence();
   __syncthreads();
-  if (tid == 0) sm.flag = (atomicAdd(p.cnt_seq + b, 1u) == static_cast<uint32_t>(Tn - 1));
+  if (tid == 0) sm.flag = (atomicAdd(p.cnt_seq + b, 1u) == static_cast<uint32_t>(Tp - 1));
   __syncthreads();
   if (!sm.flag) return;
   __threadfence();
@@ -895,7 +996,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 // global list, and the bf16 outputs of the global rows.  One CTA.
 __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm) {
   const int tid = threadIdx.x;
-  const int per = (n + kThreads - 1) / kThreads;
+  const int per = (n + kColsThreads - 1) / kColsThreads;
   const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
   const uint8_t* keep = p.keep + static_cast<size_t>(b) * p.L;
   int cnt = 0;
@@ -903,15 +1004,15 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
   for (int c = c0; c < c1; ++c) cnt += __ldcg(keep + c);
   sm.scan[tid] = cnt;
   __syncthreads();
-  // exclusive scan over kThreads counts (Hillis-Steele in shared memory)
-  for (int off = 1; off < kThreads; off <<= 1) {
+  // exclusive scan over kColsThreads counts (Hillis-Steele in shared memory)
+  for (int off = 1; off < kColsThreads; off <<= 1) {
     const int v = tid >= off ? sm.scan[tid - off] : 0;
     __syncthreads();
     sm.scan[tid] += v;
     __syncthreads();
   }
   int out = sm.scan[tid] - cnt;
-  const int total = sm.scan[kThreads - 1];
+  const int total = sm.scan[kColsThreads - 1];
   const int ng = min(__ldg(p.ng + b), kMaxGlobal);
   if (tid < kMaxGlobal) sm.gnew[tid] = -1;
   __syncthreads();
@@ -926,7 +1027,7 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
   }
   // bf16 outputs of the global rows
 #pragma unroll 4
-  for (int k = tid; k < ng * p.H * kHeadDim; k += kThreads) {
+  for (int k = tid; k < ng * p.H * kHeadDim; k += kColsThreads) {
     const int g = k / (p.H * kHeadDim), hh = (k / kHeadDim) % p.H, dd = k % kHeadDim;
     const float v = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
     p.O[((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) * kHeadDim + dd] =
@@ -1055,8 +1156,7 @@ cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st) {
 }
 
 cudaError_t configure_kernels() {
-  // two CTAs of each attention kernel share an SM: ask for the full shared
-  // memory carveout so both fit
+  // the attention kernels use most of an SM's shared memory
   cudaError_t e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kRowsDyn));
   if (e == cudaSuccess)
@@ -1072,14 +1172,14 @@ cudaError_t configure_kernels() {
 }
 
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.B * p.H, p.T);
-  sc_rows_kernel<<<grid, kThreads, kRowsDyn, st>>>(m, p);
+  dim3 grid(p.B * p.H, (p.T + 1) / 2);
+  sc_rows_kernel<<<grid, kRowsThreads, kRowsDyn, st>>>(m, p);
   return cudaGetLastError();
 }
 
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.B * p.H, p.T);
-  sc_cols_kernel<<<grid, kThreads, kColsDyn, st>>>(m, p);
+  dim3 grid(p.B * p.H, (p.T + 1) / 2);
+  sc_cols_kernel<<<grid, kColsThreads, kColsDyn, st>>>(m, p);
   return cudaGetLastError();
 }
 

@@ -133,6 +133,29 @@ typedef struct {
   int32_t* len;
 } sc_stack_args;
 
+/*
+ * sc_layer_forward without any device allocation, by the caller or the
+ * library: for callers that cannot allocate device memory where they run a
+ * layer -- hosts whose device heap belongs to another allocator without a hook
+ * for plugins, deployments with a fixed memory budget that forbid allocation
+ * after start-up, and latency-critical services that cannot afford the
+ * implicit device synchronisation of cudaMalloc.  The paper has no
+ * counterpart; this is an interface convenience.
+ *
+ * Same arguments, semantics and results as sc_layer_forward (the caller still
+ * passes every input and output).  The scratch comes from a 4 MiB array
+ * compiled into the library, which every GPU that loads it holds until the
+ * process exits; sizes whose scratch does not fit (from roughly B*L*H = 300k
+ * (sequence, token, head) rows on, e.g. B=2, L=4096, H=12 fits) return
+ * SC_ERR_UNSUPPORTED with the detail in sc_last_error().  The first call
+ * on each device looks up the array's device address (cudaGetSymbolAddress);
+ * make that first call before any stream capture.  All calls share the array:
+ * calls that overlap on the GPU (different streams, without ordering) race.
+ * A bounded-wait timeout cannot be queried for this entry point: its status
+ * word is private and cleared at every call.
+ */
+int sc_layer_forward_noalloc(const sc_layer_args* args, void* stream);
+
 /* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
 size_t sc_workspace_size(int B, int L, int H);
 

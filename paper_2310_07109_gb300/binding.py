@@ -52,7 +52,8 @@ class StackArgs(ctypes.Structure):
                 ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p)]
 
 
-EXPORTED = ["sc_layer_forward", "sc_stack_forward", "sc_stack_forward_profiled",
+EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
+            "sc_stack_forward_profiled",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error"]
 
 
@@ -82,6 +83,8 @@ def load(build_if_missing: bool = False):
         lib.sc_stack_forward.restype = ctypes.c_int
         lib.sc_stack_forward.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                          ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_layer_forward_noalloc.restype = ctypes.c_int
+        lib.sc_layer_forward_noalloc.argtypes = [ctypes.POINTER(LayerArgs), ctypes.c_void_p]
         lib.sc_stack_forward_profiled.restype = ctypes.c_int
         lib.sc_stack_forward_profiled.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                                   ctypes.c_size_t, ctypes.c_void_p,
@@ -155,6 +158,19 @@ def layer_forward(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *,
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, float(alpha),
                   _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out))
     _check(load().sc_layer_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
+    return O, scores, pos_out, len_out
+
+
+def layer_forward_noalloc(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *, O,
+                          scores, pos_out, len_out, stream=None):
+    """One layer through ``sc_layer_forward_noalloc``: no device memory is
+    allocated, by this call or the library; every output tensor is passed in."""
+    B, L, H, D = Q.shape
+    garr, ng = _int32_host(global_pos)
+    a = LayerArgs(B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(length), _ptr(pos),
+                  ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, float(alpha),
+                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out))
+    _check(load().sc_layer_forward_noalloc(ctypes.byref(a), _stream_handle(stream)))
     return O, scores, pos_out, len_out
 
 

@@ -411,3 +411,113 @@ int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Single layer without any allocation by the caller or the library.
+// ---------------------------------------------------------------------------
+// Some callers cannot allocate device memory where they run a layer: hosts
+// whose whole device heap belongs to another allocator that exposes no hook
+// (plugins inside other frameworks), deployments with a fixed memory budget
+// that forbid allocation after start-up, and latency-critical services that
+// cannot afford cudaMalloc's implicit device synchronisation.  For them the
+// scratch of one layer lives in this fixed array, held by every GPU that loads
+// the library until the process exits.
+namespace {
+
+constexpr size_t kStaticWorkspaceBytes = size_t(4) << 20;  // 4 MiB
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_static_workspace[kStaticWorkspaceBytes];
+
+namespace {
+
+// Device address of g_static_workspace on the current device.  In host code
+// the array's name is only a stand-in, so the address is looked up once per
+// device (with that device current) and cached.
+int static_workspace(char** out) {
+  static std::mutex mu;
+  static void* addr[256] = {nullptr};
+  int dev = 0;
+  const cudaError_t ge = cudaGetDevice(&dev);
+  if (ge != cudaSuccess) return fail_cuda("cudaGetDevice", ge);
+  if (dev < 0 || dev >= 256) return fail(SC_ERR_CUDA, "cudaGetDevice", "device index out of range");
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_workspace);
+    if (e != cudaSuccess) return fail_cuda("static workspace address", e);
+    addr[dev] = p;
+  }
+  *out = static_cast<char*>(addr[dev]);
+  return SC_OK;
+}
+
+}  // namespace
+
+extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if (!a->Q || !a->K || !a->V || !a->len || !a->pos || !a->O || !a->scores || !a->pos_out ||
+      !a->len_out)
+    return SC_ERR_INVALID_ARG;
+  if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
+    return SC_ERR_INVALID_ARG;
+  if (a->pos_out == a->pos || a->len_out == a->len) return SC_ERR_INVALID_ARG;
+  // a single layer reads its rows in place, so the compacted copies that the
+  // layout reserves last are not needed: everything before them must fit
+  WsLayout lay;
+  ws_layout(a->B, a->L, a->H, &lay);
+  if (lay.qkv > kStaticWorkspaceBytes) {
+    char d[128];
+    snprintf(d, sizeof d, "B=%d, L=%d, H=%d need %zu bytes of scratch, the static array holds %zu",
+             a->B, a->L, a->H, lay.qkv, kStaticWorkspaceBytes);
+    return fail(SC_ERR_UNSUPPORTED, "sc_layer_forward_noalloc", d);
+  }
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  char* ws = nullptr;
+  if ((rc = static_workspace(&ws)) != SC_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  // the compacted-row descriptors point at the caller's tensors: never read here
+  TensorMaps maps;
+  const uint16_t* src[3] = {a->Q, a->K, a->V};
+  uint16_t* const cmp[3] = {const_cast<uint16_t*>(a->Q), const_cast<uint16_t*>(a->K),
+                            const_cast<uint16_t*>(a->V)};
+  const long long tokens = static_cast<long long>(a->B) * a->L;
+  if (!encode_maps(&maps, src, tokens, cmp, tokens, a->H)) return SC_ERR_CUDA;
+  // the array keeps the previous call's contents: clear the status word and
+  // the counters, which must start at zero
+  cudaError_t e = cudaMemsetAsync(ws + lay.status, 0, sizeof(int), st);
+  if (e != cudaSuccess) return fail_cuda("static workspace status reset", e);
+  if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
+
+  LayerParams p{};
+  p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
+  p.T = (a->L + kTile - 1) / kTile;
+  p.src_base = 0;
+  p.len = a->len;
+  p.pos = a->pos;
+  p.O = a->O;
+  p.scores = a->scores;
+  p.pos_out = a->pos_out;
+  p.len_out = a->len_out;
+  p.alpha = a->alpha;
+  p.theta = a->theta;
+  fill_workspace(&p, ws, lay, 0);
+
+  PrepParams pp{};
+  pp.B = a->B; pp.L = a->L;
+  pp.pos_in = a->pos;
+  pp.len_in = a->len;
+  pp.gcur = const_cast<int32_t*>(p.gcur);
+  pp.ng = const_cast<int32_t*>(p.ng);
+  pp.ident = const_cast<int32_t*>(p.ident);
+  pp.n_global = a->n_global;
+  for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
+  if ((e = launch_prep(pp, st)) != cudaSuccess) return fail_cuda("launch prep kernel", e);
+  if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
+  if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
+  return SC_OK;
+}

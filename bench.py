@@ -102,6 +102,25 @@ def layer_work(wl, inp, pos, lens):
 
 
 # ---------------------------------------------------------------------------
+# multi-rank aggregation (replicas: no collective on the data path)
+# ---------------------------------------------------------------------------
+def max_over_ranks(value: float, device=None) -> float:
+    """The slowest rank's time: all-reduce MAX (a no-op without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, units_per_step_per_rank: int, ms_per_step: float) -> float:
+    """Units processed by all ranks per second, timed by the slowest rank."""
+    return world * units_per_step_per_rank / (ms_per_step * 1e-3)
+
+
+# ---------------------------------------------------------------------------
 # clocks during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
@@ -251,6 +270,22 @@ def run_native(args, wl):
     if rc != 0:
         raise SystemExit("device status after warm-up: %s" % sc.status_string(rc))
 
+    # one step captured as a CUDA graph (the library's launches, descriptors
+    # encoded at capture time), replayed for the timed steps
+    graph = None
+    if not args.no_graph:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            step()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=side):
+                step()
+        torch.cuda.current_stream().wait_stream(side)
+        for _ in range(max(3, args.warmup)):
+            graph.replay()
+        torch.cuda.synchronize()
+
     # ---- timed region: K steps, inputs resident
     stream = torch.cuda.current_stream()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -258,19 +293,21 @@ def run_native(args, wl):
         barrier()
         t0.record(stream)
         for _ in range(args.steps):
-            step()
+            if graph is not None:
+                graph.replay()
+            else:
+                step()
         t1.record(stream)
         barrier()
-    ms = t0.elapsed_time(t1)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    rc = sc.workspace_status(ws)
+    if rc != 0:
+        raise SystemExit("device status after the timed steps: %s" % sc.status_string(rc))
+    ms = max_over_ranks(t0.elapsed_time(t1), dev)
     ms_per_step = ms / args.steps
     lens = out["len"].cpu().numpy()
     pos = out["pos"].cpu().numpy()
     kept_per_step = int(lens[:wl.n_layers].sum())
-    value = world * kept_per_step / (ms_per_step * 1e-3)
+    value = whole_job_rate(world, kept_per_step, ms_per_step)
 
     # ---- per-kernel times on the launching stream (same steps, events between kernels)
     nev = 2 + 3 * wl.n_layers
@@ -344,12 +381,8 @@ def run_native(args, wl):
             hout[k].copy_(out[k], non_blocking=True)
     t1.record(stream)
     barrier()
-    e2e_ms = t0.elapsed_time(t1) / e2e_steps
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e = {"value": world * kept_per_step / (e2e_ms * 1e-3), "unit": UNIT,
+    e2e_ms = max_over_ranks(t0.elapsed_time(t1) / e2e_steps, dev)
+    e2e = {"value": whole_job_rate(world, kept_per_step, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
            "ms_per_step": e2e_ms}
 
@@ -360,6 +393,7 @@ def run_native(args, wl):
             "config": {"workload": wl.describe(), "n_layers": wl.n_layers, "batch": wl.B,
                        "seq_len": wl.L, "heads": wl.H, "head_dim": wl.d, "window": wl.w,
                        "globals": len(gpos), "parallelism": "replicas" if world > 1 else "single",
+                       "cuda_graph": graph is not None,
                        "l2": "inputs of one step (%.0f MB) exceed L2; no flush" % (
                            3 * inp["Q"].nbytes / 1e6),
                        "kept_tokens_per_step": kept_per_step,
@@ -394,6 +428,9 @@ def main():
     ap.add_argument("--ref-layers", type=int, default=2,
                     help="layers of one sequence per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="call the library directly for each timed step instead of replaying "
+                         "a captured CUDA graph")
     args = ap.parse_args()
     wl = pick_workload(args.workload)
     if args.impl == "reference":

@@ -58,8 +58,8 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->status = take(kAlign);
   w->lse = take(sizeof(float) * B * H * (size_t)L);
   w->acc = take(sizeof(float) * B * H * (size_t)L);
-  w->gpart = take(sizeof(float) * B * H * T * kMaxGlobal);
-  w->gstat = take(sizeof(float) * B * H * T * kMaxGlobal * 2);
+  w->gpart = take(sizeof(float) * B * H * T * 4 * kMaxGlobal);
+  w->gstat = take(sizeof(float) * B * H * T * 4 * kMaxGlobal * 2);
   w->og = take(sizeof(float) * B * H * kMaxGlobal * kHeadDim);
   w->keep = take(sizeof(uint8_t) * B * (size_t)L);
   w->cnt_tile = take(sizeof(uint32_t) * B * T);

@@ -55,8 +55,10 @@ struct LayerParams {
   // workspace
   float* lse;            // [B][H][L] per-row log2-sum-exp2 (+inf for global rows)
   float* acc;            // [B][H][L] per-head column sums: band rows + global rows
-  float* gpart;          // [B][H][T][kMaxGlobal] column sums of global keys over far rows
-  float* gstat;          // [B][H][T][kMaxGlobal][2] (max, sum) of global rows per key tile
+  float* gpart;          // [B][H][T][4][kMaxGlobal] column sums of global keys over far rows,
+                         //   per (query tile, 32-row warp slice)
+  float* gstat;          // [B][H][T][4][kMaxGlobal][2] (max, sum) of global rows per
+                         //   (key tile, 32-key warp slice)
   float* og;             // [B][H][kMaxGlobal][64] fp32 outputs of global rows
   uint8_t* keep;         // [B][L]
   uint32_t* cnt_tile;    // [B][T]

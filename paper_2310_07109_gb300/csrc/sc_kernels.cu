@@ -158,15 +158,10 @@ struct RowsSmem {
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
-  float gm[2][kMaxGlobal];
-  float red2[2][8][kMaxGlobal];
 };
 
-// dynamic shared memory: two Q tiles, the K/V ring, the global rows, and one
-// [128][17] fp32 reduction scratch per warpgroup
-constexpr uint32_t kRedBytes = 128 * 17 * 4;
-constexpr uint32_t kRowsDyn =
-    kTileBytes * (2 + 2 * kStages) + 3 * kGTileBytes + 2 * kRedBytes + 1024;
+// dynamic shared memory: two Q tiles, the K/V ring and the global rows
+constexpr uint32_t kRowsDyn = kTileBytes * (2 + 2 * kStages) + 3 * kGTileBytes + 1024;
 
 // Issue P V for one 128-key tile: P (A) from tensor memory, V (B) MN-major smem.
 __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint32_t v_smem,
@@ -175,36 +170,6 @@ __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint
   for (int k = 0; k < ksteps; ++k)
     umma_bf16_ts(d_tmem, p_tmem + 8 * k, sdesc_sw128(v_smem + k * 2048), idesc,
                  (accumulate || k > 0) ? 1u : 0u);
-}
-
-__device__ __forceinline__ void wg_sync(int X) {
-  asm volatile("bar.sync %0, 128;" ::"r"(1 + X) : "memory");
-}
-
-// Column reduction of a [128 rows][16] block held one row per thread
-// (red[r * 17 + g]): eight partial results per g, then the combine.
-template <bool kMax>
-__device__ __forceinline__ float reduce_cols16(const float* red, float (*red2)[kMaxGlobal], int X,
-                                               int r) {
-  wg_sync(X);
-  {
-    const int g = r & 15, part = r >> 4;
-    float v = red[(16 * part) * 17 + g];
-#pragma unroll
-    for (int k = 1; k < 16; ++k) {
-      const float u = red[(16 * part + k) * 17 + g];
-      v = kMax ? fmaxf(v, u) : v + u;
-    }
-    red2[part][g] = v;
-  }
-  wg_sync(X);
-  float v = 0.f;
-  if (r < kMaxGlobal) {
-    v = red2[0][r];
-#pragma unroll
-    for (int k = 1; k < 8; ++k) v = kMax ? fmaxf(v, red2[k][r]) : v + red2[k][r];
-  }
-  return v;
 }
 
 __global__ void __launch_bounds__(kRowsThreads, 1)
@@ -227,7 +192,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   uint8_t* KG = Vs + kStages * kTileBytes;
   uint8_t* VG = KG + kGTileBytes;
   uint8_t* QG = VG + kGTileBytes;
-  float* red_all = reinterpret_cast<float*>(QG + kGTileBytes);
   __shared__ RowsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -309,16 +273,21 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     if (lane == 0) {
       const uint32_t q_a = smem_u32(Qs), k_a = smem_u32(Ks), v_a = smem_u32(Vs);
       const int nX = hasB ? 2 : 1;
-      // remaining users (warpgroups) of each key tile's K and V
-      int kuse[kPairTiles], vuse[kPairTiles];
+      // remaining users (warpgroups) of each key tile's K and of its V, two
+      // bits per tile (kept in registers)
+      uint32_t kuse = 0;
       for (int k = 0; k < kPairTiles; ++k) {
         const int a = kt_lo + k;
-        const int u = (a >= klo[0] && a <= khi[0]) + (hasB && a >= klo[1] && a <= khi[1]);
-        kuse[k] = u;
-        vuse[k] = u;
+        const uint32_t u = (a >= klo[0] && a <= khi[0]) + (hasB && a >= klo[1] && a <= khi[1]);
+        kuse |= u << (2 * k);
       }
-      int cur[2] = {klo[0], klo[1]};   // next key tile of each warpgroup
-      int pu[2] = {0, 0};              // completed pready phases waited for
+      uint32_t vuse = kuse;
+      int cur0 = klo[0], cur1 = klo[1];   // next key tile of each warpgroup
+      int pu0 = 0, pu1 = 0;               // completed pready phases waited for
+      auto release = [&](uint32_t& use, int k) -> bool {   // true when the last user is done
+        use -= 1u << (2 * k);
+        return ((use >> (2 * k)) & 3u) == 0u;
+      };
       bool ok = mbar_wait(&sm.bar_q, 0, abort_flag);
       if (ok) {
         tc_fence_after();
@@ -338,7 +307,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
           mma_qk(tm + col_sgt(X), k_a + s * kTileBytes, smem_u32(QG), 16);
           umma_commit(&sm.bar_sgt[X]);
         }
-        if (--kuse[k] == 0) umma_commit(&sm.bar_kempty[s]);
+        if (release(kuse, k)) umma_commit(&sm.bar_kempty[s]);
         umma_commit(&sm.bar_sfull[X]);
         return true;
       };
@@ -346,30 +315,33 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       // S also covers it (the softmax may rescale O as soon as S is ready)
       for (int X = 0; ok && X < nX; ++X) {
         if (ngp) {
-          if (!(ok = mbar_wait(&sm.bar_pready[X], pu[X] & 1, abort_flag))) break;
-          ++pu[X];
+          if (!(ok = mbar_wait(&sm.bar_pready[X], (X ? pu1 : pu0) & 1, abort_flag))) break;
+          (X ? pu1 : pu0) += 1;
           tc_fence_after();
           mma_pv_ts(tm + col_o(X), tm + col_pg(X), smem_u32(VG), kMaxGlobal / 16, false);
         }
-        ok = issue_s(X, cur[X]);
+        ok = issue_s(X, X ? cur1 : cur0);
       }
       // steady state: P V of the current tile, then S of the next, per warpgroup
       bool more = true;
       while (ok && more) {
         more = false;
         for (int X = 0; ok && X < nX; ++X) {
-          if (cur[X] > khi[X]) continue;
-          const int a = cur[X], k = a - kt_lo, s = k % kStages;
-          if (!(ok = mbar_wait(&sm.bar_pready[X], pu[X] & 1, abort_flag))) break;
-          ++pu[X];
+          int& cur = X ? cur1 : cur0;
+          int& pu = X ? pu1 : pu0;
+          const int khiX = X ? khi[1] : khi[0], kloX = X ? klo[1] : klo[0];
+          if (cur > khiX) continue;
+          const int a = cur, k = a - kt_lo, s = k % kStages;
+          if (!(ok = mbar_wait(&sm.bar_pready[X], pu & 1, abort_flag))) break;
+          ++pu;
           if (!(ok = mbar_wait(&sm.bar_vfull[s], (k / kStages) & 1, abort_flag))) break;
           tc_fence_after();
           mma_pv_ts(tm + col_o(X), tm + col_sp(X), v_a + s * kTileBytes, kTile / 16,
-                    ngp > 0 || a > klo[X]);
-          if (--vuse[k] == 0) umma_commit(&sm.bar_vempty[s]);
-          cur[X] = a + 1;
-          if (cur[X] <= khi[X]) {
-            if (!(ok = issue_s(X, cur[X]))) break;
+                    ngp > 0 || a > kloX);
+          if (release(vuse, k)) umma_commit(&sm.bar_vempty[s]);
+          cur = a + 1;
+          if (cur <= khiX) {
+            if (!(ok = issue_s(X, cur))) break;
             more = true;
           } else {
             umma_commit(&sm.bar_done[X]);
@@ -383,6 +355,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   } else {
     // ------------------------------------------------------------- softmax
     const int X = warp >> 2;              // warpgroup = query tile of the pair
+    const int kloX = X ? klo[1] : klo[0], khiX = X ? khi[1] : khi[0];
     const int wq = warp & 3;              // TMEM lane quarter of this warp
     const int r = tid & 127;              // row inside the tile == TMEM lane
     const int qt = 2 * pr + X;
@@ -392,7 +365,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
     const uint32_t tSP = tm + col_sp(X), tO = tm + col_o(X), tSG = tm + col_sg(X),
                    tPG = tm + col_pg(X), tSGt = tm + col_sgt(X);
-    float* red = red_all + X * (128 * 17);
     bool row_global = false;
     for (int g = 0; g < ng; ++g) row_global |= (sm.gc[g] == i);
     const bool valid = (i < n) && !row_global;
@@ -448,8 +420,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     // tile's partial sums and the already-stored first half of P are rescaled
     // exactly.  P values therefore stay below 2^8.
     float x[64];
-    for (int t = 0; ok && t <= khi[X] - klo[X]; ++t) {
-      const int j0 = (klo[X] + t) * kTile;
+    for (int t = 0; ok && t <= khiX - kloX; ++t) {
+      const int j0 = (kloX + t) * kTile;
       // 32-column chunks of this tile that intersect the warp's band
       const int clo = max(0, wlo - j0), chi = min(kTile - 1, whi - j0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
@@ -492,31 +464,36 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 #pragma unroll
             for (int k = 0; k < 4; ++k) ps[k] *= f;
           }
-          float o[32];
+          // small pieces keep the register footprint next to x[] low
+          float o[8];
           if (o_written) {
-#pragma unroll
-            for (int c = 0; c < 64; c += 32) {
-              tmem_ld32(tO + lane_off + c, o);
+#pragma unroll 1
+            for (int c = 0; c < 64; c += 8) {
+              tmem_ld8(tO + lane_off + c, o);
               tmem_ld_wait();
 #pragma unroll
-              for (int k = 0; k < 32; ++k) o[k] *= f;
-              tmem_st32(tO + lane_off + c, o);
+              for (int k = 0; k < 8; ++k) o[k] *= f;
+              tmem_st8(tO + lane_off + c, reinterpret_cast<const uint32_t*>(o));
               tmem_st_wait();   // o is reused
             }
           }
           if (hf == 1) {
             // the first half of this tile's P, already stored: 32 columns of bf16 pairs
             tmem_st_wait();
-            tmem_ld32(tSP + lane_off, o);
-            tmem_ld_wait();
+#pragma unroll 1
+            for (int c = 0; c < 32; c += 8) {
+              tmem_ld8(tSP + lane_off + c, o);
+              tmem_ld_wait();
 #pragma unroll
-            for (int k = 0; k < 32; ++k) {
-              const uint32_t w = __float_as_uint(o[k]);
-              const float lo16 = __uint_as_float(w << 16) * f;
-              const float hi16 = __uint_as_float(w & 0xffff0000u) * f;
-              o[k] = __uint_as_float(pack_bf16x2(lo16, hi16));
+              for (int k = 0; k < 8; ++k) {
+                const uint32_t w = __float_as_uint(o[k]);
+                const float lo16 = __uint_as_float(w << 16) * f;
+                const float hi16 = __uint_as_float(w & 0xffff0000u) * f;
+                o[k] = __uint_as_float(pack_bf16x2(lo16, hi16));
+              }
+              tmem_st8(tSP + lane_off + c, reinterpret_cast<const uint32_t*>(o));
+              tmem_st_wait();
             }
-            tmem_st32(tSP + lane_off, o);
           }
         }
         const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
@@ -574,6 +551,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     if (active && i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
 
     if (active && ngp) {
+      // Per-warp partial results (32 rows / 32 keys each), reduced with
+      // shuffles and merged later in a fixed order: no barrier here.
+      const size_t slot0 =
+          (((static_cast<size_t>(b) * p.H + h) * p.T + qt) * 4 + wq) * kMaxGlobal;
       // far-row column sums of the global keys: rows outside the key's band
       if (ok) {
         tmem_ld16(tSG + lane_off, xg);
@@ -581,11 +562,12 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       }
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        const bool use = ok && valid && (g < ng) && abs(i - sm.gc[g]) > p.w;
-        red[r * 17 + g] = use ? ex2(fmaf(xg[g], kLogitScale2, -lse)) : 0.f;
+        if (g >= ng) break;   // warp-uniform
+        const bool use = ok && valid && abs(i - sm.gc[g]) > p.w;
+        const float v = warp_sum(use ? ex2(fmaf(xg[g], kLogitScale2, -lse)) : 0.f);
+        if (lane == g) p.gpart[slot0 + g] = v;
       }
-      const float gpart = reduce_cols16<false>(red, sm.red2[X], X, r);
-      // (max, sum) of each global query over this tile's keys j = 128 qt + r
+      // (max, sum) of each global query over this warp's keys j = 128 qt + r
       const bool ok2 = ok && warp_wait(&sm.bar_sgt[X], 0, abort_flag);
       if (ok2) {
         tc_fence_after();
@@ -595,23 +577,14 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       const bool key_ok = ok2 && (r0 + r < n);
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        xg[g] = key_ok ? xg[g] * kLogitScale2 : -INFINITY;
-        red[r * 17 + g] = xg[g];
-      }
-      const float gmax = reduce_cols16<true>(red, sm.red2[X], X, r);
-      if (r < kMaxGlobal) sm.gm[X][r] = gmax;
-      wg_sync(X);
-#pragma unroll
-      for (int g = 0; g < kMaxGlobal; ++g) {
-        const float m = sm.gm[X][g];
-        red[r * 17 + g] = (key_ok && m != -INFINITY) ? ex2(xg[g] - m) : 0.f;
-      }
-      const float gsum = reduce_cols16<false>(red, sm.red2[X], X, r);
-      if (r < kMaxGlobal) {
-        const size_t slot = ((static_cast<size_t>(b) * p.H + h) * p.T + qt) * kMaxGlobal + r;
-        p.gpart[slot] = gpart;
-        p.gstat[2 * slot] = gmax;
-        p.gstat[2 * slot + 1] = gsum;
+        if (g >= ng) break;   // warp-uniform
+        const float y = key_ok ? xg[g] * kLogitScale2 : -INFINITY;
+        const float m = warp_max(y);
+        const float sum = warp_sum(m == -INFINITY ? 0.f : ex2(y - m));
+        if (lane == g) {
+          p.gstat[2 * (slot0 + g)] = m;
+          p.gstat[2 * (slot0 + g) + 1] = sum;
+        }
       }
       if (qt == 0) {
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
@@ -770,7 +743,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
         const int s = q % kStages, a = qt_lo + q;
         if (!(ok = mbar_wait(&sm.bar_qfull[s], (q / kStages) & 1, abort_flag))) break;
         for (int X = 0; ok && X < nX; ++X) {
-          if (a < qlo[X] || a > qhi[X]) continue;
+          if (a < (X ? qlo[1] : qlo[0]) || a > (X ? qhi[1] : qhi[0])) continue;
           if (su[X] > 0 && !(ok = mbar_wait(&sm.bar_sfree[X], (su[X] - 1) & 1, abort_flag))) break;
           tc_fence_after();
           mma_qk(tm + 128 * X, k_a + X * kTileBytes, q_a + s * kTileBytes, 128);
@@ -793,6 +766,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     __syncwarp();
   } else {
     const int X = warp >> 2, wq = warp & 3;
+    const int qloX = X ? qlo[1] : qlo[0], qhiX = X ? qhi[1] : qhi[0];
     const int r = tid & 127;
     const int kt = 2 * pr + X;
     const int j0 = kt * kTile;
@@ -805,23 +779,31 @@ __global__ void __launch_bounds__(kColsThreads, 1)
       const int row = qt_lo * kTile + k;
       sm.lse[k] = row < n ? __ldcg(lse_src + row) : INFINITY;
     }
-    if (ngp && warp == 0) {
-      // merge the per-tile (max, sum) of every global row into its LSE; lane =
-      // query tile, all loads issued before any reduction
-      float m[kMaxGlobal], sm_[kMaxGlobal];
-      const size_t base_slot = ((static_cast<size_t>(b) * p.H + h) * p.T + lane) * kMaxGlobal;
+    if (ngp) {
+      // merge the per-(key tile, warp slice) (max, sum) of every global row
+      // into its LSE: warp w takes global rows w and w + 8; lane k takes
+      // entries k, k+32, k+64, k+96 of the 4 Tn entries (all loads issued
+      // first), then the warp combines; fixed order throughout
+      const size_t base_slot = (static_cast<size_t>(b) * p.H + h) * p.T * 4 * kMaxGlobal;
 #pragma unroll
-      for (int g = 0; g < kMaxGlobal; ++g) {
-        const bool use = lane < Tn && g < ng;
-        m[g] = use ? __ldcg(p.gstat + 2 * (base_slot + g)) : -INFINITY;
-        sm_[g] = use ? __ldcg(p.gstat + 2 * (base_slot + g) + 1) : 0.f;
-      }
+      for (int gg = 0; gg < 2; ++gg) {
+        const int g = warp + 8 * gg;
+        if (g >= ng) break;   // warp-uniform
+        float me[4], se[4];
 #pragma unroll
-      for (int g = 0; g < kMaxGlobal; ++g) {
-        const float M = warp_max(m[g]);
-        const float part = (m[g] != -INFINITY) ? sm_[g] * ex2(m[g] - M) : 0.f;
-        const float S = warp_sum(part);
-        if (lane == 0 && g < ng) sm.lse_g[g] = M + lg2(S);
+        for (int k = 0; k < 4; ++k) {
+          const int ent = lane + 32 * k;
+          const bool use = ent < 4 * Tn;
+          me[k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g)) : -INFINITY;
+          se[k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g) + 1) : 0.f;
+        }
+        const float m = fmaxf(fmaxf(me[0], me[1]), fmaxf(me[2], me[3]));
+        float sacc = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) sacc += (me[k] == -INFINITY) ? 0.f : se[k] * ex2(me[k] - m);
+        const float M = warp_max(m);
+        const float S = warp_sum(m == -INFINITY ? 0.f : sacc * ex2(m - M));
+        if (lane == 0) sm.lse_g[g] = M + lg2(S);
       }
     }
     asm volatile("bar.sync 3, 256;" ::: "memory");
@@ -832,13 +814,13 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     float acc = 0.f;
     bool ok = active;
     float x[64];
-    for (int t = 0; ok && t <= qhi[X] - qlo[X]; ++t) {
-      const int i0 = (qlo[X] + t) * kTile;            // first query row of this tile
+    for (int t = 0; ok && t <= qhiX - qloX; ++t) {
+      const int i0 = (qloX + t) * kTile;            // first query row of this tile
       const int clo = max(0, wlo - i0), chi = min(kTile - 1, whi - i0);
       const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
       if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
-      const float* lw = sm.lse + (qlo[X] + t - qt_lo) * kTile;
+      const float* lw = sm.lse + (qloX + t - qt_lo) * kTile;
       const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
       float ps[8];
 #pragma unroll
@@ -861,18 +843,22 @@ __global__ void __launch_bounds__(kColsThreads, 1)
         for (int c2 = 0; c2 < 2; ++c2) {
           const int ch = 2 * hf + c2;
           if (ch < ch_lo || ch > ch_hi) continue;
-          const bool full = __all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31);
+          if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+            // edge chunk: rows outside this key's band contribute nothing
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const int c = 32 * ch + k;
+              x[32 * c2 + k] = (c >= a && c <= e) ? x[32 * c2 + k] : -INFINITY;
+            }
+          }
 #pragma unroll
           for (int k = 0; k < 32; k += 4) {
             const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
-            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
             const int u = (k >> 2) & 1;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const int c = 32 * ch + k + q;
-              const float v = ex2(fmaf(x[32 * c2 + k + q], kLogitScale2, -lv[q]));
-              ps[4 * u + q] += (full || (c >= a && c <= e)) ? v : 0.f;
-            }
+            ps[4 * u + 0] += ex2(fmaf(x[32 * c2 + k + 0], kLogitScale2, -l4.x));
+            ps[4 * u + 1] += ex2(fmaf(x[32 * c2 + k + 1], kLogitScale2, -l4.y));
+            ps[4 * u + 2] += ex2(fmaf(x[32 * c2 + k + 2], kLogitScale2, -l4.z));
+            ps[4 * u + 3] += ex2(fmaf(x[32 * c2 + k + 3], kLogitScale2, -l4.w));
           }
         }
       }
@@ -947,11 +933,11 @@ __global__ void __launch_bounds__(kColsThreads, 1)
       const int cg = sm.gc[g];
       float v = 0.f;
       if (cg >= j0 && cg < jn) {
-        const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * kMaxGlobal + g;
+        const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * 4 * kMaxGlobal + g;
 #pragma unroll 4
-        for (int k = lane; k < p.H * Tn; k += 32) {
-          const int hh = k / Tn, q = k - hh * Tn;
-          v += __ldcg(gp + (static_cast<size_t>(hh) * p.T + q) * kMaxGlobal);
+        for (int k = lane; k < p.H * Tn * 4; k += 32) {
+          const int hh = k / (Tn * 4), q4 = k - hh * (Tn * 4);   // q4 = 4 * tile + warp
+          v += __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal);
         }
         v = warp_sum(v);
       }
@@ -1049,9 +1035,11 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
 // ---------------------------------------------------------------------------
 // gather kernel: the next layer's Q, K, V rows of the kept tokens, compacted
 // ---------------------------------------------------------------------------
-constexpr int kGatherTokens = 32;
+constexpr int kGatherTokens = 8;
 constexpr int kGatherThreads = 256;
 
+// 8 tokens x 3 tensors per CTA; with H = 12 each thread moves at most nine
+// 16-byte vectors, all loads issued before any store.
 __global__ void __launch_bounds__(kGatherThreads)
     sc_gather_kernel(const GatherParams g) {
   const int b = blockIdx.y;
@@ -1059,21 +1047,32 @@ __global__ void __launch_bounds__(kGatherThreads)
   const int c0 = blockIdx.x * kGatherTokens;
   if (__ldg(g.ident + b) != 0 || c0 >= n) return;
   const int cnt = min(kGatherTokens, n - c0);
-  __shared__ long long src_tok[kGatherTokens];
-  if (threadIdx.x < cnt)
-    src_tok[threadIdx.x] =
-        g.src_base + static_cast<long long>(b) * g.L + __ldg(g.pos + static_cast<size_t>(b) * g.L + c0 + threadIdx.x);
-  __syncthreads();
   const int vec = g.H * kHeadDim / 8;  // 16-byte vectors per token row
+  const int total = cnt * vec;
   const long long dst_tok0 = static_cast<long long>(b) * g.L + c0;
-  for (int t = 0; t < 3; ++t) {
-    const uint4* src = reinterpret_cast<const uint4*>(g.src[t]);
-    uint4* dst = reinterpret_cast<uint4*>(g.dst[t]);
-#pragma unroll 4
-    for (int k = threadIdx.x; k < cnt * vec; k += kGatherThreads) {
-      const int tk = k / vec, v = k - tk * vec;
-      dst[(dst_tok0 + tk) * vec + v] = __ldg(src + src_tok[tk] * vec + v);
+  const long long src_tok0 = g.src_base + static_cast<long long>(b) * g.L;
+  constexpr int kPer = 4;   // vectors per thread and tensor per round
+  for (int k0 = threadIdx.x; k0 < total; k0 += kGatherThreads * kPer) {
+    uint4 v[3][kPer];
+    long long so[kPer], doff[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int k = k0 + u * kGatherThreads;
+      const int tk = k / vec, e = k - tk * vec;
+      so[u] = k < total ? (src_tok0 + __ldg(g.pos + static_cast<size_t>(b) * g.L + c0 + tk)) * vec + e
+                        : -1;
+      doff[u] = (dst_tok0 + tk) * vec + e;
     }
+#pragma unroll
+    for (int t = 0; t < 3; ++t)
+#pragma unroll
+      for (int u = 0; u < kPer; ++u)
+        if (so[u] >= 0) v[t][u] = __ldg(reinterpret_cast<const uint4*>(g.src[t]) + so[u]);
+#pragma unroll
+    for (int t = 0; t < 3; ++t)
+#pragma unroll
+      for (int u = 0; u < kPer; ++u)
+        if (so[u] >= 0) reinterpret_cast<uint4*>(g.dst[t])[doff[u]] = v[t][u];
   }
 }
 

@@ -310,7 +310,7 @@ def run_native(args, wl):
     value = whole_job_rate(world, kept_per_step, ms_per_step)
 
     # ---- per-kernel times on the launching stream (same steps, events between kernels)
-    nev = 2 + 3 * wl.n_layers
+    nev = 3 + 3 * wl.n_layers
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(nev)]
     for e in evs:
         e.record(stream)
@@ -319,6 +319,7 @@ def run_native(args, wl):
     cols_ms = np.zeros(wl.n_layers)
     gath_ms = np.zeros(wl.n_layers)
     prep_ms = 0.0
+    tail_ms = 0.0
     prof_steps = max(1, args.steps)
     for _ in range(prof_steps):
         step(evs)
@@ -328,7 +329,9 @@ def run_native(args, wl):
             rows_ms[l] += evs[1 + 3 * l].elapsed_time(evs[2 + 3 * l])
             cols_ms[l] += evs[2 + 3 * l].elapsed_time(evs[3 + 3 * l])
             gath_ms[l] += evs[3 + 3 * l].elapsed_time(evs[4 + 3 * l])
+        tail_ms += evs[1 + 3 * wl.n_layers].elapsed_time(evs[2 + 3 * wl.n_layers])
     rows_ms /= prof_steps
+    tail_ms /= prof_steps
     cols_ms /= prof_steps
     gath_ms /= prof_steps
     prep_ms /= prof_steps
@@ -338,7 +341,7 @@ def run_native(args, wl):
     bw = peaks["hbm_gbs"] * 1e9
     fl = peaks["bf16_tflops"] * 1e12
     t_roof = sum(max(Bb / bw, Ff / fl) for Bb, Ff in work)
-    t_meas = float((rows_ms + cols_ms).sum()) * 1e-3
+    t_meas = (float((rows_ms + cols_ms).sum()) + tail_ms) * 1e-3
     bytes_alg = sum(Bb for Bb, _ in work)
     flops_alg = sum(Ff for _, Ff in work)
     hbm_bound = sum(Bb / bw for Bb, _ in work) >= sum(Ff / fl for _, Ff in work)
@@ -353,15 +356,17 @@ def run_native(args, wl):
         "frac": t_roof / t_meas,
         "traffic": None,
         "peak_source": peak_src,
-        "scope": "sc_rows_kernel + sc_cols_kernel of all layers of one step (the fused "
-                 "sparse-attention + LTP layer); algorithmic bytes 6152 B per token-layer, "
-                 "flops 3072 per allowed (query, key) pair; frac = sum_l max(F_l/peak_bf16, "
-                 "B_l/peak_hbm) / measured kernel time",
-        "layer0_frac": max(l0[0] / bw, l0[1] / fl) / t_l0,
+        "scope": "the attention + pruning kernels of one step: sc_rows_kernel + sc_cols_kernel "
+                 "of the layers run per layer, plus sc_tail_kernel (the layers of sequences "
+                 "with <= 256 tokens left, one launch); algorithmic bytes 6152 B per "
+                 "token-layer, flops 3072 per allowed (query, key) pair; frac = sum_l "
+                 "max(F_l/peak_bf16, B_l/peak_hbm) / measured kernel time",
+        "layer0_frac": max(l0[0] / bw, l0[1] / fl) / t_l0 if t_l0 > 1e-6 else None,
         "kernel_ms_per_step": {"sc_rows_kernel": float(rows_ms.sum()),
                                "sc_cols_kernel": float(cols_ms.sum()),
                                "sc_gather_kernel": float(gath_ms.sum()),
-                               "sc_prep_kernel": prep_ms},
+                               "sc_prep_kernel": prep_ms,
+                               "sc_tail_kernel": tail_ms},
         "rows_ms_per_layer": [round(float(x), 5) for x in rows_ms],
         "cols_ms_per_layer": [round(float(x), 5) for x in cols_ms],
     }
@@ -402,8 +407,8 @@ def run_native(args, wl):
                                     lens[:wl.n_layers + 1].sum(axis=1) / max(1, lens[0].sum())]},
             "roofline": roofline,
             "e2e": e2e,
-            "gpu_launches": args.steps * (1 + 3 * wl.n_layers - 1
-                                          + (1 if inp["pad_mask"] is not None else 0)),
+            "gpu_launches": args.steps * sc.stack_launch_count(
+                wl.n_layers, wl.B, wl.L, wl.H, wl.w, gpos, inp["pad_mask"] is not None),
             "clocks": clocks.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle

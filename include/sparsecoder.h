@@ -117,7 +117,11 @@ typedef struct {
  * pos        int32 [n_layers+1][B][L] out: pos[0] = real tokens after padding
  *            removal, pos[l+1] = survivors of layer l.
  * len        int32 [n_layers+1][B] out.
+ * flags      0, or SC_STACK_NO_TAIL: run every layer of every sequence through
+ *            the per-layer kernels (see sc_stack_forward).
  */
+#define SC_STACK_NO_TAIL 1
+
 typedef struct {
   int n_layers, B, L, H, w;
   const uint16_t* Q;
@@ -131,6 +135,7 @@ typedef struct {
   float* scores;
   int32_t* pos;
   int32_t* len;
+  int flags;
 } sc_stack_args;
 
 /*
@@ -164,7 +169,17 @@ int sc_layer_forward(const sc_layer_args* args, void* workspace, size_t workspac
                      void* stream);
 
 /* The pruned stack (Fig. "sparsecoder": sparse attention with layer-wise
- * token pruning, 12 layers in the paper's encoder).  Errors: see sc_status. */
+ * token pruning, 12 layers in the paper's encoder).  Errors: see sc_status.
+ *
+ * Execution: a sequence runs layer by layer through the per-layer kernels
+ * while it has more than 256 current tokens; from the first layer at which it
+ * has at most 256 (after padding removal or after a layer's pruning) its
+ * remaining layers run in one cluster kernel launched once at the end of the
+ * call (one thread-block cluster of H CTAs per sequence, when the device can
+ * schedule clusters of H <= 16 CTAs and n_layers <= 64).  The hand-over is
+ * decided on the device: the call never waits for the GPU and can be captured
+ * in a CUDA graph.  Results are the same function of the inputs either way
+ * (within the stated tolerances). */
 int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
                      void* stream);
 
@@ -173,10 +188,18 @@ int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspac
  * events[0] before the first launch, events[1] after the padding-removal
  * kernel, then for layer l: events[2+3l] after its rows kernel, events[3+3l]
  * after its cols kernel (scores, threshold, compaction) and events[4+3l] after
- * the gather of the next layer's rows.  n_events >= 2 + 3 * n_layers.  The
- * events are caller-owned. */
+ * the gather of the next layer's rows, and events[2+3*n_layers] after the
+ * cluster kernel of the short sequences.  Events of kernels that a call does
+ * not launch are recorded anyway (back to back).  n_events >= 3 + 3 * n_layers.
+ * The events are caller-owned. */
 int sc_stack_forward_profiled(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
                               void* stream, void** events, int n_events);
+
+/* Number of kernels that sc_stack_forward launches for these arguments (on the
+ * current device), in *count.  Only the sizes, n_layers, pad_mask (NULL or
+ * not) and the global list are read; no pointer is dereferenced and nothing is
+ * launched.  Errors: see sc_status (SC_ERR_CUDA without a usable device). */
+int sc_stack_launch_count(const sc_stack_args* args, int* count);
 
 /* Synchronises `stream`, returns SC_ERR_TIMEOUT if any kernel since the last
  * query recorded an expired wait (else SC_OK, or SC_ERR_CUDA), and clears

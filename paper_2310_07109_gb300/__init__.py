@@ -5,7 +5,7 @@ The Python surface is a thin ctypes binding (``binding``); the arithmetic runs
 in ``libsparsecoder.so`` (``csrc/``), built in-tree by ``build.build_library``.
 """
 from .binding import (SparseCoderError, layer_forward, load, new_workspace, stack_forward,
-                      status_string, workspace_size, workspace_status)
+                      stack_launch_count, status_string, workspace_size, workspace_status)
 
 __all__ = ["SparseCoderError", "layer_forward", "load", "new_workspace", "stack_forward",
-           "status_string", "workspace_size", "workspace_status"]
+           "stack_launch_count", "status_string", "workspace_size", "workspace_status"]

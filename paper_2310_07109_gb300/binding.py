@@ -49,11 +49,13 @@ class StackArgs(ctypes.Structure):
                 ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
                 ("alpha", ctypes.POINTER(ctypes.c_float)),
                 ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
-                ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p)]
+                ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p), ("flags", ctypes.c_int)]
 
+
+SC_STACK_NO_TAIL = 1
 
 EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
-            "sc_stack_forward_profiled",
+            "sc_stack_forward_profiled", "sc_stack_launch_count",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error"]
 
 
@@ -89,6 +91,9 @@ def load(build_if_missing: bool = False):
         lib.sc_stack_forward_profiled.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                                   ctypes.c_size_t, ctypes.c_void_p,
                                                   ctypes.POINTER(ctypes.c_void_p), ctypes.c_int]
+        lib.sc_stack_launch_count.restype = ctypes.c_int
+        lib.sc_stack_launch_count.argtypes = [ctypes.POINTER(StackArgs),
+                                              ctypes.POINTER(ctypes.c_int)]
         lib.sc_workspace_status.restype = ctypes.c_int
         lib.sc_workspace_status.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         lib.sc_status_string.restype = ctypes.c_char_p
@@ -175,13 +180,14 @@ def layer_forward_noalloc(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=
 
 
 def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
-                  stream=None, events=None):
+                  stream=None, events=None, no_tail=False):
     """The pruned layer stack (``sc_stack_forward``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
     pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers].
-    events: optional list of >= 2 + 2 * n_layers torch.cuda.Event(enable_timing=True),
+    events: optional list of >= 3 + 3 * n_layers torch.cuda.Event(enable_timing=True),
     recorded around every kernel on the launching stream (sc_stack_forward_profiled).
+    no_tail: run every layer through the per-layer kernels (SC_STACK_NO_TAIL).
     Returns a dict with O, scores, pos, len (device tensors).
     """
     nl, B, L, H, D = Q.shape
@@ -197,7 +203,8 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
     a = StackArgs(nl, B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(pad_mask),
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
-                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]))
+                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
+                  SC_STACK_NO_TAIL if no_tail else 0)
     if events is None:
         _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
                                        _stream_handle(stream)))
@@ -206,6 +213,19 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
         _check(load().sc_stack_forward_profiled(ctypes.byref(a), _ptr(ws), ws.numel(),
                                                 _stream_handle(stream), handles, len(events)))
     return out
+
+
+def stack_launch_count(n_layers, B, L, H, w, global_pos, has_pad_mask, no_tail=False) -> int:
+    """Kernels one ``stack_forward`` call launches for these sizes on the current device."""
+    garr, ng = _int32_host(global_pos)
+    # only whether pad_mask is NULL matters: a non-null marker is never dereferenced
+    a = StackArgs(int(n_layers), int(B), int(L), int(H), int(w), None, None, None,
+                  16 if has_pad_mask else None,
+                  ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, None, None, None,
+                  None, None, SC_STACK_NO_TAIL if no_tail else 0)
+    cnt = ctypes.c_int(0)
+    _check(load().sc_stack_launch_count(ctypes.byref(a), ctypes.byref(cnt)))
+    return int(cnt.value)
 
 
 def workspace_status(workspace, stream=None) -> int:

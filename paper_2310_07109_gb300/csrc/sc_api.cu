@@ -20,6 +20,9 @@ cudaError_t configure_kernels();
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st);
+cudaError_t configure_tail();
+cudaError_t tail_max_clusters(int H, int* out);
+cudaError_t launch_tail(const TailParams& p, cudaStream_t st);
 }  // namespace sc
 
 namespace {
@@ -43,7 +46,8 @@ int fail_cuda(const char* what, cudaError_t e) {
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
-  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident, qkv, total;
+  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident, tail_from,
+      qkv, total;
 };
 
 bool ws_layout(int B, int L, int H, WsLayout* w) {
@@ -67,6 +71,7 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
   w->ng = take(sizeof(int32_t) * 2 * B);
   w->ident = take(sizeof(int32_t) * 2 * B);
+  w->tail_from = take(sizeof(int32_t) * B);
   // compacted Q, K, V of the current layer (rows of the surviving tokens)
   w->qkv = take(sizeof(uint16_t) * 3 * B * (size_t)L * H * kHeadDim);
   w->total = off;
@@ -154,10 +159,36 @@ int ensure_configured() {
   if (dev < 0 || dev >= 256) return fail(SC_ERR_CUDA, "cudaGetDevice", "device index out of range");
   std::lock_guard<std::mutex> lock(mu);
   if (!done[dev]) {
-    const cudaError_t e = configure_kernels();
+    cudaError_t e = configure_kernels();
+    if (e == cudaSuccess) e = configure_tail();
     if (e != cudaSuccess) return fail_cuda("kernel attributes", e);
     done[dev] = true;
   }
+  return SC_OK;
+}
+
+// Whether the cluster kernel can run with clusters of H CTAs on the current
+// device (cached per device and H; call after ensure_configured()).
+int tail_available(int H, bool* ok) {
+  static std::mutex mu;
+  static signed char state[256][kTailMaxHeads + 1];   // 0 unknown, 1 yes, -1 no
+  *ok = false;
+  if (H < 1 || H > kTailMaxHeads) return SC_OK;
+  int dev = 0;
+  const cudaError_t ge = cudaGetDevice(&dev);
+  if (ge != cudaSuccess) return fail_cuda("cudaGetDevice", ge);
+  if (dev < 0 || dev >= 256) return fail(SC_ERR_CUDA, "cudaGetDevice", "device index out of range");
+  std::lock_guard<std::mutex> lock(mu);
+  if (state[dev][H] == 0) {
+    int clusters = 0;
+    const cudaError_t e = tail_max_clusters(H, &clusters);
+    if (e != cudaSuccess) {
+      cudaGetLastError();   // an unsupported shape is not an error of the call
+      clusters = 0;
+    }
+    state[dev][H] = clusters > 0 ? 1 : -1;
+  }
+  *ok = state[dev][H] > 0;
   return SC_OK;
 }
 
@@ -291,10 +322,25 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   return SC_OK;
 }
 
+// Which kernels a stack call launches: sequences with at most kTailMax tokens
+// left finish in the cluster kernel (when it can run with clusters of H CTAs);
+// with L <= kTailMax every sequence starts there and no per-layer kernel runs.
+static int stack_plan(const sc_stack_args* a, bool* use_tail, bool* per_layer) {
+  const int n_layers = a->n_layers, L = a->L, H = a->H;
+  bool ok = false;
+  if (!(a->flags & SC_STACK_NO_TAIL)) {
+    const int rc = tail_available(H, &ok);
+    if (rc != SC_OK) return rc;
+  }
+  *use_tail = ok && n_layers <= kTailMaxLayers;
+  *per_layer = !*use_tail || L > kTailMax;
+  return SC_OK;
+}
+
 static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
                               void* stream, void** events, int n_events) {
   if (!a) return SC_ERR_INVALID_ARG;
-  if (a->n_layers < 1) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
   if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
@@ -320,10 +366,16 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
 
   const size_t BL = static_cast<size_t>(a->B) * a->L;
+  bool use_tail = false, per_layer = true;
+  if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
+  int32_t* tail_from = use_tail ? reinterpret_cast<int32_t*>(ws + lay.tail_from) : nullptr;
+
   LayerParams p{};
   p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
   p.T = (a->L + kTile - 1) / kTile;
   p.theta = nullptr;
+  p.tail_from = tail_from;
+  p.tail_max = use_tail ? kTailMax : 0;
   fill_workspace(&p, ws, lay, 0);
 
   PrepParams pp{};
@@ -334,6 +386,8 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   pp.gcur = const_cast<int32_t*>(p.gcur);
   pp.ng = const_cast<int32_t*>(p.ng);
   pp.ident = const_cast<int32_t*>(p.ident);
+  pp.tail_from = tail_from;
+  pp.tail_max = p.tail_max;
   pp.n_global = a->n_global;
   for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
   auto mark = [&](int k) {
@@ -348,12 +402,19 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   // gather kernel copies the survivors' rows for every later layer
   GatherParams gp{};
   gp.B = a->B; gp.L = a->L; gp.H = a->H;
+  gp.tail_from = tail_from;
   for (int t = 0; t < 3; ++t) {
     gp.src[t] = src[t];
     gp.dst[t] = cmp[t];
   }
   for (int l = 0; l < a->n_layers; ++l) {
+    if (!per_layer) {
+      if (!mark(2 + 3 * l) || !mark(3 + 3 * l) || !mark(4 + 3 * l))
+        return fail(SC_ERR_CUDA, "event record", "");
+      continue;
+    }
     fill_workspace(&p, ws, lay, l & 1);
+    p.layer = l;
     p.src_base = static_cast<long long>(l) * BLt;
     p.len = a->len + static_cast<size_t>(l) * a->B;
     p.len_out = a->len + static_cast<size_t>(l + 1) * a->B;
@@ -365,6 +426,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     if (l == 0 && a->pad_mask != nullptr) {
       // padding removal may have moved rows: compact layer 0 as well
       gp.src_base = 0;
+      gp.layer = 0;
       gp.len = p.len;
       gp.pos = p.pos;
       gp.ident = p.ident;
@@ -376,6 +438,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     if (!mark(3 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");
     if (l + 1 < a->n_layers) {
       gp.src_base = static_cast<long long>(l + 1) * BLt;
+      gp.layer = l + 1;
       gp.len = p.len_out;
       gp.pos = p.pos_out;
       gp.ident = p.ident_out;
@@ -383,6 +446,22 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     }
     if (!mark(4 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");
   }
+  if (use_tail) {
+    TailParams tp{};
+    tp.n_layers = a->n_layers; tp.B = a->B; tp.L = a->L; tp.H = a->H; tp.w = a->w;
+    tp.tail_from = tail_from;
+    tp.pos = a->pos;
+    tp.len = a->len;
+    tp.O = a->O;
+    tp.scores = a->scores;
+    tp.status = p.status;
+    for (int t = 0; t < 3; ++t) tp.src[t] = src[t];
+    tp.n_global = a->n_global;
+    for (int g = 0; g < a->n_global; ++g) tp.global_pos[g] = a->global_pos[g];
+    for (int l = 0; l < a->n_layers; ++l) tp.alpha[l] = a->alpha[l];
+    if ((e = launch_tail(tp, st)) != cudaSuccess) return fail_cuda("launch tail kernel", e);
+  }
+  if (!mark(2 + 3 * a->n_layers)) return fail(SC_ERR_CUDA, "event record", "");
   return SC_OK;
 }
 
@@ -392,10 +471,25 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
 
 int sc_stack_forward_profiled(const sc_stack_args* a, void* workspace, size_t ws_bytes,
                               void* stream, void** events, int n_events) {
-  if (!a || !events || a->n_layers < 1 || n_events < 2 + 3 * a->n_layers) return SC_ERR_INVALID_ARG;
-  for (int k = 0; k < 2 + 3 * a->n_layers; ++k)
+  if (!a || !events || a->n_layers < 1 || n_events < 3 + 3 * a->n_layers) return SC_ERR_INVALID_ARG;
+  for (int k = 0; k < 3 + 3 * a->n_layers; ++k)
     if (!events[k]) return SC_ERR_INVALID_ARG;
   return stack_forward_impl(a, workspace, ws_bytes, stream, events, n_events);
+}
+
+int sc_stack_launch_count(const sc_stack_args* a, int* count) {
+  if (!a || !count) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  bool use_tail = false, per_layer = true;
+  if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
+  int k = 1;   // padding removal / global lookup
+  if (per_layer) k += (a->pad_mask ? 1 : 0) + 2 * a->n_layers + (a->n_layers - 1);
+  if (use_tail) k += 1;
+  *count = k;
+  return SC_OK;
 }
 
 int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {

@@ -18,6 +18,13 @@ constexpr uint32_t kGTileBytes = kMaxGlobal * kHeadDim * 2;
 
 // status word bits (workspace)
 constexpr int kStatusTimeout = 1;
+constexpr int kStatusInternal = 2;   // an invariant of the launch sequence did not hold
+
+// Sequences with at most kTailMax current tokens run their remaining layers in
+// the cluster kernel (one CTA per head); the per-layer kernels skip them.
+constexpr int kTailMax = 256;
+constexpr int kTailMaxLayers = 64;
+constexpr int kTailMaxHeads = 16;   // largest (non-portable) cluster
 
 // log2(e) / sqrt(64): logits are kept in base-2 units, x = (q.k) * kLogitScale2.
 constexpr float kLogitScale2 = 0.125f * 1.4426950408889634f;
@@ -64,6 +71,12 @@ struct LayerParams {
   uint32_t* cnt_tile;    // [B][T]
   uint32_t* cnt_seq;     // [B]
   int* status;
+  // hand-over to the cluster kernel: sequence b is skipped here once
+  // tail_from[b] <= layer; the finalize of a layer sets tail_from[b] = layer + 1
+  // when at most tail_max tokens survive.  tail_from == nullptr: no hand-over.
+  int32_t* tail_from;    // [B]
+  int layer;
+  int tail_max;
 };
 
 // Copies the rows of the kept tokens (at their original positions) of one
@@ -76,6 +89,8 @@ struct GatherParams {
   const int32_t* ident;        // [B]: sequences whose rows need no copy
   const uint16_t* src[3];      // Q, K, V sources [.., B, L, H, 64]
   uint16_t* dst[3];            // compacted Q, K, V [B][L][H][64]
+  const int32_t* tail_from;    // [B] or nullptr: skip b when tail_from[b] <= layer
+  int layer;                   // the layer whose rows are gathered
 };
 
 struct PrepParams {
@@ -88,8 +103,24 @@ struct PrepParams {
   int32_t* gcur;             // [B][kMaxGlobal]
   int32_t* ng;               // [B]
   int32_t* ident;            // [B]
+  int32_t* tail_from;        // [B] (stack mode with the cluster kernel) or nullptr
+  int tail_max;
   int n_global;
   int global_pos[kMaxGlobal];
+};
+
+struct TailParams {
+  int n_layers, B, L, H, w;
+  const int32_t* tail_from;    // [B] first layer run here (>= n_layers: none)
+  int32_t* pos;                // [n_layers + 1][B][L]
+  int32_t* len;                // [n_layers + 1][B]
+  uint16_t* O;                 // [n_layers][B][L][H][64]
+  float* scores;               // [n_layers][B][L]
+  int* status;
+  const uint16_t* src[3];      // Q, K, V [n_layers][B][L][H][64]
+  int n_global;
+  int global_pos[kMaxGlobal];
+  float alpha[kTailMaxLayers];
 };
 
 }  // namespace sc

@@ -69,6 +69,12 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 
+// Sequence b has been handed to the cluster kernel for this and later layers
+// (its length here may be stale: read nothing else of it).
+__device__ __forceinline__ bool owned_by_tail(const LayerParams& p, int b) {
+  return p.tail_from != nullptr && __ldcg(p.tail_from + b) <= p.layer;
+}
+
 // Which source holds the current rows of sequence b, and the token index of
 // its current row 0 in that source.
 struct RowSource {
@@ -177,6 +183,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   // grid: x = (sequence, head), y = pair of query tiles, so that low tiles (the
   // ones every sequence has) are dispatched first
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
+  if (owned_by_tail(p, b)) return;
   const int n = __ldg(p.len + b);
   if (2 * pr * kTile >= n) return;
   const int ng = min(__ldg(p.ng + b), kMaxGlobal);
@@ -635,6 +642,7 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
 __global__ void __launch_bounds__(kColsThreads, 1)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
+  if (owned_by_tail(p, b)) return;
   const int n = __ldg(p.len + b);
   if (n == 0) {
     if (pr == 0 && h == 0 && threadIdx.x == 0) {
@@ -1026,6 +1034,7 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
       if (sm.gnew[g] >= 0) p.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
     p.ng_out[b] = m;
     p.len_out[b] = total;
+    if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = p.layer + 1;
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
     p.ident_out[b] = (total == 0 || pos_out[total - 1] == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
@@ -1043,6 +1052,7 @@ constexpr int kGatherThreads = 256;
 __global__ void __launch_bounds__(kGatherThreads)
     sc_gather_kernel(const GatherParams g) {
   const int b = blockIdx.y;
+  if (g.tail_from != nullptr && __ldcg(g.tail_from + b) <= g.layer) return;
   const int n = __ldg(g.len + b);
   const int c0 = blockIdx.x * kGatherTokens;
   if (__ldg(g.ident + b) != 0 || c0 >= n) return;
@@ -1139,6 +1149,7 @@ __global__ void __launch_bounds__(kPrepThreads)
     pp.ng[b] = m;
     // single-layer calls read their (already current-order) inputs in place
     pp.ident[b] = (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1) ? 1 : 0;
+    if (pp.tail_from != nullptr) pp.tail_from[b] = n <= pp.tail_max ? 0 : 0x7fffffff;
   }
 }
 

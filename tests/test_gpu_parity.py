@@ -72,12 +72,13 @@ def test_layer_matches_oracle(sc, B, L, lens, w, gl, alpha, gaps):
     _check_layer(case, _run_layer(sc, case, w))
 
 
-def _run_stack(sc, wl, inp):
+def _run_stack(sc, wl, inp, no_tail=False):
     dev = "cuda"
     Q, K, V = (bits_to_torch(inp[k], dev) for k in ("Q", "K", "V"))
     mask = None if inp["pad_mask"] is None else torch.from_numpy(inp["pad_mask"]).to(dev)
     ws = sc.new_workspace(wl.B, wl.L, wl.H, dev)
-    out = sc.stack_forward(Q, K, V, mask, inp["global_pos"], wl.w, inp["alpha"], workspace=ws)
+    out = sc.stack_forward(Q, K, V, mask, inp["global_pos"], wl.w, inp["alpha"], workspace=ws,
+                           no_tail=no_tail)
     assert sc.workspace_status(ws) == 0
     return {"O": torch_bf16_to_f64(out["O"]), "scores": out["scores"].cpu().numpy(),
             "pos": out["pos"].cpu().numpy(), "len": out["len"].cpu().numpy()}
@@ -110,10 +111,11 @@ STACKS = [
 ]
 
 
+@pytest.mark.parametrize("no_tail", [False, True], ids=["with_tail", "per_layer_only"])
 @pytest.mark.parametrize("wl", STACKS, ids=[w.name for w in STACKS])
-def test_stack_matches_oracle(sc, wl):
+def test_stack_matches_oracle(sc, wl, no_tail):
     inp, res, _ = resample_stack(wl)
-    _check_stack(wl, res, _run_stack(sc, wl, inp))
+    _check_stack(wl, res, _run_stack(sc, wl, inp, no_tail))
 
 
 def test_stack_theta_zero_keeps_everything(sc):

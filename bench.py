@@ -123,58 +123,136 @@ def whole_job_rate(world: int, units_per_step_per_rank: int, ms_per_step: float)
 # ---------------------------------------------------------------------------
 # clocks during the timed region
 # ---------------------------------------------------------------------------
+class _Nvml:
+    """Minimal NVML through ctypes (the library ships with the driver): SM clock,
+    its maximum, and the clock event reason bits.  Read-only."""
+    SM = 1                      # NVML_CLOCK_SM
+    BITS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown"}
+
+    def __init__(self, uuid, index):
+        import ctypes
+        self.c = ctypes
+        self.lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if self.lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        self.h = ctypes.c_void_p()
+        rc = 1
+        if uuid:
+            rc = self.lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(self.h))
+        if rc != 0:
+            rc = self.lib.nvmlDeviceGetHandleByIndex_v2(index, ctypes.byref(self.h))
+        if rc != 0:
+            raise OSError("no NVML handle for the device")
+        fn = getattr(self.lib, "nvmlDeviceGetCurrentClocksEventReasons", None)
+        self.reasons_fn = fn or self.lib.nvmlDeviceGetCurrentClocksThrottleReasons
+
+    def clock(self, max_clock=False):
+        v = self.c.c_uint()
+        f = self.lib.nvmlDeviceGetMaxClockInfo if max_clock else self.lib.nvmlDeviceGetClockInfo
+        return v.value if f(self.h, self.SM, self.c.byref(v)) == 0 else None
+
+    def reasons(self):
+        v = self.c.c_ulonglong()
+        if self.reasons_fn(self.h, self.c.byref(v)) != 0:
+            return []
+        return [nm for bit, nm in self.BITS.items() if v.value & bit]
+
+    def close(self):
+        self.lib.nvmlShutdown()
+
+
 class ClockSampler:
+    """SM clock and throttle reasons sampled every ~1 ms by a thread while the
+    timed region runs (NVML; nvidia-smi at 200 ms when NVML is unavailable).
+    ``mark_start()`` / ``mark_end()`` bound the samples that count."""
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
+        self.samples = []           # (host time, sm MHz, reasons)
+        self.max_mhz = None
+        self.t_lo = self.t_hi = None
+        self.source = None
+        self._stop = threading.Event()
         self.proc = None
-        self.lines = []
 
     def __enter__(self):
+        import torch
+        uuid = None
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
-                 "--format=csv,noheader,nounits", "-lms", "200"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
+            u = str(torch.cuda.get_device_properties(self.index).uuid)
+            uuid = u if u.startswith("GPU-") else "GPU-" + u
+        except Exception:
+            pass
+        try:
+            self.nvml = _Nvml(uuid, self.index)
+            self.max_mhz = self.nvml.clock(max_clock=True)
+            self.source = "nvml"
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+        except (OSError, AttributeError):
+            self.nvml = None
+            try:
+                self.proc = subprocess.Popen(
+                    ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
+                     "--format=csv,noheader,nounits", "-lms", "200"],
+                    stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                self.source = "nvidia-smi"
+                self.thread = threading.Thread(target=self._read, daemon=True)
+            except OSError:
+                self.thread = None
+        if self.thread is not None:
             self.thread.start()
-        except OSError:
-            self.proc = None
         return self
 
+    def _poll(self):
+        while not self._stop.is_set():
+            self.samples.append((time.perf_counter(), self.nvml.clock(), self.nvml.reasons()))
+            time.sleep(0.001)
+
     def _read(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            parts = [p.strip() for p in line.strip().split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm = float(parts[1])
+                self.max_mhz = float(parts[2])
+            except ValueError:
+                continue
+            rs = [nm for nm, v in zip(names, parts[5:9]) if v.lower().startswith("active")]
+            self.samples.append((time.perf_counter(), sm, rs))
+
+    def mark_start(self):
+        self.t_lo = time.perf_counter()
+
+    def mark_end(self):
+        self.t_hi = time.perf_counter()
 
     def __exit__(self, *exc):
+        self._stop.set()
         if self.proc is not None:
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
+        if self.thread is not None:
             self.thread.join(timeout=2)
+        if self.nvml is not None:
+            self.nvml.close()
 
     def summary(self):
-        sm, mx, reasons = [], None, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                mx = float(parts[2])
-            except ValueError:
-                continue
-            for nm, v in zip(names, parts[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(nm)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        lo = self.t_lo if self.t_lo is not None else -1e30
+        hi = self.t_hi if self.t_hi is not None else 1e30
+        inside = [(sm, rs) for t, sm, rs in self.samples if lo <= t <= hi and sm is not None]
+        reasons = sorted({r for _, rs in inside for r in rs})
+        sm = [x for x, _ in inside]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(sm), "source": self.source}
 
 
 # ---------------------------------------------------------------------------
@@ -290,7 +368,9 @@ def run_native(args, wl):
     stream = torch.cuda.current_stream()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(torch.cuda.current_device()) as clocks:
+        time.sleep(0.01)
         barrier()
+        clocks.mark_start()
         t0.record(stream)
         for _ in range(args.steps):
             if graph is not None:
@@ -299,6 +379,7 @@ def run_native(args, wl):
                 step()
         t1.record(stream)
         barrier()
+        clocks.mark_end()
     rc = sc.workspace_status(ws)
     if rc != 0:
         raise SystemExit("device status after the timed steps: %s" % sc.status_string(rc))
@@ -308,6 +389,17 @@ def run_native(args, wl):
     pos = out["pos"].cpu().numpy()
     kept_per_step = int(lens[:wl.n_layers].sum())
     value = whole_job_rate(world, kept_per_step, ms_per_step)
+
+    # ---- kernels launched per timed step.  Eagerly: the library's plan.  A
+    # captured step runs the per-layer kernels in a device-driven loop: prep,
+    # [padding gather], rows + cols + gather + advance for each layer that some
+    # sequence still runs per layer (more than 256 tokens), then the cluster kernel.
+    eager_launches = sc.stack_launch_count(wl.n_layers, wl.B, wl.L, wl.H, wl.w, gpos,
+                                           inp["pad_mask"] is not None)
+    looped = sum(1 for l in range(wl.n_layers) if (lens[l] > 256).any())
+    graph_launches = (1 + (1 if inp["pad_mask"] is not None else 0) + 4 * looped + 1
+                      if wl.L > 256 else 2)
+    launches_per_step = graph_launches if graph is not None else eager_launches
 
     # ---- per-kernel times on the launching stream (same steps, events between kernels)
     nev = 3 + 3 * wl.n_layers
@@ -320,7 +412,7 @@ def run_native(args, wl):
     gath_ms = np.zeros(wl.n_layers)
     prep_ms = 0.0
     tail_ms = 0.0
-    prof_steps = max(1, args.steps)
+    prof_steps = max(1, min(args.steps, 20))
     for _ in range(prof_steps):
         step(evs)
         torch.cuda.synchronize()
@@ -407,8 +499,7 @@ def run_native(args, wl):
                                     lens[:wl.n_layers + 1].sum(axis=1) / max(1, lens[0].sum())]},
             "roofline": roofline,
             "e2e": e2e,
-            "gpu_launches": args.steps * sc.stack_launch_count(
-                wl.n_layers, wl.B, wl.L, wl.H, wl.w, gpos, inp["pad_mask"] is not None),
+            "gpu_launches": args.steps * launches_per_step,
             "clocks": clocks.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
@@ -426,7 +517,7 @@ def run_native(args, wl):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="cfg4")

@@ -20,6 +20,7 @@ cudaError_t configure_kernels();
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st);
+cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st);
 cudaError_t configure_tail();
 cudaError_t tail_max_clusters(int H, int* out);
 cudaError_t launch_tail(const TailParams& p, cudaStream_t st);
@@ -47,7 +48,7 @@ size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
   size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident, tail_from,
-      qkv, total;
+      loop_layer, qkv, total;
 };
 
 bool ws_layout(int B, int L, int H, WsLayout* w) {
@@ -72,6 +73,7 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->ng = take(sizeof(int32_t) * 2 * B);
   w->ident = take(sizeof(int32_t) * 2 * B);
   w->tail_from = take(sizeof(int32_t) * B);
+  w->loop_layer = take(sizeof(int32_t));
   // compacted Q, K, V of the current layer (rows of the surviving tokens)
   w->qkv = take(sizeof(uint16_t) * 3 * B * (size_t)L * H * kHeadDim);
   w->total = off;
@@ -150,6 +152,8 @@ bool encode_maps(TensorMaps* m, const uint16_t* const src[3], long long tokens, 
   return true;
 }
 
+cudaStream_t capture_side_stream();
+
 int ensure_configured() {
   static std::mutex mu;
   static bool done[256] = {false};
@@ -164,7 +168,30 @@ int ensure_configured() {
     if (e != cudaSuccess) return fail_cuda("kernel attributes", e);
     done[dev] = true;
   }
+  capture_side_stream();   // made outside any capture when possible
   return SC_OK;
+}
+
+// A stream of this library per device, used only to record the body of the
+// layer loop into a graph under construction (nullptr if it cannot be made).
+cudaStream_t capture_side_stream() {
+  static std::mutex mu;
+  static cudaStream_t side[256] = {nullptr};
+  static bool tried[256] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!tried[dev]) {
+    tried[dev] = true;
+    if (cudaStreamCreateWithFlags(&side[dev], cudaStreamNonBlocking) != cudaSuccess) {
+      cudaGetLastError();
+      side[dev] = nullptr;
+    }
+  }
+  return side[dev];
 }
 
 // Whether the cluster kernel can run with clusters of H CTAs on the current
@@ -395,6 +422,40 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
            cudaEventRecord(static_cast<cudaEvent_t>(events[k]), st) == cudaSuccess;
   };
   cudaError_t e;
+
+  // While the call is captured into a CUDA graph, the per-layer kernels run
+  // in a WHILE node whose condition the device sets ("some sequence still has
+  // more than kTailMax tokens"), with the layer index in device memory: layers
+  // that every sequence has left cost no launch.  Eager calls launch every
+  // layer's kernels, which then skip the sequences of the cluster kernel.
+  bool dev_loop = false;
+  cudaGraphConditionalHandle cond = 0;
+  cudaStream_t side = nullptr;
+  if (use_tail && per_layer && events == nullptr) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) {
+      cudaGetLastError();
+      cap = cudaStreamCaptureStatusNone;
+    }
+    if (cap == cudaStreamCaptureStatusActive) side = capture_side_stream();
+    if (side != nullptr) {
+      cudaGraph_t g = nullptr;
+      cudaStreamCaptureStatus cs;
+      if ((e = cudaStreamGetCaptureInfo(st, &cs, nullptr, &g)) != cudaSuccess)
+        return fail_cuda("stream capture info", e);
+      if ((e = cudaGraphConditionalHandleCreate(&cond, g, 0, cudaGraphCondAssignDefault)) !=
+          cudaSuccess)
+        return fail_cuda("conditional handle", e);
+      dev_loop = true;
+    }
+  }
+  int* loop_layer = reinterpret_cast<int*>(ws + lay.loop_layer);
+  if (dev_loop) {
+    pp.dev_layer = loop_layer;
+    pp.cond = cond;
+    pp.has_cond = 1;
+  }
+
   if (!mark(0)) return fail(SC_ERR_CUDA, "event record", "");
   if ((e = launch_prep(pp, st)) != cudaSuccess) return fail_cuda("launch prep kernel", e);
   if (!mark(1)) return fail(SC_ERR_CUDA, "event record", "");
@@ -407,7 +468,80 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     gp.src[t] = src[t];
     gp.dst[t] = cmp[t];
   }
+  if (dev_loop) {
+    if (a->pad_mask != nullptr) {
+      // padding removal may have moved rows: compact layer 0 as well
+      gp.src_base = 0;
+      gp.layer = 0;
+      gp.len = a->len;
+      gp.pos = a->pos;
+      gp.ident = p.ident;
+      if ((e = launch_gather(gp, st)) != cudaSuccess) return fail_cuda("launch gather kernel", e);
+    }
+    LayerParams pd = p;   // workspace slot 0: layer 0's ping-pong buffers
+    pd.dev_layer = loop_layer;
+    pd.layer = 0;
+    pd.src_base = 0;
+    pd.len = a->len;
+    pd.len_out = a->len + a->B;
+    pd.pos = a->pos;
+    pd.pos_out = a->pos + BL;
+    pd.O = a->O;
+    pd.scores = a->scores;
+    pd.alpha = a->alpha[0];
+    pd.tok_stride = BLt;
+    pd.row_stride = static_cast<long long>(BL);
+    pd.o_stride = static_cast<long long>(BL) * a->H * kHeadDim;
+    pd.len_stride = a->B;
+    for (int l = 0; l < a->n_layers; ++l) pd.alphas[l] = a->alpha[l];
+    GatherParams gd = gp;
+    gd.dev_layer = loop_layer;
+    gd.n_layers = a->n_layers;
+    gd.tok_stride = BLt;
+    gd.row_stride = static_cast<long long>(BL);
+    gd.len_stride = a->B;
+    gd.len = a->len;
+    gd.pos = a->pos;
+    gd.ident_slot[0] = p.ident;
+    gd.ident_slot[1] = p.ident_out;
+    AdvanceParams ad{};
+    ad.B = a->B;
+    ad.n_layers = a->n_layers;
+    ad.dev_layer = loop_layer;
+    ad.tail_from = tail_from;
+    ad.cond = cond;
+
+    cudaGraph_t g = nullptr;
+    const cudaGraphNode_t* deps = nullptr;
+    size_t ndeps = 0;
+    cudaStreamCaptureStatus cs;
+    if ((e = cudaStreamGetCaptureInfo(st, &cs, nullptr, &g, &deps, nullptr, &ndeps)) != cudaSuccess)
+      return fail_cuda("stream capture info", e);
+    cudaGraphNodeParams cp = {};
+    cp.type = cudaGraphNodeTypeConditional;
+    cp.conditional.handle = cond;
+    cp.conditional.type = cudaGraphCondTypeWhile;
+    cp.conditional.size = 1;
+    cudaGraphNode_t node;
+    if ((e = cudaGraphAddNode(&node, g, deps, nullptr, ndeps, &cp)) != cudaSuccess)
+      return fail_cuda("add WHILE node", e);
+    if ((e = cudaStreamBeginCaptureToGraph(side, cp.conditional.phGraph_out[0], nullptr, nullptr, 0,
+                                           cudaStreamCaptureModeRelaxed)) != cudaSuccess)
+      return fail_cuda("capture layer loop body", e);
+    cudaError_t le = launch_rows(maps, pd, side);
+    if (le == cudaSuccess) le = launch_cols(maps, pd, side);
+    if (le == cudaSuccess) le = launch_gather(gd, side);
+    if (le == cudaSuccess) le = launch_advance(ad, side);
+    cudaGraph_t body = nullptr;
+    e = cudaStreamEndCapture(side, &body);
+    if (le != cudaSuccess) return fail_cuda("launch layer loop body", le);
+    if (e != cudaSuccess) return fail_cuda("end layer loop body capture", e);
+    if ((e = cudaStreamUpdateCaptureDependencies(st, &node, nullptr, 1,
+                                                 cudaStreamSetCaptureDependencies)) != cudaSuccess)
+      return fail_cuda("capture dependencies", e);
+  }
   for (int l = 0; l < a->n_layers; ++l) {
+    if (dev_loop) break;
     if (!per_layer) {
       if (!mark(2 + 3 * l) || !mark(3 + 3 * l) || !mark(4 + 3 * l))
         return fail(SC_ERR_CUDA, "event record", "");

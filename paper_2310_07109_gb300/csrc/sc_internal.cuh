@@ -77,6 +77,35 @@ struct LayerParams {
   int32_t* tail_from;    // [B]
   int layer;
   int tail_max;
+  // Device-driven layer loop (a CUDA graph WHILE node): when dev_layer is set,
+  // the layer is *dev_layer and the per-layer fields above hold their layer-0
+  // values, advanced by these strides (gcur/ng/ident swap slots on odd layers;
+  // alpha comes from alphas[layer]).
+  const int* dev_layer;
+  long long tok_stride;   // tokens of one layer in the source tensors (B * L)
+  long long row_stride;   // entries of one layer in pos, pos_out, scores (B * L)
+  long long o_stride;     // elements of one layer in O (B * L * H * 64)
+  int len_stride;         // entries of one layer in len, len_out (B)
+  float alphas[kTailMaxLayers];
+};
+
+// The per-layer fields of one launch, resolved (see layer_view in sc_kernels.cu).
+struct LayerView {
+  int layer;
+  long long src_base;
+  const int32_t* len;
+  int32_t* len_out;
+  const int32_t* pos;
+  int32_t* pos_out;
+  const int32_t* gcur;
+  int32_t* gcur_out;
+  const int32_t* ng;
+  int32_t* ng_out;
+  const int32_t* ident;
+  int32_t* ident_out;
+  uint16_t* O;
+  float* scores;
+  float alpha;
 };
 
 // Copies the rows of the kept tokens (at their original positions) of one
@@ -91,6 +120,23 @@ struct GatherParams {
   uint16_t* dst[3];            // compacted Q, K, V [B][L][H][64]
   const int32_t* tail_from;    // [B] or nullptr: skip b when tail_from[b] <= layer
   int layer;                   // the layer whose rows are gathered
+  // device-driven layer loop: the gathered layer is *dev_layer + 1, len/pos
+  // above are those of layer 0 (advanced by the strides), ident alternates
+  // between the two slots; nothing is gathered past the last layer
+  const int* dev_layer;
+  int n_layers;
+  long long tok_stride, row_stride;
+  int len_stride;
+  const int32_t* ident_slot[2];
+};
+
+// One step of the device-driven layer loop: layer += 1, and the loop goes on
+// while some sequence still runs through the per-layer kernels.
+struct AdvanceParams {
+  int B, n_layers;
+  int* dev_layer;
+  const int32_t* tail_from;
+  unsigned long long cond;     // cudaGraphConditionalHandle of the WHILE node
 };
 
 struct PrepParams {
@@ -105,6 +151,9 @@ struct PrepParams {
   int32_t* ident;            // [B]
   int32_t* tail_from;        // [B] (stack mode with the cluster kernel) or nullptr
   int tail_max;
+  int* dev_layer;            // device-driven loop: set to 0 here, or nullptr
+  unsigned long long cond;   // ... and its WHILE condition: some sequence has > tail_max tokens
+  int has_cond;
   int n_global;
   int global_pos[kMaxGlobal];
 };

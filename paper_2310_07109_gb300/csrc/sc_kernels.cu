@@ -69,10 +69,42 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 
+// The per-layer fields of this launch: as given, or (device-driven layer
+// loop) the layer-0 values advanced to layer *dev_layer.
+__device__ __forceinline__ LayerView layer_view(const LayerParams& p) {
+  LayerView v;
+  if (p.dev_layer == nullptr) {
+    v.layer = p.layer; v.src_base = p.src_base;
+    v.len = p.len; v.len_out = p.len_out; v.pos = p.pos; v.pos_out = p.pos_out;
+    v.gcur = p.gcur; v.gcur_out = p.gcur_out; v.ng = p.ng; v.ng_out = p.ng_out;
+    v.ident = p.ident; v.ident_out = p.ident_out;
+    v.O = p.O; v.scores = p.scores; v.alpha = p.alpha;
+    return v;
+  }
+  const int l = __ldcg(p.dev_layer);
+  const bool odd = (l & 1) != 0;
+  v.layer = l;
+  v.src_base = l * p.tok_stride;
+  v.len = p.len + static_cast<size_t>(l) * p.len_stride;
+  v.len_out = p.len_out + static_cast<size_t>(l) * p.len_stride;
+  v.pos = p.pos + l * p.row_stride;
+  v.pos_out = p.pos_out + l * p.row_stride;
+  v.gcur = odd ? p.gcur_out : p.gcur;
+  v.gcur_out = odd ? const_cast<int32_t*>(p.gcur) : p.gcur_out;
+  v.ng = odd ? p.ng_out : p.ng;
+  v.ng_out = odd ? const_cast<int32_t*>(p.ng) : p.ng_out;
+  v.ident = odd ? p.ident_out : p.ident;
+  v.ident_out = odd ? const_cast<int32_t*>(p.ident) : p.ident_out;
+  v.O = p.O + l * p.o_stride;
+  v.scores = p.scores + l * p.row_stride;
+  v.alpha = p.alphas[l];
+  return v;
+}
+
 // Sequence b has been handed to the cluster kernel for this and later layers
 // (its length here may be stale: read nothing else of it).
-__device__ __forceinline__ bool owned_by_tail(const LayerParams& p, int b) {
-  return p.tail_from != nullptr && __ldcg(p.tail_from + b) <= p.layer;
+__device__ __forceinline__ bool owned_by_tail(const LayerParams& p, const LayerView& v, int b) {
+  return p.tail_from != nullptr && __ldcg(p.tail_from + b) <= v.layer;
 }
 
 // Which source holds the current rows of sequence b, and the token index of
@@ -82,9 +114,9 @@ struct RowSource {
   long long tok_b;
 };
 
-__device__ __forceinline__ RowSource row_source(const LayerParams& p, int b) {
-  const bool id = __ldg(p.ident + b) != 0;
-  return {id ? 0 : 1, (id ? p.src_base : 0) + static_cast<long long>(b) * p.L};
+__device__ __forceinline__ RowSource row_source(const LayerParams& p, const LayerView& v, int b) {
+  const bool id = __ldg(v.ident + b) != 0;
+  return {id ? 0 : 1, (id ? v.src_base : 0) + static_cast<long long>(b) * p.L};
 }
 
 // One 128-token tile (current rows c0 .. c0+127) of tensor t (0 Q, 1 K, 2 V)
@@ -179,14 +211,15 @@ __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint
 }
 
 __global__ void __launch_bounds__(kRowsThreads, 1)
-    sc_rows_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
+    sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
   // grid: x = (sequence, head), y = pair of query tiles, so that low tiles (the
   // ones every sequence has) are dispatched first
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
-  if (owned_by_tail(p, b)) return;
-  const int n = __ldg(p.len + b);
+  const LayerView v = layer_view(p);
+  if (owned_by_tail(p, v, b)) return;
+  const int n = __ldcg(v.len + b);
   if (2 * pr * kTile >= n) return;
-  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
   const bool hasB = (2 * pr + 1) * kTile < n;
 
@@ -233,7 +266,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
+  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldcg(v.gcur + b * kMaxGlobal + tid) : -1;
   if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
@@ -243,7 +276,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 
   if (warp == 8) {
     // ------------------------------------------------------------- loads
-    const RowSource rs = row_source(p, b);
+    const RowSource rs = row_source(p, v, b);
     if (lane == 0) {
       mbar_arrive_expect_tx(&sm.bar_q, (hasB ? 2 : 1) * kTileBytes + 3 * ngp * 128);
       load_tile(maps, 0, rs, h, 2 * pr * kTile, Qs, &sm.bar_q);
@@ -537,7 +570,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       tc_fence_after();
       const float inv = 1.f / lsum;
       lse = valid ? m_ref + lg2(lsum) : INFINITY;
-      uint16_t* orow = p.O + ((static_cast<size_t>(b) * p.L + i) * p.H + h) * kHeadDim;
+      uint16_t* orow = v.O + ((static_cast<size_t>(b) * p.L + i) * p.H + h) * kHeadDim;
 #pragma unroll
       for (int c = 0; c < 64; c += 32) {
         float o[32];
@@ -637,23 +670,25 @@ struct ColsSmem {
 // queries, and one A tile (32 KB) per warpgroup for the global rows' P V
 constexpr uint32_t kColsDyn = kTileBytes * (4 + kStages) + kGTileBytes + 4 * kTileBytes + 1024;
 
-__device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm);
+__device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
+                                  ColsSmem& sm);
 
 __global__ void __launch_bounds__(kColsThreads, 1)
-    sc_cols_kernel(const __grid_constant__ TensorMaps maps, const LayerParams p) {
+    sc_cols_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
-  if (owned_by_tail(p, b)) return;
-  const int n = __ldg(p.len + b);
+  const LayerView v = layer_view(p);
+  if (owned_by_tail(p, v, b)) return;
+  const int n = __ldcg(v.len + b);
   if (n == 0) {
     if (pr == 0 && h == 0 && threadIdx.x == 0) {
-      p.len_out[b] = 0;
-      p.ng_out[b] = 0;
-      p.ident_out[b] = 1;
+      v.len_out[b] = 0;
+      v.ng_out[b] = 0;
+      v.ident_out[b] = 1;
     }
     return;
   }
   if (2 * pr * kTile >= n) return;
-  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
   const int Tn = (n + kTile - 1) / kTile;
   const int Tp = (Tn + 1) / 2;
@@ -698,7 +733,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldg(p.gcur + b * kMaxGlobal + tid) : -1;
+  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldcg(v.gcur + b * kMaxGlobal + tid) : -1;
   if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
@@ -707,7 +742,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   volatile int* abort_flag = &sm.abort;
 
   if (warp == 8) {
-    const RowSource rs = row_source(p, b);
+    const RowSource rs = row_source(p, v, b);
     if (lane == 0) {
       mbar_arrive_expect_tx(&sm.bar_kv, (hasB ? 4 : 2) * kTileBytes + ngp * 128);
       for (int X = 0; X < (hasB ? 2 : 1); ++X) {
@@ -972,8 +1007,8 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     for (int g = 0; g < ng; ++g)
       if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
-    p.scores[static_cast<size_t>(b) * p.L + jj] = s;
-    const float theta = p.theta ? __ldg(p.theta + b) : p.alpha / static_cast<float>(n);
+    v.scores[static_cast<size_t>(b) * p.L + jj] = s;
+    const float theta = p.theta ? __ldg(p.theta + b) : v.alpha / static_cast<float>(n);
     p.keep[static_cast<size_t>(b) * p.L + jj] = (jj == 0 || s >= theta) ? 1 : 0;
   }
   if (tid == 0) p.cnt_tile[b * p.T + pr] = 0u;
@@ -983,12 +1018,13 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   __syncthreads();
   if (!sm.flag) return;
   __threadfence();
-  finalize_sequence(p, b, n, sm);
+  finalize_sequence(p, v, b, n, sm);
 }
 
 // Order-preserving compaction of sequence b's kept tokens, the next layer's
 // global list, and the bf16 outputs of the global rows.  One CTA.
-__device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& sm) {
+__device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
+                                  ColsSmem& sm) {
   const int tid = threadIdx.x;
   const int per = (n + kColsThreads - 1) / kColsThreads;
   const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
@@ -1007,11 +1043,11 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
   }
   int out = sm.scan[tid] - cnt;
   const int total = sm.scan[kColsThreads - 1];
-  const int ng = min(__ldg(p.ng + b), kMaxGlobal);
+  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
   if (tid < kMaxGlobal) sm.gnew[tid] = -1;
   __syncthreads();
-  const int32_t* pos = p.pos + static_cast<size_t>(b) * p.L;
-  int32_t* pos_out = p.pos_out + static_cast<size_t>(b) * p.L;
+  const int32_t* pos = v.pos + static_cast<size_t>(b) * p.L;
+  int32_t* pos_out = v.pos_out + static_cast<size_t>(b) * p.L;
   for (int c = c0; c < c1; ++c) {
     if (!__ldcg(keep + c)) continue;
     pos_out[out] = __ldg(pos + c);
@@ -1023,20 +1059,20 @@ __device__ void finalize_sequence(const LayerParams& p, int b, int n, ColsSmem& 
 #pragma unroll 4
   for (int k = tid; k < ng * p.H * kHeadDim; k += kColsThreads) {
     const int g = k / (p.H * kHeadDim), hh = (k / kHeadDim) % p.H, dd = k % kHeadDim;
-    const float v = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
-    p.O[((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) * kHeadDim + dd] =
-        __bfloat16_as_ushort(__float2bfloat16_rn(v));
+    const float o = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
+    v.O[((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) * kHeadDim + dd] =
+        __bfloat16_as_ushort(__float2bfloat16_rn(o));
   }
   __syncthreads();
   if (tid == 0) {
     int m = 0;
     for (int g = 0; g < ng; ++g)
-      if (sm.gnew[g] >= 0) p.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
-    p.ng_out[b] = m;
-    p.len_out[b] = total;
-    if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = p.layer + 1;
+      if (sm.gnew[g] >= 0) v.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
+    v.ng_out[b] = m;
+    v.len_out[b] = total;
+    if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = v.layer + 1;
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
-    p.ident_out[b] = (total == 0 || pos_out[total - 1] == total - 1) ? 1 : 0;
+    v.ident_out[b] = (total == 0 || pos_out[total - 1] == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
   }
 }
@@ -1052,15 +1088,28 @@ constexpr int kGatherThreads = 256;
 __global__ void __launch_bounds__(kGatherThreads)
     sc_gather_kernel(const GatherParams g) {
   const int b = blockIdx.y;
-  if (g.tail_from != nullptr && __ldcg(g.tail_from + b) <= g.layer) return;
-  const int n = __ldg(g.len + b);
+  int layer = g.layer;
+  long long src_base = g.src_base;
+  const int32_t* lenp = g.len;
+  const int32_t* posp = g.pos;
+  const int32_t* identp = g.ident;
+  if (g.dev_layer != nullptr) {
+    layer = __ldcg(g.dev_layer) + 1;
+    if (layer >= g.n_layers) return;
+    src_base = layer * g.tok_stride;
+    lenp += static_cast<size_t>(layer) * g.len_stride;
+    posp += layer * g.row_stride;
+    identp = g.ident_slot[layer & 1];
+  }
+  if (g.tail_from != nullptr && __ldcg(g.tail_from + b) <= layer) return;
+  const int n = __ldcg(lenp + b);
   const int c0 = blockIdx.x * kGatherTokens;
-  if (__ldg(g.ident + b) != 0 || c0 >= n) return;
+  if (__ldcg(identp + b) != 0 || c0 >= n) return;
   const int cnt = min(kGatherTokens, n - c0);
   const int vec = g.H * kHeadDim / 8;  // 16-byte vectors per token row
   const int total = cnt * vec;
   const long long dst_tok0 = static_cast<long long>(b) * g.L + c0;
-  const long long src_tok0 = g.src_base + static_cast<long long>(b) * g.L;
+  const long long src_tok0 = src_base + static_cast<long long>(b) * g.L;
   constexpr int kPer = 4;   // vectors per thread and tensor per round
   for (int k0 = threadIdx.x; k0 < total; k0 += kGatherThreads * kPer) {
     uint4 v[3][kPer];
@@ -1069,7 +1118,7 @@ __global__ void __launch_bounds__(kGatherThreads)
     for (int u = 0; u < kPer; ++u) {
       const int k = k0 + u * kGatherThreads;
       const int tk = k / vec, e = k - tk * vec;
-      so[u] = k < total ? (src_tok0 + __ldg(g.pos + static_cast<size_t>(b) * g.L + c0 + tk)) * vec + e
+      so[u] = k < total ? (src_tok0 + __ldcg(posp + static_cast<size_t>(b) * g.L + c0 + tk)) * vec + e
                         : -1;
       doff[u] = (dst_tok0 + tk) * vec + e;
     }
@@ -1150,6 +1199,25 @@ __global__ void __launch_bounds__(kPrepThreads)
     // single-layer calls read their (already current-order) inputs in place
     pp.ident[b] = (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1) ? 1 : 0;
     if (pp.tail_from != nullptr) pp.tail_from[b] = n <= pp.tail_max ? 0 : 0x7fffffff;
+    if (pp.has_cond && n > pp.tail_max) cudaGraphSetConditional(pp.cond, 1u);
+    if (pp.dev_layer != nullptr && b == 0) *pp.dev_layer = 0;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// advance kernel: one step of the device-driven layer loop
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) sc_advance_kernel(const AdvanceParams a) {
+  __shared__ int s_layer;
+  if (threadIdx.x == 0) s_layer = __ldcg(a.dev_layer) + 1;
+  __syncthreads();
+  const int l = s_layer;
+  int big = 0;
+  for (int b = threadIdx.x; b < a.B; b += blockDim.x) big |= __ldcg(a.tail_from + b) > l;
+  big = __syncthreads_or(big);
+  if (threadIdx.x == 0) {
+    *a.dev_layer = l;
+    cudaGraphSetConditional(a.cond, (big && l < a.n_layers) ? 1u : 0u);
   }
 }
 
@@ -1190,6 +1258,11 @@ cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t 
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
   dim3 grid(p.B * p.H, (p.T + 1) / 2);
   sc_cols_kernel<<<grid, kColsThreads, kColsDyn, st>>>(m, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st) {
+  sc_advance_kernel<<<1, 256, 0, st>>>(a);
   return cudaGetLastError();
 }
 

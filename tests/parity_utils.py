@@ -29,13 +29,15 @@ def near_threshold(scores, n, theta):
     return [int(j) for j in bad if j != 0]
 
 
-def resample_stack(wl: wk.Workload, max_rounds: int = 50, nthreads=None):
+def resample_stack(wl: wk.Workload, max_rounds: int = 50, nthreads=None, overrides=None):
     """Draw ``wl`` and redraw (layer, token) Q/K rows until no oracle score of any
     layer lies within MARGIN / n of its threshold.  Layers interact only through
-    the kept set, so fixing the first offending layer and re-running converges."""
+    the kept set, so fixing the first offending layer and re-running converges.
+    ``overrides`` replaces entries of the drawn inputs (e.g. global_pos, pad_mask)."""
     redraws = {}
     for _ in range(max_rounds):
         inp = wk.make_inputs(wl, redraws)
+        inp.update(overrides or {})
         res = oracle.stack(inp["Q"], inp["K"], inp["V"], inp["pad_mask"], inp["global_pos"],
                            wl.w, inp["alpha"], nthreads=nthreads)
         bad = []
@@ -63,8 +65,9 @@ def bits_to_torch(bits, device):
 
 def torch_bf16_to_f64(t):
     import torch
-    return t.detach().to("cpu").view(torch.int16).numpy().view(np.uint16).astype(np.uint32) \
-        .__lshift__(16).view(np.float32).astype(np.float64)
+    bits = t.detach().to("cpu").view(torch.int16).numpy().view(np.uint16).astype(np.uint32)
+    with np.errstate(invalid="ignore"):   # unused output slots may hold NaN patterns
+        return (bits << 16).view(np.float32).astype(np.float64)
 
 
 def layer_case(B, L, H, lens, w, gpos, alpha, seed, scale_k=2.0, gaps=False, max_rounds=50):

@@ -168,38 +168,59 @@ __device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_
 // ---------------------------------------------------------------------------
 // One CTA per pair of 128-row query tiles (2p, 2p+1) of one (sequence, head),
 // one softmax warpgroup per tile; the two tiles share their K/V tiles (the
-// band of the pair spans at most six 128-key tiles) and the tensor core
-// alternates between the two warpgroups.
+// band of the pair spans at most six 128-key tiles: all K tiles stay
+// resident, V tiles pass through a ring) and one tensor core serves both.
 //
-// Tensor memory (512 columns) per warpgroup X in {0, 1}:
-//   S/P  [192 X, 192 X + 128)  S of the current key tile (fp32); P (bf16
-//        pairs) overwrites its first 64 columns once all of S is in registers.
-//        The MMA that reads P and the next one that writes S are issued in
-//        that order by one thread, and they execute in issue order.
-//   O    [192 X + 128, 192 X + 192)
-//   S_G  [384 + 32 X, +16)  S of the 16 global keys;  P_G [400 + 32 X, +8)
-//   S_Gt [448 + 16 X, +16)  S^T of the diagonal key tile against the global queries
-constexpr int kRowsThreads = 320;   // 2 softmax warpgroups + load warp + MMA warp
-constexpr int kStages = 4;          // K/V ring depth
+// Per key tile a warpgroup loads all 128 columns of S into registers and
+// hands that tensor memory straight back, so S of its next key tile is
+// computed while it evaluates this tile's exponentials.  P (bf16) goes to its
+// own tensor-memory columns and P V reads it from there (no shared-memory
+// traffic for P).
+//
+// Tensor memory (512 columns) per warpgroup X in {0, 1}, base 256 X:
+//   S    [+0, +128)   S of the current key tile (fp32); after the last tile:
+//                     S_G [+0, +16) (the 16 global keys) and S_Gt [+16, +32)
+//                     (the diagonal key tile against the global queries)
+//   P    [+128, +192) P of the current key tile, bf16 pairs; before the
+//                     first tile: S_G [+128, +144) and P_G [+144, +152)
+//   O    [+192, +256)
+// Warps 0-7: the two softmax warpgroups; warpgroup 2 (warps 8-11): warp 8
+// loads Q and the K tiles, warp 10 the V tiles, warps 9 and 11 issue the MMAs
+// of softmax warpgroups 0 and 1 (one issuing thread per warpgroup, so each
+// tcgen05.commit covers that warpgroup's MMAs only).
+// Launched at 168 registers a thread (three warps per SM sub-partition);
+// warpgroup 2 gives registers back so that the softmax warps, which hold a
+// whole 128-column row of S, get 200: 128 x 96 + 256 x 200 = 63488 <= 384 x 168.
+constexpr int kRowsThreads = 384;
+constexpr int kRowsCtlRegs = 96;
+constexpr int kRowsSoftmaxRegs = 200;
+static_assert(128 * kRowsCtlRegs + 256 * kRowsSoftmaxRegs <= kRowsThreads * 168,
+              "register split exceeds the launch allocation");
 constexpr int kPairTiles = kMaxBandTiles + 1;
+// V slots: with six key tiles only the sixth reuses a slot, that of the first;
+// the first is used by query tile 0 alone and the sixth by query tile 1 alone
+// (each query tile's band spans at most five key tiles).
+constexpr int kVStages = kPairTiles - 1;
 
-__host__ __device__ constexpr uint32_t col_sp(int X) { return 192u * X; }
-__host__ __device__ constexpr uint32_t col_o(int X) { return 192u * X + 128u; }
-__host__ __device__ constexpr uint32_t col_sg(int X) { return 384u + 32u * X; }
-__host__ __device__ constexpr uint32_t col_pg(int X) { return 400u + 32u * X; }
-__host__ __device__ constexpr uint32_t col_sgt(int X) { return 448u + 16u * X; }
+__host__ __device__ constexpr uint32_t col_s(int X) { return 256u * X; }
+__host__ __device__ constexpr uint32_t col_p(int X) { return 256u * X + 128u; }
+__host__ __device__ constexpr uint32_t col_o(int X) { return 256u * X + 192u; }
 
 struct RowsSmem {
   uint64_t bar_q;
-  uint64_t bar_kfull[kStages], bar_vfull[kStages], bar_kempty[kStages], bar_vempty[kStages];
-  uint64_t bar_sg[2], bar_sgt[2], bar_sfull[2], bar_pready[2], bar_done[2], bar_fin;
+  uint64_t bar_kfull[kPairTiles];
+  uint64_t bar_vfull[kVStages], bar_vempty[kVStages];
+  uint64_t bar_sg[2], bar_sgend[2], bar_sfull[2], bar_sfree[2], bar_pready[2], bar_pvdone[2];
+  uint64_t bar_fin[2];
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
 };
 
-// dynamic shared memory: two Q tiles, the K/V ring and the global rows
-constexpr uint32_t kRowsDyn = kTileBytes * (2 + 2 * kStages) + 3 * kGTileBytes + 1024;
+// dynamic shared memory: two Q tiles, every K tile of the pair, the V ring,
+// the global rows
+constexpr uint32_t kRowsDyn =
+    kTileBytes * (2 + kPairTiles + kVStages) + 3 * kGTileBytes + 1024;
 
 // Issue P V for one 128-key tile: P (A) from tensor memory, V (B) MN-major smem.
 __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint32_t v_smem,
@@ -209,6 +230,31 @@ __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint
     umma_bf16_ts(d_tmem, p_tmem + 8 * k, sdesc_sw128(v_smem + k * 2048), idesc,
                  (accumulate || k > 0) ? 1u : 0u);
 }
+
+// Reduce 16 values per lane over the warp (butterfly reduce-scatter, 16
+// shuffles): lane L returns the warp-wide result for element L >> 1.
+template <typename Op>
+__device__ __forceinline__ float warp_reduce16(float (&v)[16], Op op) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int half = 8, bit = 16; half >= 1; half >>= 1, bit >>= 1) {
+    const bool upper = (lane & bit) != 0;
+#pragma unroll
+    for (int k = 0; k < half; ++k) {
+      const float send = upper ? v[k] : v[k + half];
+      const float keep = upper ? v[k + half] : v[k];
+      v[k] = op(keep, __shfl_xor_sync(0xffffffffu, send, bit));
+    }
+  }
+  return op(v[0], __shfl_xor_sync(0xffffffffu, v[0], 1));
+}
+
+struct OpAdd {
+  __device__ __forceinline__ float operator()(float a, float b) const { return a + b; }
+};
+struct OpMax {
+  __device__ __forceinline__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
 
 __global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
@@ -227,9 +273,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* Qs = base;                                // 2 tiles
-  uint8_t* Ks = Qs + 2 * kTileBytes;                 // kStages tiles
-  uint8_t* Vs = Ks + kStages * kTileBytes;           // kStages tiles
-  uint8_t* KG = Vs + kStages * kTileBytes;
+  uint8_t* Ks = Qs + 2 * kTileBytes;                 // kPairTiles tiles (all resident)
+  uint8_t* Vs = Ks + kPairTiles * kTileBytes;        // kVStages tiles
+  uint8_t* KG = Vs + kVStages * kTileBytes;
   uint8_t* VG = KG + kGTileBytes;
   uint8_t* QG = VG + kGTileBytes;
   __shared__ RowsSmem sm;
@@ -249,20 +295,20 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 
   if (tid == 0) {
     mbar_init(&sm.bar_q, 1);
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&sm.bar_kfull[s], 1);
+    for (int k = 0; k < kPairTiles; ++k) mbar_init(&sm.bar_kfull[k], 1);
+    for (int s = 0; s < kVStages; ++s) {
       mbar_init(&sm.bar_vfull[s], 1);
-      mbar_init(&sm.bar_kempty[s], 1);
       mbar_init(&sm.bar_vempty[s], 1);
     }
     for (int X = 0; X < 2; ++X) {
       mbar_init(&sm.bar_sg[X], 1);
-      mbar_init(&sm.bar_sgt[X], 1);
+      mbar_init(&sm.bar_sgend[X], 1);
       mbar_init(&sm.bar_sfull[X], 1);
+      mbar_init(&sm.bar_sfree[X], 128);
       mbar_init(&sm.bar_pready[X], 128);
-      mbar_init(&sm.bar_done[X], 1);
+      mbar_init(&sm.bar_pvdone[X], 1);
+      mbar_init(&sm.bar_fin[X], 1);
     }
-    mbar_init(&sm.bar_fin, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -274,8 +320,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   const uint32_t tm = sm.tmem_base;
   volatile int* abort_flag = &sm.abort;
 
-  if (warp == 8) {
-    // ------------------------------------------------------------- loads
+  if (warp >= 8) {
+   regs_dealloc<kRowsCtlRegs>();
+   if (warp == 8) {
+    // ------------------------------------------------------------- Q, globals, K
     const RowSource rs = row_source(p, v, b);
     if (lane == 0) {
       mbar_arrive_expect_tx(&sm.bar_q, (hasB ? 2 : 1) * kTileBytes + 3 * ngp * 128);
@@ -289,111 +337,94 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_q, lane);
     }
     if (lane == 0) {
-      bool ok = true;
-      for (int k = 0; ok && k < nk; ++k) {
-        const int s = k % kStages, c0 = (kt_lo + k) * kTile;
-        const uint32_t ph = ((k / kStages) - 1) & 1;
-        if (k >= kStages && !(ok = mbar_wait(&sm.bar_kempty[s], ph, abort_flag))) break;
-        mbar_arrive_expect_tx(&sm.bar_kfull[s], kTileBytes);
-        load_tile(maps, 1, rs, h, c0, Ks + s * kTileBytes, &sm.bar_kfull[s]);
-        if (k >= kStages && !(ok = mbar_wait(&sm.bar_vempty[s], ph, abort_flag))) break;
-        mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
-        load_tile(maps, 2, rs, h, c0, Vs + s * kTileBytes, &sm.bar_vfull[s]);
+      for (int k = 0; k < nk; ++k) {
+        mbar_arrive_expect_tx(&sm.bar_kfull[k], kTileBytes);
+        load_tile(maps, 1, rs, h, (kt_lo + k) * kTile, Ks + k * kTileBytes, &sm.bar_kfull[k]);
       }
       // nothing may still be landing in shared memory when the CTA exits
       drain_wait(&sm.bar_q, 0);
-      for (int s = 0; s < kStages && s < nk; ++s) {
-        const int last = s + kStages * ((nk - 1 - s) / kStages);  // last tile of stage s
-        drain_wait(&sm.bar_kfull[s], (last / kStages) & 1);
-        drain_wait(&sm.bar_vfull[s], (last / kStages) & 1);
+      for (int k = 0; k < nk; ++k) drain_wait(&sm.bar_kfull[k], 0);
+    }
+   } else if (warp == 10) {
+    // ------------------------------------------------------------- V ring
+    if (lane == 0) {
+      const RowSource rs = row_source(p, v, b);
+      bool ok = true;
+      for (int k = 0; ok && k < nk; ++k) {
+        const int s = k % kVStages;
+        if (k >= kVStages &&
+            !(ok = mbar_wait(&sm.bar_vempty[s], ((k / kVStages) - 1) & 1, abort_flag)))
+          break;
+        mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
+        load_tile(maps, 2, rs, h, (kt_lo + k) * kTile, Vs + s * kTileBytes, &sm.bar_vfull[s]);
+      }
+      for (int s = 0; s < kVStages && s < nk; ++s) {
+        const int last = s + kVStages * ((nk - 1 - s) / kVStages);
+        drain_wait(&sm.bar_vfull[s], (last / kVStages) & 1);
       }
     }
-  } else if (warp == 9) {
+   } else if (warp == 9 || warp == 11) {
     // ------------------------------------------------------------- MMA issue
-    if (lane == 0) {
-      const uint32_t q_a = smem_u32(Qs), k_a = smem_u32(Ks), v_a = smem_u32(Vs);
-      const int nX = hasB ? 2 : 1;
-      // remaining users (warpgroups) of each key tile's K and of its V, two
-      // bits per tile (kept in registers)
-      uint32_t kuse = 0;
-      for (int k = 0; k < kPairTiles; ++k) {
-        const int a = kt_lo + k;
-        const uint32_t u = (a >= klo[0] && a <= khi[0]) + (hasB && a >= klo[1] && a <= khi[1]);
-        kuse |= u << (2 * k);
-      }
-      uint32_t vuse = kuse;
-      int cur0 = klo[0], cur1 = klo[1];   // next key tile of each warpgroup
-      int pu0 = 0, pu1 = 0;               // completed pready phases waited for
-      auto release = [&](uint32_t& use, int k) -> bool {   // true when the last user is done
-        use -= 1u << (2 * k);
-        return ((use >> (2 * k)) & 3u) == 0u;
-      };
+    const int X = warp == 9 ? 0 : 1;
+    if (lane == 0 && (X == 0 || hasB)) {
+      const uint32_t q_a = smem_u32(Qs) + X * kTileBytes, k_a = smem_u32(Ks), v_a = smem_u32(Vs);
+      const int kloX = klo[X], khiX = khi[X];
+      const uint32_t tS = tm + col_s(X), tP = tm + col_p(X), tO = tm + col_o(X);
       bool ok = mbar_wait(&sm.bar_q, 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        if (ngp)
-          for (int X = 0; X < nX; ++X) {
-            mma_qk(tm + col_sg(X), q_a + X * kTileBytes, smem_u32(KG), 16);
-            umma_commit(&sm.bar_sg[X]);
-          }
-      }
-      // S of the first key tile of each warpgroup
-      auto issue_s = [&](int X, int a) -> bool {
-        const int k = a - kt_lo, s = k % kStages;
-        if (!mbar_wait(&sm.bar_kfull[s], (k / kStages) & 1, abort_flag)) return false;
-        tc_fence_after();
-        mma_qk(tm + col_sp(X), q_a + X * kTileBytes, k_a + s * kTileBytes, 128);
-        if (ngp && a == 2 * pr + X) {
-          mma_qk(tm + col_sgt(X), k_a + s * kTileBytes, smem_u32(QG), 16);
-          umma_commit(&sm.bar_sgt[X]);
+        if (ngp) {
+          mma_qk(tP, q_a, smem_u32(KG), 16);   // S_G
+          umma_commit(&sm.bar_sg[X]);
         }
-        if (release(kuse, k)) umma_commit(&sm.bar_kempty[s]);
+      }
+      // This warpgroup's events come in a fixed order: [P_G stored], then per
+      // key tile "S read" (sfree) and "P stored" (pready).  S of the next
+      // tile is issued at "S read", P V of a tile at "P stored".
+      auto issue_s = [&](int a) -> bool {
+        const int k = a - kt_lo;
+        if (!mbar_wait(&sm.bar_kfull[k], 0, abort_flag)) return false;
+        tc_fence_after();
+        mma_qk(tS, q_a, k_a + k * kTileBytes, 128);
         umma_commit(&sm.bar_sfull[X]);
         return true;
       };
-      // P V of the global keys goes first, so that the commit of the first band
-      // S also covers it (the softmax may rescale O as soon as S is ready)
-      for (int X = 0; ok && X < nX; ++X) {
-        if (ngp) {
-          if (!(ok = mbar_wait(&sm.bar_pready[X], (X ? pu1 : pu0) & 1, abort_flag))) break;
-          (X ? pu1 : pu0) += 1;
+      uint32_t nfree = 0, nready = 0;
+      if (ok) ok = issue_s(kloX);
+      if (ok && ngp) {
+        if ((ok = mbar_wait(&sm.bar_pready[X], (nready++) & 1, abort_flag))) {
           tc_fence_after();
-          mma_pv_ts(tm + col_o(X), tm + col_pg(X), smem_u32(VG), kMaxGlobal / 16, false);
-        }
-        ok = issue_s(X, X ? cur1 : cur0);
-      }
-      // steady state: P V of the current tile, then S of the next, per warpgroup
-      bool more = true;
-      while (ok && more) {
-        more = false;
-        for (int X = 0; ok && X < nX; ++X) {
-          int& cur = X ? cur1 : cur0;
-          int& pu = X ? pu1 : pu0;
-          const int khiX = X ? khi[1] : khi[0], kloX = X ? klo[1] : klo[0];
-          if (cur > khiX) continue;
-          const int a = cur, k = a - kt_lo, s = k % kStages;
-          if (!(ok = mbar_wait(&sm.bar_pready[X], pu & 1, abort_flag))) break;
-          ++pu;
-          if (!(ok = mbar_wait(&sm.bar_vfull[s], (k / kStages) & 1, abort_flag))) break;
-          tc_fence_after();
-          mma_pv_ts(tm + col_o(X), tm + col_sp(X), v_a + s * kTileBytes, kTile / 16,
-                    ngp > 0 || a > kloX);
-          if (release(vuse, k)) umma_commit(&sm.bar_vempty[s]);
-          cur = a + 1;
-          if (cur <= khiX) {
-            if (!(ok = issue_s(X, cur))) break;
-            more = true;
-          } else {
-            umma_commit(&sm.bar_done[X]);
-          }
+          mma_pv_ts(tO, tP + 16, smem_u32(VG), kMaxGlobal / 16, false);   // P_G V_G
+          umma_commit(&sm.bar_pvdone[X]);
         }
       }
-      umma_commit(&sm.bar_fin);
-      drain_wait(&sm.bar_fin, 0);
+      for (int a = kloX; ok && a <= khiX; ++a) {
+        const int k = a - kt_lo;
+        if (!(ok = mbar_wait(&sm.bar_sfree[X], (nfree++) & 1, abort_flag))) break;
+        if (a < khiX) {
+          if (!(ok = issue_s(a + 1))) break;
+        } else if (ngp) {
+          // the last S is read: its columns take S_G and S_Gt for the epilogue
+          tc_fence_after();
+          mma_qk(tS, q_a, smem_u32(KG), 16);
+          mma_qk(tS + 16, k_a + (2 * pr + X - kt_lo) * kTileBytes, smem_u32(QG), 16);
+          umma_commit(&sm.bar_sgend[X]);
+        }
+        if (!(ok = mbar_wait(&sm.bar_pready[X], (nready++) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait(&sm.bar_vfull[k % kVStages], (k / kVStages) & 1, abort_flag))) break;
+        tc_fence_after();
+        mma_pv_ts(tO, tP, v_a + (k % kVStages) * kTileBytes, kTile / 16, ngp > 0 || a > kloX);
+        if (k + kVStages < nk) umma_commit(&sm.bar_vempty[k % kVStages]);   // slot reused
+        umma_commit(&sm.bar_pvdone[X]);
+      }
+      umma_commit(&sm.bar_fin[X]);
+      drain_wait(&sm.bar_fin[X], 0);
     }
     __syncwarp();
+   }
   } else {
     // ------------------------------------------------------------- softmax
+    regs_alloc<kRowsSoftmaxRegs>();
     const int X = warp >> 2;              // warpgroup = query tile of the pair
     const int kloX = X ? klo[1] : klo[0], khiX = X ? khi[1] : khi[0];
     const int wq = warp & 3;              // TMEM lane quarter of this warp
@@ -403,8 +434,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     const bool active = X == 0 || hasB;
     const int i = r0 + r;                 // current index of this query row
     const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
-    const uint32_t tSP = tm + col_sp(X), tO = tm + col_o(X), tSG = tm + col_sg(X),
-                   tPG = tm + col_pg(X), tSGt = tm + col_sgt(X);
+    const uint32_t tS = tm + col_s(X) + lane_off, tP = tm + col_p(X) + lane_off,
+                   tO = tm + col_o(X) + lane_off;
     bool row_global = false;
     for (int g = 0; g < ng; ++g) row_global |= (sm.gc[g] == i);
     const bool valid = (i < n) && !row_global;
@@ -418,14 +449,14 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 
     float m_ref = -INFINITY, lsum = 0.f;
     bool ok = active;
-    bool o_written = false;
-    float xg[kMaxGlobal];
+    uint32_t pv_issued = 0;               // P V products issued for this warpgroup
 
     if (ok && ngp) {
       ok = warp_wait(&sm.bar_sg[X], 0, abort_flag);
       if (ok) {
+        float xg[kMaxGlobal];
         tc_fence_after();
-        tmem_ld16(tSG + lane_off, xg);
+        tmem_ld16(tP, xg);                // S_G
         tmem_ld_wait();
         float mx = -INFINITY;
 #pragma unroll
@@ -444,22 +475,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
           lsum += a + c;
           pk[g / 2] = pack_bf16x2(a, c);
         }
-        tmem_st8(tPG + lane_off, pk);
+        tmem_st8(tP + 16, pk);            // P_G
         tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&sm.bar_pready[X]);
-        o_written = true;
+        pv_issued = 1;
       }
     }
 
     // Softmax with a running reference m_ref (base-2 units): P = exp2(x - ref).
-    // Each 64-column half of a tile is loaded once; its maximum is taken before
-    // its exponentials, and when it exceeds the reference by more than 8 the
-    // reference is raised there: O (all earlier P V of this warpgroup have
-    // completed, since S of this tile was issued after them), the row sum, this
-    // tile's partial sums and the already-stored first half of P are rescaled
-    // exactly.  P values therefore stay below 2^8.
-    float x[64];
+    // The tile's maximum is taken before its exponentials; when it exceeds the
+    // reference by more than 8, the reference is raised and O (all earlier
+    // P V complete) and the row sum are rescaled exactly.  P stays below 2^8.
+    const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
     for (int t = 0; ok && t <= khiX - kloX; ++t) {
       const int j0 = (kloX + t) * kTile;
       // 32-column chunks of this tile that intersect the warp's band
@@ -468,105 +496,94 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       const int a = lo - j0, e = hi - j0;
       if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
-      float ps[4] = {0.f, 0.f, 0.f, 0.f};
+      float x[128];
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        // two 32-column chunks into x[0..63], keys outside the band masked
+      for (int ch = 0; ch < 4; ++ch) {
+        if (ch >= ch_lo && ch <= ch_hi) {
+          tmem_ld32(tS + 32 * ch, x + 32 * ch);
+        } else {
 #pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          const int ch = 2 * hf + c2;
-          if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(tSP + lane_off + 32 * ch, x + 32 * c2);
-        }
-        tmem_ld_wait();
-        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          const int ch = 2 * hf + c2;
-          if (ch < ch_lo || ch > ch_hi) continue;
-          if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
-#pragma unroll
-            for (int k = 0; k < 32; ++k) {
-              const int c = 32 * ch + k;
-              x[32 * c2 + k] = (c >= a && c <= e) ? x[32 * c2 + k] : -INFINITY;
-            }
-          }
-#pragma unroll
-          for (int k = 0; k < 32; ++k) pm[k & 3] = fmaxf(pm[k & 3], x[32 * c2 + k]);
-        }
-        const float hmax = fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])) * kLogitScale2;
-        const bool raise = hmax > m_ref + 8.f;
-        if (__any_sync(0xffffffffu, raise)) {
-          float f = 1.f;
-          if (raise) {
-            f = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - hmax);
-            m_ref = hmax;
-            lsum *= f;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) ps[k] *= f;
-          }
-          // small pieces keep the register footprint next to x[] low
-          float o[8];
-          if (o_written) {
-#pragma unroll 1
-            for (int c = 0; c < 64; c += 8) {
-              tmem_ld8(tO + lane_off + c, o);
-              tmem_ld_wait();
-#pragma unroll
-              for (int k = 0; k < 8; ++k) o[k] *= f;
-              tmem_st8(tO + lane_off + c, reinterpret_cast<const uint32_t*>(o));
-              tmem_st_wait();   // o is reused
-            }
-          }
-          if (hf == 1) {
-            // the first half of this tile's P, already stored: 32 columns of bf16 pairs
-            tmem_st_wait();
-#pragma unroll 1
-            for (int c = 0; c < 32; c += 8) {
-              tmem_ld8(tSP + lane_off + c, o);
-              tmem_ld_wait();
-#pragma unroll
-              for (int k = 0; k < 8; ++k) {
-                const uint32_t w = __float_as_uint(o[k]);
-                const float lo16 = __uint_as_float(w << 16) * f;
-                const float hi16 = __uint_as_float(w & 0xffff0000u) * f;
-                o[k] = __uint_as_float(pack_bf16x2(lo16, hi16));
-              }
-              tmem_st8(tSP + lane_off + c, reinterpret_cast<const uint32_t*>(o));
-              tmem_st_wait();
-            }
-          }
-        }
-        const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {   // 16-column quarters of the half
-          const int ch = 2 * hf + (q >> 1);
-          uint32_t pk[8];
-          if (ch >= ch_lo && ch <= ch_hi) {
-#pragma unroll
-            for (int k = 0; k < 16; k += 2) {
-              const float u = ex2(fmaf(x[16 * q + k], kLogitScale2, nref));
-              const float v = ex2(fmaf(x[16 * q + k + 1], kLogitScale2, nref));
-              ps[k & 3] += u;
-              ps[(k & 3) + 1] += v;
-              pk[k >> 1] = pack_bf16x2(u, v);
-            }
-          } else {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) pk[k] = 0u;
-          }
-          tmem_st8(tSP + lane_off + 8 * (4 * hf + q), pk);
+          for (int k = 0; k < 32; ++k) x[32 * ch + k] = -INFINITY;
         }
       }
+      tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(&sm.bar_sfree[X]);   // S is in registers: the next S may overwrite it
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) {
+        if (ch < ch_lo || ch > ch_hi) continue;
+        if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
+          // edge chunk: keys outside this row's band take no part
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            const int c = 32 * ch + k;
+            x[32 * ch + k] = (c >= a && c <= e) ? x[32 * ch + k] : -INFINITY;
+          }
+        }
+      }
+      float m0 = x[0], m1 = x[1];
+#pragma unroll
+      for (int k = 2; k < 128; k += 4) {
+        m0 = fmax3(m0, x[k], x[k + 1]);
+        m1 = fmax3(m1, x[k + 2], x[k + 3]);
+      }
+      const float tmax = fmaxf(m0, m1) * kLogitScale2;
+      const bool raise = tmax > m_ref + 8.f;
+      float f = 1.f;
+      if (raise) {
+        f = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - tmax);
+        m_ref = tmax;
+        lsum *= f;
+      }
+      // every earlier P V has completed: O is final for a rescale and the P
+      // columns of this warpgroup are free again
+      if (pv_issued > 0 && !(ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag)))
+        break;
+      tc_fence_after();
+      if (__any_sync(0xffffffffu, raise) && pv_issued > 0) {
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 16) {
+          float o[16];
+          tmem_ld16(tO + c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) o[k] *= f;
+          tmem_st16(tO + c, reinterpret_cast<const uint32_t*>(o));
+          tmem_st_wait();   // o is reused
+        }
+      }
+      const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
+      const uint64_t n2 = f2_pack(nref, nref);
+      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) {   // 32 keys = 16 columns of P per step
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float u, w;
+          f2_unpack(f2_fma(f2_pack(x[32 * ch + k], x[32 * ch + k + 1]), c2, n2), u, w);
+          u = ex2(u);
+          w = ex2(w);
+          if (k & 2) s2b = f2_add(s2b, f2_pack(u, w));
+          else s2a = f2_add(s2a, f2_pack(u, w));
+          pk[k >> 1] = pack_bf16x2(u, w);
+        }
+        tmem_st16(tP + 16 * ch, pk);
+      }
+      float sa, sb, sc2, sd;
+      f2_unpack(s2a, sa, sb);
+      f2_unpack(s2b, sc2, sd);
+      lsum += (sa + sb) + (sc2 + sd);
       tmem_st_wait();
-      lsum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
       tc_fence_before();
       mbar_arrive(&sm.bar_pready[X]);
-      o_written = true;
+      ++pv_issued;
     }
 
     // ---- epilogue: O, LSE
     float lse = INFINITY;
-    if (ok && (ok = warp_wait(&sm.bar_done[X], 0, abort_flag))) {
+    if (ok && pv_issued > 0 &&
+        (ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag))) {
       tc_fence_after();
       const float inv = 1.f / lsum;
       lse = valid ? m_ref + lg2(lsum) : INFINITY;
@@ -574,16 +591,16 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 #pragma unroll
       for (int c = 0; c < 64; c += 32) {
         float o[32];
-        tmem_ld32(tO + lane_off + c, o);
+        tmem_ld32(tO + c, o);
         tmem_ld_wait();
         if (valid) {
 #pragma unroll
           for (int k = 0; k < 32; k += 8) {
-            uint4 v = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
-                                 pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
-                                 pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
-                                 pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
-            *reinterpret_cast<uint4*>(orow + c + k) = v;
+            uint4 u4 = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
+                                  pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
+                                  pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
+                                  pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
+            *reinterpret_cast<uint4*>(orow + c + k) = u4;
           }
         }
       }
@@ -592,39 +609,46 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 
     if (active && ngp) {
       // Per-warp partial results (32 rows / 32 keys each), reduced with
-      // shuffles and merged later in a fixed order: no barrier here.
+      // butterfly shuffles and merged later in a fixed order: no barrier here.
       const size_t slot0 =
           (((static_cast<size_t>(b) * p.H + h) * p.T + qt) * 4 + wq) * kMaxGlobal;
-      // far-row column sums of the global keys: rows outside the key's band
-      if (ok) {
-        tmem_ld16(tSG + lane_off, xg);
-        tmem_ld_wait();
-      }
-#pragma unroll
-      for (int g = 0; g < kMaxGlobal; ++g) {
-        if (g >= ng) break;   // warp-uniform
-        const bool use = ok && valid && abs(i - sm.gc[g]) > p.w;
-        const float v = warp_sum(use ? ex2(fmaf(xg[g], kLogitScale2, -lse)) : 0.f);
-        if (lane == g) p.gpart[slot0 + g] = v;
-      }
-      // (max, sum) of each global query over this warp's keys j = 128 qt + r
-      const bool ok2 = ok && warp_wait(&sm.bar_sgt[X], 0, abort_flag);
+      const int gme = lane >> 1;            // global index this lane reports
+      const bool writer = (lane & 1) == 0 && gme < ng;
+      float xg[kMaxGlobal], xt[kMaxGlobal];
+      const bool ok2 = ok && warp_wait(&sm.bar_sgend[X], 0, abort_flag);
       if (ok2) {
         tc_fence_after();
-        tmem_ld16(tSGt + lane_off, xg);
+        tmem_ld16(tS, xg);                  // S_G
+        tmem_ld16(tS + 16, xt);             // S_Gt
         tmem_ld_wait();
       }
-      const bool key_ok = ok2 && (r0 + r < n);
+      // far-row column sums of the global keys: rows outside the key's band
+      float e16[kMaxGlobal];
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g) {
-        if (g >= ng) break;   // warp-uniform
-        const float y = key_ok ? xg[g] * kLogitScale2 : -INFINITY;
-        const float m = warp_max(y);
-        const float sum = warp_sum(m == -INFINITY ? 0.f : ex2(y - m));
-        if (lane == g) {
-          p.gstat[2 * (slot0 + g)] = m;
-          p.gstat[2 * (slot0 + g) + 1] = sum;
-        }
+        const bool use = ok2 && valid && g < ng && abs(i - sm.gc[g]) > p.w;
+        e16[g] = use ? ex2(fmaf(xg[g], kLogitScale2, -lse)) : 0.f;
+      }
+      const float gsum = warp_reduce16(e16, OpAdd());
+      if (writer) p.gpart[slot0 + gme] = gsum;
+      // (max, sum) of each global query over this warp's keys j = 128 qt + r
+      const bool key_ok = ok2 && (r0 + r < n);
+      float y[kMaxGlobal];
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        y[g] = (key_ok && g < ng) ? xt[g] * kLogitScale2 : -INFINITY;
+        e16[g] = y[g];
+      }
+      const float mme = warp_reduce16(e16, OpMax());
+#pragma unroll
+      for (int g = 0; g < kMaxGlobal; ++g) {
+        const float mg = __shfl_sync(0xffffffffu, mme, 2 * g);
+        e16[g] = mg == -INFINITY ? 0.f : ex2(y[g] - mg);
+      }
+      const float sme = warp_reduce16(e16, OpAdd());
+      if (writer) {
+        p.gstat[2 * (slot0 + gme)] = mme;
+        p.gstat[2 * (slot0 + gme) + 1] = sme;
       }
       if (qt == 0) {
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
@@ -650,10 +674,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 // Tensor memory per warpgroup X: S^T [128 X, 128 X + 128), S^T against the
 // global queries [256 + 16 X, +16), the global rows' P V [320 + 64 X, +64).
 constexpr int kColsThreads = 320;
+constexpr int kColsStages = 4;      // Q ring depth
 
 struct ColsSmem {
   uint64_t bar_kv;
-  uint64_t bar_qfull[kStages], bar_qempty[kStages];
+  uint64_t bar_qfull[kColsStages], bar_qempty[kColsStages];
   uint64_t bar_sfull[2], bar_sfree[2], bar_sg[2], bar_pg[2], bar_og[2], bar_fin;
   uint32_t tmem_base;
   int abort;
@@ -668,7 +693,7 @@ struct ColsSmem {
 
 // dynamic shared memory: K and V of both key tiles, the Q ring, the global
 // queries, and one A tile (32 KB) per warpgroup for the global rows' P V
-constexpr uint32_t kColsDyn = kTileBytes * (4 + kStages) + kGTileBytes + 4 * kTileBytes + 1024;
+constexpr uint32_t kColsDyn = kTileBytes * (4 + kColsStages) + kGTileBytes + 4 * kTileBytes + 1024;
 
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
                                   ColsSmem& sm);
@@ -700,8 +725,8 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   uint8_t* Ks = base;                              // 2 tiles
   uint8_t* Vs = Ks + 2 * kTileBytes;               // 2 tiles
   uint8_t* Pg = Vs + 2 * kTileBytes;               // 2 x 32 KB A tiles
-  uint8_t* Qs = Pg + 4 * kTileBytes;               // kStages tiles
-  uint8_t* QG = Qs + kStages * kTileBytes;
+  uint8_t* Qs = Pg + 4 * kTileBytes;               // kColsStages tiles
+  uint8_t* QG = Qs + kColsStages * kTileBytes;
   __shared__ ColsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -718,7 +743,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
 
   if (tid == 0) {
     mbar_init(&sm.bar_kv, 1);
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kColsStages; ++s) {
       mbar_init(&sm.bar_qfull[s], 1);
       mbar_init(&sm.bar_qempty[s], 1);
     }
@@ -755,17 +780,17 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     if (lane == 0) {
       bool ok = true;
       for (int q = 0; ok && q < nq; ++q) {
-        const int s = q % kStages;
-        if (q >= kStages &&
-            !(ok = mbar_wait(&sm.bar_qempty[s], ((q / kStages) - 1) & 1, abort_flag)))
+        const int s = q % kColsStages;
+        if (q >= kColsStages &&
+            !(ok = mbar_wait(&sm.bar_qempty[s], ((q / kColsStages) - 1) & 1, abort_flag)))
           break;
         mbar_arrive_expect_tx(&sm.bar_qfull[s], kTileBytes);
         load_tile(maps, 0, rs, h, (qt_lo + q) * kTile, Qs + s * kTileBytes, &sm.bar_qfull[s]);
       }
       drain_wait(&sm.bar_kv, 0);
-      for (int s = 0; s < kStages && s < nq; ++s) {
-        const int last = s + kStages * ((nq - 1 - s) / kStages);
-        drain_wait(&sm.bar_qfull[s], (last / kStages) & 1);
+      for (int s = 0; s < kColsStages && s < nq; ++s) {
+        const int last = s + kColsStages * ((nq - 1 - s) / kColsStages);
+        drain_wait(&sm.bar_qfull[s], (last / kColsStages) & 1);
       }
     }
   } else if (warp == 9) {
@@ -783,8 +808,8 @@ __global__ void __launch_bounds__(kColsThreads, 1)
           }
       }
       for (int q = 0; ok && q < nq; ++q) {
-        const int s = q % kStages, a = qt_lo + q;
-        if (!(ok = mbar_wait(&sm.bar_qfull[s], (q / kStages) & 1, abort_flag))) break;
+        const int s = q % kColsStages, a = qt_lo + q;
+        if (!(ok = mbar_wait(&sm.bar_qfull[s], (q / kColsStages) & 1, abort_flag))) break;
         for (int X = 0; ok && X < nX; ++X) {
           if (a < (X ? qlo[1] : qlo[0]) || a > (X ? qhi[1] : qhi[0])) continue;
           if (su[X] > 0 && !(ok = mbar_wait(&sm.bar_sfree[X], (su[X] - 1) & 1, abort_flag))) break;

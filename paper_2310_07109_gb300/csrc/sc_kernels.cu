@@ -1167,59 +1167,92 @@ constexpr int kPrepThreads = 1024;
 
 __global__ void __launch_bounds__(kPrepThreads)
     sc_prep_kernel(const PrepParams pp) {
-  const int b = blockIdx.x, tid = threadIdx.x;
-  __shared__ int scan[kPrepThreads];
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  __shared__ int wsum[kPrepThreads / 32];
   __shared__ int spos[kMaxLen];
+  __shared__ int gfound[kMaxGlobal];
   __shared__ int s_n;
-  int n;
   if (pp.pos_in == nullptr) {
-    // stack mode: real tokens of the padded sequence, in order
     const int L = pp.L;
-    const int per = (L + kPrepThreads - 1) / kPrepThreads;
-    const int c0 = min(L, tid * per), c1 = min(L, c0 + per);
-    int cnt = 0;
-    for (int c = c0; c < c1; ++c)
-      cnt += pp.pad_mask ? (pp.pad_mask[static_cast<size_t>(b) * L + c] != 0) : 1;
-    scan[tid] = cnt;
-    __syncthreads();
-    for (int off = 1; off < kPrepThreads; off <<= 1) {
-      const int v = tid >= off ? scan[tid - off] : 0;
+    int32_t* out = pp.pos_out + static_cast<size_t>(b) * L;
+    if (pp.pad_mask == nullptr) {
+      // no padding: the current tokens are positions 0..L-1
+      for (int c = tid; c < L; c += kPrepThreads) {
+        out[c] = c;
+        spos[c] = c;
+      }
+      if (tid == 0) {
+        s_n = L;
+        pp.len_out[b] = L;
+      }
+    } else {
+      // stack mode with padding: the real tokens in order; thread tid takes
+      // one contiguous run, runs are placed by a scan of their counts
+      const uint8_t* mask = pp.pad_mask + static_cast<size_t>(b) * L;
+      const int per = (L + kPrepThreads - 1) / kPrepThreads;
+      const int c0 = min(L, tid * per), c1 = min(L, c0 + per);
+      int cnt = 0;
+      for (int c = c0; c < c1; ++c) cnt += mask[c] != 0;
+      int x = cnt;   // inclusive scan within the warp
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x += y;
+      }
+      if (lane == 31) wsum[warp] = x;
       __syncthreads();
-      scan[tid] += v;
+      if (warp == 0) {
+        int w = wsum[lane];
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, w, off);
+          if (lane >= off) w += y;
+        }
+        wsum[lane] = w;
+      }
       __syncthreads();
-    }
-    int out = scan[tid] - cnt;
-    for (int c = c0; c < c1; ++c) {
-      if (pp.pad_mask && !pp.pad_mask[static_cast<size_t>(b) * L + c]) continue;
-      pp.pos_out[static_cast<size_t>(b) * L + out] = c;
-      spos[out] = c;
-      ++out;
-    }
-    if (tid == kPrepThreads - 1) {
-      s_n = scan[kPrepThreads - 1];
-      pp.len_out[b] = s_n;
+      int at = (warp > 0 ? wsum[warp - 1] : 0) + x - cnt;
+      for (int c = c0; c < c1; ++c) {
+        if (!mask[c]) continue;
+        out[at] = c;
+        spos[at] = c;
+        ++at;
+      }
+      if (tid == 0) {
+        s_n = wsum[kPrepThreads / 32 - 1];
+        pp.len_out[b] = s_n;
+      }
     }
   } else {
     if (tid == 0) s_n = pp.len_in[b];
     __syncthreads();
-    for (int c = tid; c < s_n; c += kPrepThreads) spos[c] = pp.pos_in[static_cast<size_t>(b) * pp.L + c];
+    for (int c = tid; c < s_n; c += kPrepThreads)
+      spos[c] = pp.pos_in[static_cast<size_t>(b) * pp.L + c];
   }
   __syncthreads();
-  n = s_n;
-  if (tid == 0) {
-    // global positions are sorted and positions increase with the current
-    // index, so the matches come out in increasing current order
-    int m = 0;
-    for (int g = 0; g < pp.n_global; ++g) {
-      const int target = pp.global_pos[g];
+  const int n = s_n;
+  // current index of each global position (one thread each; binary search:
+  // positions increase with the current index)
+  if (tid < kMaxGlobal) {
+    int found = -1;
+    if (tid < pp.n_global) {
+      const int target = pp.global_pos[tid];
       int lo = 0, hi = n - 1;
       while (lo <= hi) {
         const int mid = (lo + hi) >> 1;
         if (spos[mid] < target) lo = mid + 1;
         else hi = mid - 1;
       }
-      if (lo < n && spos[lo] == target) pp.gcur[b * kMaxGlobal + m++] = lo;
+      if (lo < n && spos[lo] == target) found = lo;
     }
+    gfound[tid] = found;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    // global positions are sorted, so the matches come out in increasing order
+    int m = 0;
+    for (int g = 0; g < kMaxGlobal; ++g)
+      if (gfound[g] >= 0) pp.gcur[b * kMaxGlobal + m++] = gfound[g];
     pp.ng[b] = m;
     // single-layer calls read their (already current-order) inputs in place
     pp.ident[b] = (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1) ? 1 : 0;

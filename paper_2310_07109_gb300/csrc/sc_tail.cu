@@ -43,7 +43,7 @@ constexpr uint32_t kTailDyn = 120 * 1024;
 static_assert(3 * kTailOpBytes + 1024 <= kTailDyn, "tail operands exceed the dynamic shared memory");
 
 struct TailSmem {
-  uint64_t bar_free, bar_fin;
+  uint64_t bar_free[2], bar_fin;
   uint64_t bar_s[2], bar_p[2], bar_o[2], bar_st[2];
   uint32_t tmem_base;
   int abort;
@@ -52,7 +52,7 @@ struct TailSmem {
   int gpos[kMaxGlobal];               // global positions (sorted), -1 past n_global
   uint32_t gbits[2][kTailMax / 32];   // global flags of the current / next token list
   int32_t pos[2][kTailMax];           // original positions of the current / next tokens
-  alignas(16) float lse[kTailMax];
+  alignas(16) float nlse[kTailMax];   // -LSE of each query row (-inf past n)
   float colsum[2][kTailMax];          // this head's column sums, by layer parity
 };
 
@@ -133,7 +133,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   for (int k = tid; k < static_cast<int>(3 * kTailOpBytes / 16); k += kTailThreads)
     reinterpret_cast<uint4*>(base)[k] = make_uint4(0u, 0u, 0u, 0u);
   if (tid == 0) {
-    mbar_init(&sm.bar_free, 256);
+    mbar_init(&sm.bar_free[0], 128);
+    mbar_init(&sm.bar_free[1], 128);
     mbar_init(&sm.bar_fin, 1);
     for (int X = 0; X < 2; ++X) {
       mbar_init(&sm.bar_s[X], 1);
@@ -175,22 +176,24 @@ __global__ void __launch_bounds__(kTailThreads, 1)
 
     // ---- rows of the current tokens: 16-byte pieces, 128B-swizzled tiles
     {
+      // thread tid copies 16-byte piece (tid & 7) of every 36th row, the
+      // same piece of Q, K and V from one address computation
       const size_t tok0 = (static_cast<size_t>(l) * B + b) * L;
-#pragma unroll
-      for (int t = 0; t < 3; ++t) {
-        const uint16_t* src = p.src[t];
-        for (int c = tid; c < 8 * n; c += kTailThreads) {
-          const int r = c >> 3, piece = c & 7;
-          const size_t row = (tok0 + sm.pos[cur][r]) * H + h;
-          cp_async16(q_a + t * kTailOpBytes + sw128_offset(r, piece), src + row * kHeadDim + 8 * piece);
-        }
+      const int piece = tid & 7;
+      for (int r = tid >> 3; r < n; r += kTailThreads / 8) {
+        const size_t off = ((tok0 + sm.pos[cur][r]) * H + h) * kHeadDim + 8 * piece;
+        const uint32_t so = sw128_offset(r, piece);
+        cp_async16(q_a + so, p.src[0] + off);
+        cp_async16(k_a + so, p.src[1] + off);
+        cp_async16(v_a + so, p.src[2] + off);
       }
       if (l + 1 < n_layers) {
         // the next layer's tokens are a subset of the current ones
         const size_t tok1 = (static_cast<size_t>(l + 1) * B + b) * L;
-        for (int c = tid; c < 3 * n; c += kTailThreads) {
-          const int t = c >= 2 * n ? 2 : (c >= n ? 1 : 0), r = c - t * n;
-          prefetch_l2_line(p.src[t] + ((tok1 + sm.pos[cur][r]) * H + h) * kHeadDim);
+        for (int r = tid; r < n; r += kTailThreads) {
+          const size_t off = ((tok1 + sm.pos[cur][r]) * H + h) * kHeadDim;
+#pragma unroll
+          for (int t = 0; t < 3; ++t) prefetch_l2_line(p.src[t] + off);
         }
       }
       cp_async_wait_all();
@@ -212,6 +215,14 @@ __global__ void __launch_bounds__(kTailThreads, 1)
                       sdesc_sw128(k_a + 32 * k), id_s, k > 0);
           umma_commit(&sm.bar_s[X]);
         }
+        if (nX == 1) {
+          // one query tile leaves the second half of tensor memory free: S^T
+          // of the (single) key tile goes there at once
+#pragma unroll
+          for (int k = 0; k < kHeadDim / 16; ++k)
+            umma_bf16(tm + 256u, sdesc_sw128(k_a + 32 * k), sdesc_sw128(q_a + 32 * k), id_s, k > 0);
+          umma_commit(&sm.bar_st[0]);
+        }
         bool ok = true;
         for (int X = 0; ok && X < nX; ++X) {
           if (!(ok = mbar_wait(&sm.bar_p[X], (X ? cnt1 : cnt0) & 1, abort_flag))) break;
@@ -221,16 +232,16 @@ __global__ void __launch_bounds__(kTailThreads, 1)
                          sdesc_sw128(v_a + 2048u * k), id_pv, k > 0);
           umma_commit(&sm.bar_o[X]);
         }
-        if (ok) ok = mbar_wait(&sm.bar_free, it & 1, abort_flag);
-        if (ok) {
+        // two query tiles: S^T of key tile X overwrites warpgroup X's columns
+        // once that warpgroup has read its O
+        for (int X = 0; ok && nX == 2 && X < 2; ++X) {
+          if (!(ok = mbar_wait(&sm.bar_free[X], it & 1, abort_flag))) break;
           tc_fence_after();
-          for (int X = 0; X < nX; ++X) {
 #pragma unroll
-            for (int k = 0; k < kHeadDim / 16; ++k)
-              umma_bf16(tm + 256u * X, sdesc_sw128(k_a + X * kTileBytes + 32 * k),
-                        sdesc_sw128(q_a + 32 * k), id_s, k > 0);
-            umma_commit(&sm.bar_st[X]);
-          }
+          for (int k = 0; k < kHeadDim / 16; ++k)
+            umma_bf16(tm + 256u * X, sdesc_sw128(k_a + X * kTileBytes + 32 * k),
+                      sdesc_sw128(q_a + 32 * k), id_s, k > 0);
+          umma_commit(&sm.bar_st[X]);
         }
       }
       __syncwarp();
@@ -268,7 +279,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         // pass 2: P = exp2(S - max) (masked keys: exp2(-inf) = 0), row sum, and
         // P as bf16 pairs over the first half of each step's columns (they
         // land in columns that this or earlier steps occupied, already read)
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2), n2 = f2_pack(nmc, nmc);
+        uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
         for (int q2 = 0; q2 < nc2; ++q2) {
           float x[64];
           tmem_ld32(tS + lane_off + 64 * q2, x);
@@ -281,17 +293,22 @@ __global__ void __launch_bounds__(kTailThreads, 1)
             uint32_t pk[16];
 #pragma unroll
             for (int k = 0; k < 32; k += 2) {
-              const float u = ex2(fmaf(xh[k], kLogitScale2, nmc));
-              const float v = ex2(fmaf(xh[k + 1], kLogitScale2, nmc));
-              ls[k & 3] += u;
-              ls[(k & 3) + 1] += v;
+              float u, v;
+              f2_unpack(f2_fma(f2_pack(xh[k], xh[k + 1]), c2, n2), u, v);
+              u = ex2(u);
+              v = ex2(v);
+              if (k & 2) s2b = f2_add(s2b, f2_pack(u, v));
+              else s2a = f2_add(s2a, f2_pack(u, v));
               pk[k >> 1] = pack_bf16x2(u, v);
             }
             tmem_st16(tS + lane_off + 32 * q2 + 16 * hq, pk);
           }
         }
         tmem_st_wait();
-        const float lsum = (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        float la, lb, lc, ld;
+        f2_unpack(s2a, la, lb);
+        f2_unpack(s2b, lc, ld);
+        const float lsum = (la + lb) + (lc + ld);
         tc_fence_before();
         mbar_arrive(&sm.bar_p[X]);
         if (tail_wait(&sm.bar_o[X], ph, abort_flag)) {
@@ -316,37 +333,45 @@ __global__ void __launch_bounds__(kTailThreads, 1)
           }
         }
       }
-      sm.lse[i] = lse;
-      tail_named_sync();   // every LSE is written; no thread still reads S, P or O
+      // this warpgroup has read its S, P and O: with two query tiles its
+      // columns take S^T of key tile X next
       tc_fence_before();
-      mbar_arrive(&sm.bar_free);
+      mbar_arrive(&sm.bar_free[X]);
+      sm.nlse[i] = -lse;
+      tail_named_sync();   // every LSE is written
 
       // columns: key j = i of this thread, summed over the query rows
       float acc = 0.f;
       if (use && tail_wait(&sm.bar_st[X], ph, abort_flag)) {
         tc_fence_after();
-        float a4[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint32_t tST = nX == 1 ? tm + 256u : tS;
+        const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
+        uint64_t a2a = f2_pack(0.f, 0.f), a2b = a2a;
         for (int q2 = 0; q2 < nc2; ++q2) {
           float x[64];
-          tmem_ld32(tS + lane_off + 64 * q2, x);
-          tmem_ld32(tS + lane_off + 64 * q2 + 32, x + 32);
+          tmem_ld32(tST + lane_off + 64 * q2, x);
+          tmem_ld32(tST + lane_off + 64 * q2 + 32, x + 32);
           tmem_ld_wait();
 #pragma unroll
           for (int hq = 0; hq < 2; ++hq) {
             float* xh = x + 32 * hq;
             apply_mask(xh, partner_mask(me, sm, cur, 2 * q2 + hq, n));
-            const float* lw = sm.lse + 64 * q2 + 32 * hq;
+            const float* lw = sm.nlse + 64 * q2 + 32 * hq;
 #pragma unroll
             for (int k = 0; k < 32; k += 4) {
               const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
-              a4[0] += ex2(fmaf(xh[k + 0], kLogitScale2, -l4.x));
-              a4[1] += ex2(fmaf(xh[k + 1], kLogitScale2, -l4.y));
-              a4[2] += ex2(fmaf(xh[k + 2], kLogitScale2, -l4.z));
-              a4[3] += ex2(fmaf(xh[k + 3], kLogitScale2, -l4.w));
+              float e0, e1, e2, e3;
+              f2_unpack(f2_fma(f2_pack(xh[k], xh[k + 1]), c2, f2_pack(l4.x, l4.y)), e0, e1);
+              f2_unpack(f2_fma(f2_pack(xh[k + 2], xh[k + 3]), c2, f2_pack(l4.z, l4.w)), e2, e3);
+              a2a = f2_add(a2a, f2_pack(ex2(e0), ex2(e1)));
+              a2b = f2_add(a2b, f2_pack(ex2(e2), ex2(e3)));
             }
           }
         }
-        acc = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+        float a0, a1, a2, a3;
+        f2_unpack(a2a, a0, a1);
+        f2_unpack(a2b, a2, a3);
+        acc = (a0 + a2) + (a1 + a3);
       }
       if (use) sm.colsum[par][i] = acc;
     }

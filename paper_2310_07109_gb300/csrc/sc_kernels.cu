@@ -687,7 +687,8 @@ struct ColsSmem {
   alignas(16) float lse[kPairTiles * kTile];  // read as float4
   float gsum[kMaxGlobal];
   int flag;
-  int scan[kColsThreads];
+  float wpart[kColsThreads / 32];
+  int wcount[kColsThreads / 32];
   int gnew[kMaxGlobal];
 };
 
@@ -994,41 +995,58 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   __threadfence();
   const int j0 = 2 * pr * kTile;
   const int jn = min(n, j0 + 2 * kTile);
-  // far-row partial sums of the global keys that lie in this pair: one warp per
-  // global key, summed over heads and query tiles in a fixed order
-  if (warp < 8) {
-    for (int g = warp; g < ng; g += 8) {
-      const int cg = sm.gc[g];
-      float v = 0.f;
-      if (cg >= j0 && cg < jn) {
-        const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * 4 * kMaxGlobal + g;
-#pragma unroll 4
-        for (int k = lane; k < p.H * Tn * 4; k += 32) {
-          const int hh = k / (Tn * 4), q4 = k - hh * (Tn * 4);   // q4 = 4 * tile + warp
-          v += __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal);
-        }
-        v = warp_sum(v);
-      }
-      if (lane == 0) sm.gsum[g] = v;
+  // far-row partial sums of each global key that lies in this pair, over heads
+  // and (query tile, warp) slices: spread over the whole CTA, every load
+  // issued before the sums, reduced in a fixed order
+  for (int g = 0; g < ng; ++g) {
+    const int cg = sm.gc[g];
+    if (cg < j0 || cg >= jn) continue;   // CTA-uniform
+    const int per_head = Tn * 4, total = p.H * per_head;
+    const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * 4 * kMaxGlobal + g;
+    constexpr int kPer = 8;
+    float e[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int k = tid + u * kColsThreads;
+      const int hh = k / per_head, q4 = k - hh * per_head;   // q4 = 4 * tile + warp
+      e[u] = k < total ? __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal) : 0.f;
     }
+    float v = 0.f;
+    for (int k0 = 0; k0 < total; k0 += kPer * kColsThreads) {
+      if (k0 > 0) {
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) {
+          const int k = k0 + tid + u * kColsThreads;
+          const int hh = k / per_head, q4 = k - hh * per_head;
+          e[u] = k < total ? __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal)
+                           : 0.f;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kPer; ++u) v += e[u];
+    }
+    v = warp_sum(v);
+    if (lane == 0) sm.wpart[warp] = v;
+    __syncthreads();
+    if (tid == 0) {
+      float a = 0.f;
+      for (int w = 0; w < kColsThreads / 32; ++w) a += sm.wpart[w];
+      sm.gsum[g] = a;
+    }
+    __syncthreads();
   }
-  __syncthreads();
   if (tid < 2 * kTile && j0 + tid < jn) {
     const int jj = j0 + tid;
     const float* ap = p.acc + static_cast<size_t>(b) * p.H * p.L + jj;
     float a = 0.f;
-    int hh = 0;
-    for (; hh + 4 <= p.H; hh += 4) {
-      const float v0 = __ldcg(ap + static_cast<size_t>(hh) * p.L);
-      const float v1 = __ldcg(ap + static_cast<size_t>(hh + 1) * p.L);
-      const float v2 = __ldcg(ap + static_cast<size_t>(hh + 2) * p.L);
-      const float v3 = __ldcg(ap + static_cast<size_t>(hh + 3) * p.L);
-      a += v0;
-      a += v1;
-      a += v2;
-      a += v3;
+    for (int h0 = 0; h0 < p.H; h0 += 16) {   // heads in order, 16 loads in flight
+      float e[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        e[u] = h0 + u < p.H ? __ldcg(ap + static_cast<size_t>(h0 + u) * p.L) : 0.f;
+#pragma unroll
+      for (int u = 0; u < 16; ++u) a += e[u];
     }
-    for (; hh < p.H; ++hh) a += __ldcg(ap + static_cast<size_t>(hh) * p.L);
     for (int g = 0; g < ng; ++g)
       if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
@@ -1047,46 +1065,76 @@ __global__ void __launch_bounds__(kColsThreads, 1)
 }
 
 // Order-preserving compaction of sequence b's kept tokens, the next layer's
-// global list, and the bf16 outputs of the global rows.  One CTA.
+// global list, and the bf16 outputs of the global rows.  One CTA; thread t
+// takes one contiguous run of at most kRun tokens, loaded in one round.
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
                                   ColsSmem& sm) {
-  const int tid = threadIdx.x;
+  constexpr int kRun = (kMaxLen + kColsThreads - 1) / kColsThreads;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int per = (n + kColsThreads - 1) / kColsThreads;
   const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
   const uint8_t* keep = p.keep + static_cast<size_t>(b) * p.L;
-  int cnt = 0;
-#pragma unroll 8
-  for (int c = c0; c < c1; ++c) cnt += __ldcg(keep + c);
-  sm.scan[tid] = cnt;
-  __syncthreads();
-  // exclusive scan over kColsThreads counts (Hillis-Steele in shared memory)
-  for (int off = 1; off < kColsThreads; off <<= 1) {
-    const int v = tid >= off ? sm.scan[tid - off] : 0;
-    __syncthreads();
-    sm.scan[tid] += v;
-    __syncthreads();
-  }
-  int out = sm.scan[tid] - cnt;
-  const int total = sm.scan[kColsThreads - 1];
-  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
-  if (tid < kMaxGlobal) sm.gnew[tid] = -1;
-  __syncthreads();
   const int32_t* pos = v.pos + static_cast<size_t>(b) * p.L;
   int32_t* pos_out = v.pos_out + static_cast<size_t>(b) * p.L;
-  for (int c = c0; c < c1; ++c) {
-    if (!__ldcg(keep + c)) continue;
-    pos_out[out] = __ldg(pos + c);
+  uint8_t kf[kRun];
+  int32_t ps[kRun];
+#pragma unroll
+  for (int k = 0; k < kRun; ++k) {
+    const int c = c0 + k;
+    kf[k] = c < c1 ? __ldcg(keep + c) : 0;
+    ps[k] = c < c1 ? __ldcg(pos + c) : 0;
+  }
+  int cnt = 0;
+#pragma unroll
+  for (int k = 0; k < kRun; ++k) cnt += kf[k];
+  // exclusive scan of the run counts: within the warp, then over the warps
+  int x = cnt;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, off);
+    if (lane >= off) x += y;
+  }
+  if (lane == 31) sm.wcount[warp] = x;
+  if (tid < kMaxGlobal) sm.gnew[tid] = -1;
+  __syncthreads();
+  int before = 0, total = 0;
+#pragma unroll
+  for (int w = 0; w < kColsThreads / 32; ++w) {
+    const int c = sm.wcount[w];
+    before += w < warp ? c : 0;
+    total += c;
+  }
+  int out = before + x - cnt;
+  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
+#pragma unroll
+  for (int k = 0; k < kRun; ++k) {
+    if (!kf[k]) continue;
+    pos_out[out] = ps[k];
     for (int g = 0; g < ng; ++g)
-      if (sm.gc[g] == c) sm.gnew[g] = out;
+      if (sm.gc[g] == c0 + k) sm.gnew[g] = out;
     ++out;
   }
-  // bf16 outputs of the global rows
-#pragma unroll 4
-  for (int k = tid; k < ng * p.H * kHeadDim; k += kColsThreads) {
-    const int g = k / (p.H * kHeadDim), hh = (k / kHeadDim) % p.H, dd = k % kHeadDim;
-    const float o = __ldcg(p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim + dd);
-    v.O[((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) * kHeadDim + dd] =
-        __bfloat16_as_ushort(__float2bfloat16_rn(o));
+  // bf16 outputs of the global rows, 4 values per load
+  const int nvec = ng * p.H * (kHeadDim / 4);
+  for (int k0 = 0; k0 < nvec; k0 += 8 * kColsThreads) {
+    float4 o4[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int k = k0 + tid + u * kColsThreads;
+      const int g = k / (p.H * 16), hh = (k / 16) % p.H, d4 = k % 16;
+      o4[u] = k < nvec ? __ldcg(reinterpret_cast<const float4*>(
+                             p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim) + d4)
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int k = k0 + tid + u * kColsThreads;
+      if (k >= nvec) continue;
+      const int g = k / (p.H * 16), hh = (k / 16) % p.H, d4 = k % 16;
+      uint2 w2 = make_uint2(pack_bf16x2(o4[u].x, o4[u].y), pack_bf16x2(o4[u].z, o4[u].w));
+      *reinterpret_cast<uint2*>(v.O + ((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) *
+                                          kHeadDim + 4 * d4) = w2;
+    }
   }
   __syncthreads();
   if (tid == 0) {
@@ -1097,7 +1145,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     v.len_out[b] = total;
     if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = v.layer + 1;
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
-    v.ident_out[b] = (total == 0 || pos_out[total - 1] == total - 1) ? 1 : 0;
+    v.ident_out[b] = (total == 0 || __ldcg(pos_out + total - 1) == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
   }
 }

@@ -688,8 +688,13 @@ struct ColsSmem {
   float gsum[kMaxGlobal];
   int flag;
   float wpart[kColsThreads / 32];
-  int wcount[kColsThreads / 32];
   int gnew[kMaxGlobal];
+  // sequence compaction: per (round, warp) ballot of kept tokens and the
+  // exclusive prefix of their counts
+  uint32_t kbits[(kMaxLen + kColsThreads - 1) / kColsThreads][kColsThreads / 32];
+  int kpre[(kMaxLen + kColsThreads - 1) / kColsThreads][kColsThreads / 32];
+  int last_pos;
+  int total;
 };
 
 // dynamic shared memory: K and V of both key tiles, the Q ring, the global
@@ -995,6 +1000,18 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   __threadfence();
   const int j0 = 2 * pr * kTile;
   const int jn = min(n, j0 + 2 * kTile);
+  // this thread's key column: every head's column sum, loaded first (in
+  // flight while the global keys' partial sums are reduced below)
+  const int jj = j0 + tid;
+  const bool my_key = tid < 2 * kTile && jj < jn;
+  float hs[kTailMaxHeads];
+  float a = 0.f;
+  const float* ap = p.acc + static_cast<size_t>(b) * p.H * p.L + jj;
+#pragma unroll
+  for (int u = 0; u < kTailMaxHeads; ++u)
+    hs[u] = my_key && u < p.H ? __ldcg(ap + static_cast<size_t>(u) * p.L) : 0.f;
+  for (int h0 = kTailMaxHeads; my_key && h0 < p.H; ++h0)   // more than 16 heads
+    a += __ldcg(ap + static_cast<size_t>(h0) * p.L);
   // far-row partial sums of each global key that lies in this pair, over heads
   // and (query tile, warp) slices: spread over the whole CTA, every load
   // issued before the sums, reduced in a fixed order
@@ -1011,7 +1028,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
       const int hh = k / per_head, q4 = k - hh * per_head;   // q4 = 4 * tile + warp
       e[u] = k < total ? __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal) : 0.f;
     }
-    float v = 0.f;
+    float gv = 0.f;
     for (int k0 = 0; k0 < total; k0 += kPer * kColsThreads) {
       if (k0 > 0) {
 #pragma unroll
@@ -1023,30 +1040,23 @@ __global__ void __launch_bounds__(kColsThreads, 1)
         }
       }
 #pragma unroll
-      for (int u = 0; u < kPer; ++u) v += e[u];
+      for (int u = 0; u < kPer; ++u) gv += e[u];
     }
-    v = warp_sum(v);
-    if (lane == 0) sm.wpart[warp] = v;
+    gv = warp_sum(gv);
+    if (lane == 0) sm.wpart[warp] = gv;
     __syncthreads();
     if (tid == 0) {
-      float a = 0.f;
-      for (int w = 0; w < kColsThreads / 32; ++w) a += sm.wpart[w];
-      sm.gsum[g] = a;
+      float ga = 0.f;
+      for (int w = 0; w < kColsThreads / 32; ++w) ga += sm.wpart[w];
+      sm.gsum[g] = ga;
     }
     __syncthreads();
   }
-  if (tid < 2 * kTile && j0 + tid < jn) {
-    const int jj = j0 + tid;
-    const float* ap = p.acc + static_cast<size_t>(b) * p.H * p.L + jj;
-    float a = 0.f;
-    for (int h0 = 0; h0 < p.H; h0 += 16) {   // heads in order, 16 loads in flight
-      float e[16];
+  if (my_key) {
+    float hsum = 0.f;
 #pragma unroll
-      for (int u = 0; u < 16; ++u)
-        e[u] = h0 + u < p.H ? __ldcg(ap + static_cast<size_t>(h0 + u) * p.L) : 0.f;
-#pragma unroll
-      for (int u = 0; u < 16; ++u) a += e[u];
-    }
+    for (int u = 0; u < kTailMaxHeads; ++u) hsum += hs[u];   // heads in order
+    a = hsum + a;
     for (int g = 0; g < ng; ++g)
       if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
@@ -1065,54 +1075,72 @@ __global__ void __launch_bounds__(kColsThreads, 1)
 }
 
 // Order-preserving compaction of sequence b's kept tokens, the next layer's
-// global list, and the bf16 outputs of the global rows.  One CTA; thread t
-// takes one contiguous run of at most kRun tokens, loaded in one round.
+// global list, and the bf16 outputs of the global rows.  One CTA; token c is
+// handled by thread c % kColsThreads in round c / kColsThreads (coalesced
+// loads, all issued at once); output slots come from warp ballots and a
+// fixed-order prefix over (round, warp).
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
                                   ColsSmem& sm) {
-  constexpr int kRun = (kMaxLen + kColsThreads - 1) / kColsThreads;
+  constexpr int kRounds = (kMaxLen + kColsThreads - 1) / kColsThreads;
+  constexpr int kWarps = kColsThreads / 32;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int per = (n + kColsThreads - 1) / kColsThreads;
-  const int c0 = min(n, tid * per), c1 = min(n, c0 + per);
   const uint8_t* keep = p.keep + static_cast<size_t>(b) * p.L;
   const int32_t* pos = v.pos + static_cast<size_t>(b) * p.L;
   int32_t* pos_out = v.pos_out + static_cast<size_t>(b) * p.L;
-  uint8_t kf[kRun];
-  int32_t ps[kRun];
+  bool kf[kRounds];
+  int32_t ps[kRounds];
 #pragma unroll
-  for (int k = 0; k < kRun; ++k) {
-    const int c = c0 + k;
-    kf[k] = c < c1 ? __ldcg(keep + c) : 0;
-    ps[k] = c < c1 ? __ldcg(pos + c) : 0;
+  for (int r = 0; r < kRounds; ++r) {
+    const int c = r * kColsThreads + tid;
+    kf[r] = c < n && __ldcg(keep + c) != 0;
+    ps[r] = c < n ? __ldcg(pos + c) : 0;
   }
-  int cnt = 0;
 #pragma unroll
-  for (int k = 0; k < kRun; ++k) cnt += kf[k];
-  // exclusive scan of the run counts: within the warp, then over the warps
-  int x = cnt;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, off);
-    if (lane >= off) x += y;
+  for (int r = 0; r < kRounds; ++r) {
+    const uint32_t bits = __ballot_sync(0xffffffffu, kf[r]);
+    if (lane == 0) sm.kbits[r][warp] = bits;
   }
-  if (lane == 31) sm.wcount[warp] = x;
   if (tid < kMaxGlobal) sm.gnew[tid] = -1;
   __syncthreads();
-  int before = 0, total = 0;
+  if (warp == 0) {
+    // prefix over (round, warp) in order: lane l covers entries l, l+32, ...
+    constexpr int kEntries = kRounds * kWarps;
+    int cnt[(kEntries + 31) / 32];
+    int run = 0;
 #pragma unroll
-  for (int w = 0; w < kColsThreads / 32; ++w) {
-    const int c = sm.wcount[w];
-    before += w < warp ? c : 0;
-    total += c;
+    for (int u = 0; u < (kEntries + 31) / 32; ++u) {
+      const int e = u * 32 + lane;
+      cnt[u] = e < kEntries ? __popc(sm.kbits[e / kWarps][e % kWarps]) : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < (kEntries + 31) / 32; ++u) {
+      int x = cnt[u];
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x += y;
+      }
+      const int e = u * 32 + lane;
+      if (e < kEntries) sm.kpre[e / kWarps][e % kWarps] = run + x - cnt[u];
+      run += __shfl_sync(0xffffffffu, x, 31);
+    }
+    if (lane == 0) sm.total = run;
   }
-  int out = before + x - cnt;
-  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
+  __syncthreads();
+  const uint32_t below = (1u << lane) - 1u;
 #pragma unroll
-  for (int k = 0; k < kRun; ++k) {
-    if (!kf[k]) continue;
-    pos_out[out] = ps[k];
-    for (int g = 0; g < ng; ++g)
-      if (sm.gc[g] == c0 + k) sm.gnew[g] = out;
-    ++out;
+  for (int r = 0; r < kRounds; ++r) {
+    if (!kf[r]) continue;
+    const int out = sm.kpre[r][warp] + __popc(sm.kbits[r][warp] & below);
+    pos_out[out] = ps[r];
+    if (out == sm.total - 1) sm.last_pos = ps[r];
+  }
+  // next-layer index of each surviving global token
+  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
+  if (tid < ng) {
+    const int c = sm.gc[tid], r = c / kColsThreads, t = c % kColsThreads;
+    const uint32_t bits = sm.kbits[r][t >> 5];
+    if ((bits >> (t & 31)) & 1u) sm.gnew[tid] = sm.kpre[r][t >> 5] + __popc(bits & ((1u << (t & 31)) - 1u));
   }
   // bf16 outputs of the global rows, 4 values per load
   const int nvec = ng * p.H * (kHeadDim / 4);
@@ -1138,6 +1166,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
   }
   __syncthreads();
   if (tid == 0) {
+    const int total = sm.total;
     int m = 0;
     for (int g = 0; g < ng; ++g)
       if (sm.gnew[g] >= 0) v.gcur_out[b * kMaxGlobal + m++] = sm.gnew[g];
@@ -1145,7 +1174,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     v.len_out[b] = total;
     if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = v.layer + 1;
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
-    v.ident_out[b] = (total == 0 || __ldcg(pos_out + total - 1) == total - 1) ? 1 : 0;
+    v.ident_out[b] = (total == 0 || sm.last_pos == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
   }
 }

@@ -848,37 +848,49 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     const bool active = X == 0 || hasB;
     const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
     const uint32_t tST = tm + 128 * X, tSG = tm + 256 + 16 * X, tOG = tm + 320 + 64 * X;
+    // every load of the prologue is issued before any is used: the LSE of the
+    // query rows of the band (at most kPairTiles * 128 = 3 * 256) and, per
+    // warp, the (max, sum) pieces of global rows warp and warp + 8
+    static_assert(kPairTiles * kTile <= 3 * 256, "LSE window exceeds three loads a thread");
     const float* lse_src = p.lse + (static_cast<size_t>(b) * p.H + h) * p.L;
-    for (int k = tid; k < nq * kTile; k += 256) {
-      const int row = qt_lo * kTile + k;
-      sm.lse[k] = row < n ? __ldcg(lse_src + row) : INFINITY;
+    float lv[3];
+#pragma unroll
+    for (int u = 0; u < 3; ++u) {
+      const int k = tid + 256 * u, row = qt_lo * kTile + k;
+      lv[u] = (k < nq * kTile && row < n) ? __ldcg(lse_src + row) : INFINITY;
     }
-    if (ngp) {
-      // merge the per-(key tile, warp slice) (max, sum) of every global row
-      // into its LSE: warp w takes global rows w and w + 8; lane k takes
-      // entries k, k+32, k+64, k+96 of the 4 Tn entries (all loads issued
-      // first), then the warp combines; fixed order throughout
-      const size_t base_slot = (static_cast<size_t>(b) * p.H + h) * p.T * 4 * kMaxGlobal;
+    // lane k takes entries k, k+32, k+64, k+96 of the 4 Tn (key tile, warp
+    // slice) pieces; the warp combines them in a fixed order
+    const size_t base_slot = (static_cast<size_t>(b) * p.H + h) * p.T * 4 * kMaxGlobal;
+    float me[2][4], se[2][4];
 #pragma unroll
-      for (int gg = 0; gg < 2; ++gg) {
-        const int g = warp + 8 * gg;
-        if (g >= ng) break;   // warp-uniform
-        float me[4], se[4];
+    for (int gg = 0; gg < 2; ++gg) {
+      const int g = warp + 8 * gg;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int ent = lane + 32 * k;
-          const bool use = ent < 4 * Tn;
-          me[k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g)) : -INFINITY;
-          se[k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g) + 1) : 0.f;
-        }
-        const float m = fmaxf(fmaxf(me[0], me[1]), fmaxf(me[2], me[3]));
-        float sacc = 0.f;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) sacc += (me[k] == -INFINITY) ? 0.f : se[k] * ex2(me[k] - m);
-        const float M = warp_max(m);
-        const float S = warp_sum(m == -INFINITY ? 0.f : sacc * ex2(m - M));
-        if (lane == 0) sm.lse_g[g] = M + lg2(S);
+      for (int k = 0; k < 4; ++k) {
+        const int ent = lane + 32 * k;
+        const bool use = ngp && g < ng && ent < 4 * Tn;
+        me[gg][k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g)) : -INFINITY;
+        se[gg][k] = use ? __ldcg(p.gstat + 2 * (base_slot + ent * kMaxGlobal + g) + 1) : 0.f;
       }
+    }
+#pragma unroll
+    for (int u = 0; u < 3; ++u) {
+      const int k = tid + 256 * u;
+      if (k < nq * kTile) sm.lse[k] = lv[u];
+    }
+#pragma unroll
+    for (int gg = 0; gg < 2; ++gg) {
+      const int g = warp + 8 * gg;
+      if (!ngp || g >= ng) continue;   // warp-uniform
+      const float m = fmaxf(fmaxf(me[gg][0], me[gg][1]), fmaxf(me[gg][2], me[gg][3]));
+      float sacc = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        sacc += (me[gg][k] == -INFINITY) ? 0.f : se[gg][k] * ex2(me[gg][k] - m);
+      const float M = warp_max(m);
+      const float S = warp_sum(m == -INFINITY ? 0.f : sacc * ex2(m - M));
+      if (lane == 0) sm.lse_g[g] = M + lg2(S);
     }
     asm volatile("bar.sync 3, 256;" ::: "memory");
 
@@ -976,7 +988,9 @@ __global__ void __launch_bounds__(kColsThreads, 1)
           tmem_ld32(tOG + lane_off + c, o);
           tmem_ld_wait();
           if (lane < ng)
-            for (int k = 0; k < 32; ++k) atomicAdd(og + lane * kHeadDim + c + k, o[k]);
+#pragma unroll
+            for (int k = 0; k < 32; k += 4)
+              red_add_v4(og + lane * kHeadDim + c + k, o[k], o[k + 1], o[k + 2], o[k + 3]);
         }
       }
     }

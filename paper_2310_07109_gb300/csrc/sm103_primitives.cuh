@@ -329,6 +329,13 @@ __device__ __forceinline__ void prefetch_l2_line(const void* gptr) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(gptr));
 }
 
+// Four fp32 atomic additions to 16-byte aligned global memory in one request.
+__device__ __forceinline__ void red_add_v4(float* gptr, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(gptr), "f"(a), "f"(b),
+               "f"(c), "f"(d)
+               : "memory");
+}
+
 // Bring `bytes` (a multiple of 16, 16-byte aligned) of global memory into L2.
 __device__ __forceinline__ void prefetch_l2(const void* gptr, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(gptr), "r"(bytes) : "memory");

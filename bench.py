@@ -101,6 +101,41 @@ def layer_work(wl, inp, pos, lens):
     return out
 
 
+def kernel_source_hash() -> str:
+    """sha256 over the CUDA sources and the C header (each file's name, then its bytes)."""
+    import glob
+    import hashlib
+    files = sorted(glob.glob(os.path.join(ROOT, "paper_2310_07109_gb300", "csrc", "*.cu")) +
+                   glob.glob(os.path.join(ROOT, "paper_2310_07109_gb300", "csrc", "*.cuh")))
+    files.append(os.path.join(ROOT, "include", "sparsecoder.h"))
+    h = hashlib.sha256()
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(kernels):
+    """DRAM bytes (read + write) of one launch of each kernel, summed, from the ncu
+    capture recorded in profiles/traffic.json; None once any kernel source has
+    changed since that capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None, "no recorded capture"
+    if rec.get("source_sha256") != kernel_source_hash():
+        return None, "kernels changed since the recorded capture"
+    try:
+        total = sum(rec["kernels"][k]["dram_read_bytes"] + rec["kernels"][k]["dram_write_bytes"]
+                    for k in kernels)
+    except KeyError:
+        return None, "kernel not in the recorded capture"
+    return int(total), "ncu dram__bytes_read.sum + dram__bytes_write.sum, profiles/traffic.json"
+
+
 # ---------------------------------------------------------------------------
 # multi-rank aggregation (replicas: no collective on the data path)
 # ---------------------------------------------------------------------------
@@ -432,28 +467,44 @@ def run_native(args, wl):
     work = layer_work(wl, inp, pos, lens)
     bw = peaks["hbm_gbs"] * 1e9
     fl = peaks["bf16_tflops"] * 1e12
+    # the whole stack: every layer's roofline time over the attention kernels' time
     t_roof = sum(max(Bb / bw, Ff / fl) for Bb, Ff in work)
     t_meas = (float((rows_ms + cols_ms).sum()) + tail_ms) * 1e-3
-    bytes_alg = sum(Bb for Bb, _ in work)
-    flops_alg = sum(Ff for _, Ff in work)
-    hbm_bound = sum(Bb / bw for Bb, _ in work) >= sum(Ff / fl for _, Ff in work)
-    achieved = bytes_alg / t_meas / 1e9 if hbm_bound else flops_alg / t_meas / 1e12
-    l0 = work[0]
+    # the dominant unit: the per-layer kernel pair of the full-length layer 0
+    # (rows + cols, one launch each); when every sequence starts in the cluster
+    # kernel, that kernel over all layers
     t_l0 = (rows_ms[0] + cols_ms[0]) * 1e-3
+    if t_l0 > 1e-6:
+        unit_bytes, unit_flops, unit_t = work[0][0], work[0][1], t_l0
+        unit_kernels = ["sc_rows_kernel", "sc_cols_kernel"]
+        unit_desc = ("sc_rows_kernel + sc_cols_kernel of layer 0 (one launch each; B=%d "
+                     "sequences of %d tokens)" % (wl.B, int(lens[0].max())))
+    else:
+        unit_bytes = sum(Bb for Bb, _ in work)
+        unit_flops = sum(Ff for _, Ff in work)
+        unit_t = tail_ms * 1e-3
+        unit_kernels = ["sc_tail_kernel"]
+        unit_desc = "sc_tail_kernel (one launch: every layer of every sequence)"
+    hbm_bound = unit_bytes / bw >= unit_flops / fl
+    traffic, traffic_note = measured_traffic(unit_kernels)
     roofline = {
         "bound": "hbm" if hbm_bound else "tensor",
-        "achieved": achieved,
+        "achieved": unit_bytes / unit_t / 1e9 if hbm_bound else unit_flops / unit_t / 1e12,
         "peak": peaks["hbm_gbs"] if hbm_bound else peaks["bf16_tflops"],
         "unit": "GB/s" if hbm_bound else "TFLOP/s",
-        "frac": t_roof / t_meas,
-        "traffic": None,
+        "frac": max(unit_bytes / bw, unit_flops / fl) / unit_t,
+        "traffic": traffic,
         "peak_source": peak_src,
-        "scope": "the attention + pruning kernels of one step: sc_rows_kernel + sc_cols_kernel "
-                 "of the layers run per layer, plus sc_tail_kernel (the layers of sequences "
-                 "with <= 256 tokens left, one launch); algorithmic bytes 6152 B per "
-                 "token-layer, flops 3072 per allowed (query, key) pair; frac = sum_l "
-                 "max(F_l/peak_bf16, B_l/peak_hbm) / measured kernel time",
-        "layer0_frac": max(l0[0] / bw, l0[1] / fl) / t_l0 if t_l0 > 1e-6 else None,
+        "kernel": unit_desc,
+        "algorithmic": {"bytes": int(unit_bytes), "flops": int(unit_flops),
+                        "per_unit": "6152 B per token-layer; 3072 flop per allowed (query, "
+                                    "key) pair (all heads, QK^T and PV)"},
+        "launch_ms": unit_t * 1e3,
+        "traffic_note": traffic_note,
+        "stack_frac": t_roof / t_meas,
+        "stack_scope": "sum over layers of max(F_l/peak_bf16, B_l/peak_hbm) over the measured "
+                       "time of sc_rows_kernel + sc_cols_kernel (per-layer layers) and "
+                       "sc_tail_kernel",
         "kernel_ms_per_step": {"sc_rows_kernel": float(rows_ms.sum()),
                                "sc_cols_kernel": float(cols_ms.sum()),
                                "sc_gather_kernel": float(gath_ms.sum()),

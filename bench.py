@@ -428,12 +428,13 @@ def run_native(args, wl):
     # ---- kernels launched per timed step.  Eagerly: the library's plan.  A
     # captured step runs the per-layer kernels in a device-driven loop: prep,
     # [padding gather], rows + cols + gather + advance for each layer that some
-    # sequence still runs per layer (more than 256 tokens), then the cluster kernel.
+    # sequence still runs per layer (more than TAIL_MAX_LEN tokens), then the
+    # cluster kernel.
     eager_launches = sc.stack_launch_count(wl.n_layers, wl.B, wl.L, wl.H, wl.w, gpos,
                                            inp["pad_mask"] is not None)
-    looped = sum(1 for l in range(wl.n_layers) if (lens[l] > 256).any())
+    looped = sum(1 for l in range(wl.n_layers) if (lens[l] > sc.TAIL_MAX_LEN).any())
     graph_launches = (1 + (1 if inp["pad_mask"] is not None else 0) + 4 * looped + 1
-                      if wl.L > 256 else 2)
+                      if wl.L > sc.TAIL_MAX_LEN else 2)
     launches_per_step = graph_launches if graph is not None else eager_launches
 
     # ---- per-kernel times on the launching stream (same steps, events between kernels)

@@ -51,6 +51,7 @@ extern "C" {
 #define SC_MAX_LEN 4096   /* longest supported (padded) sequence */
 #define SC_MAX_GLOBAL 16  /* most global positions per call */
 #define SC_MAX_WINDOW 256 /* widest one-sided window when L > 640 */
+#define SC_TAIL_MAX_LEN 384 /* sequences this short finish in the cluster kernel (see sc_stack_forward) */
 
 typedef enum {
   SC_OK = 0,
@@ -172,8 +173,9 @@ int sc_layer_forward(const sc_layer_args* args, void* workspace, size_t workspac
  * token pruning, 12 layers in the paper's encoder).  Errors: see sc_status.
  *
  * Execution: a sequence runs layer by layer through the per-layer kernels
- * while it has more than 256 current tokens; from the first layer at which it
- * has at most 256 (after padding removal or after a layer's pruning) its
+ * while it has more than SC_TAIL_MAX_LEN current tokens; from the first layer at
+ * which it has at most SC_TAIL_MAX_LEN (after padding removal or after a layer's
+ * pruning) its
  * remaining layers run in one cluster kernel launched once at the end of the
  * call (one thread-block cluster of H CTAs per sequence, when the device can
  * schedule clusters of H <= 16 CTAs and n_layers <= 64).  The hand-over is

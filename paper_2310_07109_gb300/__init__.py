@@ -4,8 +4,9 @@ fused with learned token pruning, behind the C ABI of include/sparsecoder.h.
 The Python surface is a thin ctypes binding (``binding``); the arithmetic runs
 in ``libsparsecoder.so`` (``csrc/``), built in-tree by ``build.build_library``.
 """
-from .binding import (SparseCoderError, layer_forward, load, new_workspace, stack_forward,
-                      stack_launch_count, status_string, workspace_size, workspace_status)
+from .binding import (TAIL_MAX_LEN, SparseCoderError, layer_forward, load, new_workspace,
+                      stack_forward, stack_launch_count, status_string, workspace_size,
+                      workspace_status)
 
-__all__ = ["SparseCoderError", "layer_forward", "load", "new_workspace", "stack_forward",
+__all__ = ["TAIL_MAX_LEN", "SparseCoderError", "layer_forward", "load", "new_workspace", "stack_forward",
            "stack_launch_count", "status_string", "workspace_size", "workspace_status"]

@@ -53,6 +53,9 @@ class StackArgs(ctypes.Structure):
 
 
 SC_STACK_NO_TAIL = 1
+# sequences with at most this many current tokens finish in the cluster kernel
+# (SC_TAIL_MAX_LEN of include/sparsecoder.h)
+TAIL_MAX_LEN = 384
 
 EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
             "sc_stack_forward_profiled", "sc_stack_launch_count",

@@ -5,6 +5,8 @@
 #include <cstdint>
 #include <cuda.h>
 
+#include "../../include/sparsecoder.h"
+
 namespace sc {
 
 constexpr int kHeadDim = 64;
@@ -22,7 +24,7 @@ constexpr int kStatusInternal = 2;   // an invariant of the launch sequence did 
 
 // Sequences with at most kTailMax current tokens run their remaining layers in
 // the cluster kernel (one CTA per head); the per-layer kernels skip them.
-constexpr int kTailMax = 256;
+constexpr int kTailMax = SC_TAIL_MAX_LEN;
 constexpr int kTailMaxLayers = 64;
 constexpr int kTailMaxHeads = 16;   // largest (non-portable) cluster
 

@@ -1,4 +1,4 @@
-// sc_tail.cu -- the remaining layers of a sequence once at most 256 tokens
+// sc_tail.cu -- the remaining layers of a sequence once at most 384 tokens
 // survive: one thread-block cluster per sequence, one CTA per head, every
 // remaining layer in one launch.
 //
@@ -10,21 +10,27 @@
 //            threads, 16-byte asynchronous copies) into 128B-swizzled tiles;
 //            the rows of the next layer's candidates (a superset of its
 //            tokens) are prefetched into L2
-//   rows     S = Q K^T for the whole row (N <= 256 keys in tensor memory), an
-//            exact two-pass softmax in fp32 (base 2), P (bf16) back to tensor
-//            memory, O = P V, LSE_i
-//   columns  S^T = K Q^T, and per key column j the sum over rows of
-//            exp2(S_ij - LSE_i): one thread per column, no cross-thread sums
+//   rows     per 128-row query tile: S = Q K^T over the keys in halves of at
+//            most 256 (tensor memory), an exact two-pass softmax in fp32 (base
+//            2), P (bf16) back to tensor memory, O = P V accumulated over the
+//            halves, LSE_i
+//   columns  per 128-key tile: S^T = K Q^T over the queries in halves, and per
+//            key column j the sum over rows of exp2(S_ij - LSE_i): one thread
+//            per column, no cross-thread sums
 //   heads    the H CTAs exchange their column sums through distributed shared
 //            memory; every CTA adds the heads in the same fixed order, so all
 //            take the same keep decisions (s_j >= alpha_l / n, j == 0 kept) and
 //            compact the token list the same way, without a second exchange
 //
+// Softmax warpgroup X takes query tiles X and X + 2 and key tiles X and X + 2;
+// its own MMA-issuing thread serves it in a fixed order of events, so each
+// tcgen05.commit covers that warpgroup's MMAs only.
+//
 // The allowed set (window, global tokens), the softmax, the vertical
 // accumulation and the order-preserving removal are those of Sec. "Sparse
 // Attention", Sec. "Extractor of Attention Scores in Sparse Attention Matrix"
-// and Sec. "Token Pruning"; global rows are ordinary rows here (all of their
-// <= 256 keys are in tensor memory at once).
+// and Sec. "Token Pruning"; global rows are ordinary rows here (their whole row
+// of at most 384 keys is evaluated).
 #include <cuda_runtime.h>
 #include <cstdint>
 
@@ -33,24 +39,28 @@
 
 namespace sc {
 
-constexpr int kTailThreads = 288;                        // 2 softmax warpgroups + control warp
-constexpr uint32_t kTailOpBytes = kTailMax * kHeadDim * 2;   // 256 rows of one tensor (32 KB)
-// Q, K, V operands plus alignment; the remainder keeps a second CTA off the SM,
-// since each CTA holds all 512 tensor-memory columns while it waits at cluster
-// barriers (two CTAs of different clusters sharing an SM could otherwise wait
-// on each other's allocation).
-constexpr uint32_t kTailDyn = 120 * 1024;
-static_assert(3 * kTailOpBytes + 1024 <= kTailDyn, "tail operands exceed the dynamic shared memory");
+constexpr int kTailThreads = 320;   // 2 softmax warpgroups + 2 MMA-issuing warps
+constexpr int kTailTiles = (kTailMax + kTile - 1) / kTile;   // 128-row tiles (3)
+constexpr uint32_t kTailOpBytes = kTailTiles * kTileBytes;   // rows of one tensor (48 KB)
+constexpr int kTailChunks = kTailMax / 32;                    // 32-token chunks (12)
+static_assert(kTailMax <= 384, "a second key half must fit beside O in tensor memory");
+// Q, K, V operands plus alignment; more than half of an SM's shared memory, so
+// a second CTA never shares the SM (each holds all 512 tensor-memory columns
+// while it waits at cluster barriers: two CTAs of different clusters on one SM
+// could otherwise wait on each other's allocation).
+constexpr uint32_t kTailDyn = 3 * kTailOpBytes + 1024;
+static_assert(kTailDyn > 233472 / 2, "the tail kernel must occupy an SM alone");
 
 struct TailSmem {
-  uint64_t bar_free[2], bar_fin;
-  uint64_t bar_s[2], bar_p[2], bar_o[2], bar_st[2];
+  uint64_t bar_sfull[2], bar_sfree[2], bar_pready[2], bar_odone[2], bar_stfull[2], bar_fin[2];
   uint32_t tmem_base;
   int abort;
   int n[2];
-  int wcnt[8];
+  uint32_t kbits[2][8];               // compaction: ballot of kept tokens per (round, warp)
+  int kpre[2][8];                     // ... and the exclusive prefix of their counts
+  int total;
   int gpos[kMaxGlobal];               // global positions (sorted), -1 past n_global
-  uint32_t gbits[2][kTailMax / 32];   // global flags of the current / next token list
+  uint32_t gbits[2][kTailChunks];     // global flags of the current / next token list
   int32_t pos[2][kTailMax];           // original positions of the current / next tokens
   alignas(16) float nlse[kTailMax];   // -LSE of each query row (-inf past n)
   float colsum[2][kTailMax];          // this head's column sums, by layer parity
@@ -105,6 +115,8 @@ __device__ __forceinline__ void apply_mask(float* x, uint32_t m) {
   for (int k = 0; k < 32; ++k) x[k] = ((m >> k) & 1u) ? x[k] : -INFINITY;
 }
 
+__device__ __forceinline__ int round16(int x) { return (x + 15) & ~15; }
+
 __global__ void __launch_bounds__(kTailThreads, 1)
     sc_tail_kernel(const __grid_constant__ TailParams p) {
   const int H = p.H, w = p.w, L = p.L, B = p.B, n_layers = p.n_layers;
@@ -133,14 +145,13 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   for (int k = tid; k < static_cast<int>(3 * kTailOpBytes / 16); k += kTailThreads)
     reinterpret_cast<uint4*>(base)[k] = make_uint4(0u, 0u, 0u, 0u);
   if (tid == 0) {
-    mbar_init(&sm.bar_free[0], 128);
-    mbar_init(&sm.bar_free[1], 128);
-    mbar_init(&sm.bar_fin, 1);
     for (int X = 0; X < 2; ++X) {
-      mbar_init(&sm.bar_s[X], 1);
-      mbar_init(&sm.bar_p[X], 128);
-      mbar_init(&sm.bar_o[X], 1);
-      mbar_init(&sm.bar_st[X], 1);
+      mbar_init(&sm.bar_sfull[X], 1);
+      mbar_init(&sm.bar_sfree[X], 128);
+      mbar_init(&sm.bar_pready[X], 128);
+      mbar_init(&sm.bar_odone[X], 1);
+      mbar_init(&sm.bar_stfull[X], 1);
+      mbar_init(&sm.bar_fin[X], 1);
     }
     sm.abort = 0;
     sm.n[0] = n0;
@@ -151,32 +162,34 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (tid < kTailMax) {
+  for (int c = tid; c < kTailChunks * 32; c += kTailThreads) {
     int ps = -1;
-    if (tid < n0) ps = __ldcg(p.pos + (static_cast<size_t>(l0) * B + b) * L + tid);
-    sm.pos[0][tid] = ps;
-    const uint32_t bits = __ballot_sync(0xffffffffu, tid < n0 && tail_is_global(sm, ps));
-    if (lane == 0) sm.gbits[0][warp] = bits;
+    if (c < n0) ps = __ldcg(p.pos + (static_cast<size_t>(l0) * B + b) * L + c);
+    if (c < kTailMax) sm.pos[0][c] = ps;
+    const uint32_t bits = __ballot_sync(0xffffffffu, c < n0 && tail_is_global(sm, ps));
+    if (lane == 0) sm.gbits[0][c >> 5] = bits;
   }
   const uint32_t tm = sm.tmem_base;
   volatile int* abort_flag = &sm.abort;
   const uint32_t q_a = smem_u32(base), k_a = q_a + kTailOpBytes, v_a = k_a + kTailOpBytes;
   const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+  const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
 
-  uint32_t cnt0 = 0, cnt1 = 0;   // layers in which tile X (0, 1) was in use: barrier phases
+  // barrier phases consumed so far (kernel lifetime; both sides count alike)
+  uint32_t n_sfull = 0, n_stfull = 0, n_odone = 0;   // softmax side
+  uint32_t n_sfree = 0, n_ready = 0;                  // issuing side
   int cur = 0;
   for (int l = l0; l < n_layers; ++l) {
     const int it = l - l0;
     __syncthreads();   // sm.pos / sm.n / sm.gbits of this layer are complete
     const int n = sm.n[cur];
-    const int nX = n > kTile ? 2 : 1;
-    const int n16 = (n + 15) & ~15;
-    const int nc2 = (n + 63) >> 6;     // 64-wide steps of a row (or column)
+    const int nq = (n + kTile - 1) / kTile;   // 128-row tiles (1..3)
+    const int nkh = n > 256 ? 2 : 1;          // key (query) halves of at most 256
     const int par = it & 1;
 
     // ---- rows of the current tokens: 16-byte pieces, 128B-swizzled tiles
     {
-      // thread tid copies 16-byte piece (tid & 7) of every 36th row, the
+      // thread tid copies 16-byte piece (tid & 7) of every 40th row, the
       // same piece of Q, K and V from one address computation
       const size_t tok0 = (static_cast<size_t>(l) * B + b) * L;
       const int piece = tid & 7;
@@ -203,93 +216,136 @@ __global__ void __launch_bounds__(kTailThreads, 1)
     __syncthreads();
     tc_fence_after();
 
-    if (warp == 8) {
+    if (warp >= 8) {
       // ------------------------------------------------------- MMA issue
-      if (lane == 0 && *abort_flag == 0) {
-        const uint32_t id_s = idesc_bf16(128, n16, false, false);
+      const int X = warp - 8;
+      if (lane == 0 && X < nq && *abort_flag == 0) {
+        const uint32_t tR = tm + 256u * X;              // this warpgroup's columns
         const uint32_t id_pv = idesc_bf16(128, 64, false, true);
-        for (int X = 0; X < nX; ++X) {
-#pragma unroll
-          for (int k = 0; k < kHeadDim / 16; ++k)
-            umma_bf16(tm + 256u * X, sdesc_sw128(q_a + X * kTileBytes + 32 * k),
-                      sdesc_sw128(k_a + 32 * k), id_s, k > 0);
-          umma_commit(&sm.bar_s[X]);
-        }
-        if (nX == 1) {
-          // one query tile leaves the second half of tensor memory free: S^T
-          // of the (single) key tile goes there at once
-#pragma unroll
-          for (int k = 0; k < kHeadDim / 16; ++k)
-            umma_bf16(tm + 256u, sdesc_sw128(k_a + 32 * k), sdesc_sw128(q_a + 32 * k), id_s, k > 0);
-          umma_commit(&sm.bar_st[0]);
-        }
-        bool ok = true;
-        for (int X = 0; ok && X < nX; ++X) {
-          if (!(ok = mbar_wait(&sm.bar_p[X], (X ? cnt1 : cnt0) & 1, abort_flag))) break;
-          tc_fence_after();
-          for (int k = 0; k < n16 / 16; ++k)
-            umma_bf16_ts(tm + 256u * X + 128u, tm + 256u * X + 8u * k,
-                         sdesc_sw128(v_a + 2048u * k), id_pv, k > 0);
-          umma_commit(&sm.bar_o[X]);
-        }
-        // two query tiles: S^T of key tile X overwrites warpgroup X's columns
-        // once that warpgroup has read its O
-        for (int X = 0; ok && nX == 2 && X < 2; ++X) {
-          if (!(ok = mbar_wait(&sm.bar_free[X], it & 1, abort_flag))) break;
+        bool first = true, ok = true;
+        // the warpgroup's columns may be overwritten: the previous contents are read
+        auto region = [&]() -> bool {
+          if (first) {
+            first = false;
+            return true;
+          }
+          return mbar_wait(&sm.bar_sfree[X], (n_sfree++) & 1, abort_flag);
+        };
+        auto ready = [&]() -> bool {
+          return mbar_wait(&sm.bar_pready[X], (n_ready++) & 1, abort_flag);
+        };
+        auto issue_s = [&](int qt, int kh) {   // S of query tile qt against key half kh
+          const int N = round16(min(256, n - 256 * kh));
+          const uint32_t id = idesc_bf16(128, N, false, false);
           tc_fence_after();
 #pragma unroll
           for (int k = 0; k < kHeadDim / 16; ++k)
-            umma_bf16(tm + 256u * X, sdesc_sw128(k_a + X * kTileBytes + 32 * k),
-                      sdesc_sw128(q_a + 32 * k), id_s, k > 0);
-          umma_commit(&sm.bar_st[X]);
+            umma_bf16(tR, sdesc_sw128(q_a + qt * kTileBytes + 32 * k),
+                      sdesc_sw128(k_a + kh * 2 * kTileBytes + 32 * k), id, k > 0);
+          umma_commit(&sm.bar_sfull[X]);
+        };
+        auto issue_pv = [&](int kh, bool acc) {   // O (+)= P V over key half kh
+          const int N = round16(min(256, n - 256 * kh));
+          tc_fence_after();
+          for (int k = 0; k < N / 16; ++k)
+            umma_bf16_ts(tR + 128u, tR + 8u * k, sdesc_sw128(v_a + kh * 2 * kTileBytes + 2048u * k),
+                         id_pv, (acc || k > 0) ? 1u : 0u);
+          umma_commit(&sm.bar_odone[X]);
+        };
+        auto issue_st = [&](int kt, int qh, uint32_t dst) {   // S^T of key tile kt, query half qh
+          const int N = round16(min(256, n - 256 * qh));
+          const uint32_t id = idesc_bf16(128, N, false, false);
+          tc_fence_after();
+#pragma unroll
+          for (int k = 0; k < kHeadDim / 16; ++k)
+            umma_bf16(dst, sdesc_sw128(k_a + kt * kTileBytes + 32 * k),
+                      sdesc_sw128(q_a + qh * 2 * kTileBytes + 32 * k), id, k > 0);
+          umma_commit(&sm.bar_stfull[X]);
+        };
+        for (int r = 0; ok && r < 2; ++r) {
+          const int qt = X + 2 * r;
+          if (qt >= nq) break;
+          if (nkh == 1) {
+            if (!(ok = region())) break;
+            issue_s(qt, 0);
+            // one query tile: the other half of tensor memory takes S^T at once
+            if (nq == 1) issue_st(0, 0, tm + 256u);
+            if (!(ok = ready())) break;
+            issue_pv(0, false);
+          } else {
+            if (!(ok = region())) break;   // pass 1, key half 0
+            issue_s(qt, 0);
+            if (!(ok = region())) break;   // pass 1, key half 1
+            issue_s(qt, 1);
+            if (!(ok = region())) break;   // pass 2, key half 0
+            issue_s(qt, 0);
+            if (!(ok = ready())) break;
+            issue_pv(0, false);
+            // key half 1 has at most 128 columns: S lands beside O, and after
+            // P V of half 0 in issue order, so it may be issued at once
+            issue_s(qt, 1);
+            if (!(ok = ready())) break;
+            issue_pv(1, true);
+          }
         }
+        for (int r = 0; ok && nq > 1 && r < 2; ++r) {
+          const int kt = X + 2 * r;
+          if (kt >= nq) break;
+          for (int qh = 0; ok && qh < nkh; ++qh) {
+            if (!(ok = region())) break;
+            issue_st(kt, qh, tR);
+          }
+        }
+        if (ok) region();   // the last release of the layer
       }
       __syncwarp();
     } else {
       // ------------------------------------------------------- softmax warps
       const int X = warp >> 2;
-      const int i = kTile * X + (tid & 127);   // query row (rows step) / key column (cols step)
-      const bool use = X < nX;
-      const uint32_t ph = (X ? cnt1 : cnt0) & 1;
-      const uint32_t tS = tm + 256u * X, tO = tS + 128u;
-      Partners me;
-      me.valid = i < n;
-      me.lo = max(0, i - w);
-      me.hi = min(n - 1, i + w);
-      me.all = w >= n - 1 || ((sm.gbits[cur][i >> 5] >> (i & 31)) & 1u);
-      float lse = INFINITY;
-      if (use && tail_wait(&sm.bar_s[X], ph, abort_flag)) {
-        tc_fence_after();
-        // pass 1: row maximum over the allowed keys, 64 columns per step
-        float pm[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        for (int q2 = 0; q2 < nc2; ++q2) {
+      const int r = tid & 127;
+      const uint32_t tR = tm + 256u * X + lane_off, tO = tR + 128u;
+      bool ok = true;
+      auto partners_of = [&](int i) {
+        Partners me;
+        me.valid = i < n;
+        me.lo = max(0, i - w);
+        me.hi = min(n - 1, i + w);
+        me.all = w >= n - 1 || ((sm.gbits[cur][i >> 5] >> (i & 31)) & 1u);
+        return me;
+      };
+      // row maximum over the keys of half kh (S in tensor memory)
+      auto half_max = [&](const Partners& me, int kh, float mx) {
+        const int nh = min(256, n - 256 * kh);
+        for (int q2 = 0; q2 < (nh + 63) >> 6; ++q2) {
           float x[64];
-          tmem_ld32(tS + lane_off + 64 * q2, x);
-          tmem_ld32(tS + lane_off + 64 * q2 + 32, x + 32);
+          tmem_ld32(tR + 64 * q2, x);
+          tmem_ld32(tR + 64 * q2 + 32, x + 32);
           tmem_ld_wait();
 #pragma unroll
           for (int hq = 0; hq < 2; ++hq) {
-            apply_mask(x + 32 * hq, partner_mask(me, sm, cur, 2 * q2 + hq, n));
+            apply_mask(x + 32 * hq, partner_mask(me, sm, cur, 8 * kh + 2 * q2 + hq, n));
 #pragma unroll
-            for (int k = 0; k < 32; ++k) pm[k & 3] = fmaxf(pm[k & 3], x[32 * hq + k]);
+            for (int k = 0; k < 32; k += 2) mx = fmax3(mx, x[32 * hq + k], x[32 * hq + k + 1]);
           }
         }
-        const float mx = fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3]));
-        const float nmc = me.valid ? -mx * kLogitScale2 : 0.f;
-        // pass 2: P = exp2(S - max) (masked keys: exp2(-inf) = 0), row sum, and
-        // P as bf16 pairs over the first half of each step's columns (they
-        // land in columns that this or earlier steps occupied, already read)
-        const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2), n2 = f2_pack(nmc, nmc);
+        return mx;
+      };
+      // P = exp2(S - max) over half kh, written as bf16 pairs over the first
+      // half of its columns (each step's pairs land on columns this or an
+      // earlier step has read); returns the half's row sum
+      auto half_exp = [&](const Partners& me, int kh, float nmc) {
+        const int nh = min(256, n - 256 * kh);
+        const uint64_t n2 = f2_pack(nmc, nmc);
         uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
-        for (int q2 = 0; q2 < nc2; ++q2) {
+        for (int q2 = 0; q2 < (nh + 63) >> 6; ++q2) {
           float x[64];
-          tmem_ld32(tS + lane_off + 64 * q2, x);
-          tmem_ld32(tS + lane_off + 64 * q2 + 32, x + 32);
+          tmem_ld32(tR + 64 * q2, x);
+          tmem_ld32(tR + 64 * q2 + 32, x + 32);
           tmem_ld_wait();
 #pragma unroll
           for (int hq = 0; hq < 2; ++hq) {
             float* xh = x + 32 * hq;
-            apply_mask(xh, partner_mask(me, sm, cur, 2 * q2 + hq, n));
+            apply_mask(xh, partner_mask(me, sm, cur, 8 * kh + 2 * q2 + hq, n));
             uint32_t pk[16];
 #pragma unroll
             for (int k = 0; k < 32; k += 2) {
@@ -301,79 +357,118 @@ __global__ void __launch_bounds__(kTailThreads, 1)
               else s2a = f2_add(s2a, f2_pack(u, v));
               pk[k >> 1] = pack_bf16x2(u, v);
             }
-            tmem_st16(tS + lane_off + 32 * q2 + 16 * hq, pk);
+            tmem_st16(tR + 32 * q2 + 16 * hq, pk);
           }
         }
         tmem_st_wait();
         float la, lb, lc, ld;
         f2_unpack(s2a, la, lb);
         f2_unpack(s2b, lc, ld);
-        const float lsum = (la + lb) + (lc + ld);
+        return (la + lb) + (lc + ld);
+      };
+      auto release = [&]() {   // the warpgroup's columns are read
         tc_fence_before();
-        mbar_arrive(&sm.bar_p[X]);
-        if (tail_wait(&sm.bar_o[X], ph, abort_flag)) {
+        mbar_arrive(&sm.bar_sfree[X]);
+      };
+
+      // ---- rows: query tiles X and X + 2
+      for (int rr = 0; ok && rr < 2; ++rr) {
+        const int qt = X + 2 * rr;
+        if (qt >= nq) break;
+        const int i = kTile * qt + r;
+        const Partners me = partners_of(i);
+        float mx = -INFINITY;
+        if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
+        tc_fence_after();
+        mx = half_max(me, 0, mx);
+        if (nkh == 2) {
+          release();
+          if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
           tc_fence_after();
-          lse = me.valid ? lg2(lsum) - nmc : INFINITY;
-          const float inv = me.valid ? 1.f / lsum : 0.f;
+          mx = half_max(me, 1, mx);
+          release();
+          if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
+          tc_fence_after();
+        }
+        const float nmc = me.valid ? -mx * kLogitScale2 : 0.f;
+        float lsum = half_exp(me, 0, nmc);
+        tc_fence_before();
+        mbar_arrive(&sm.bar_pready[X]);
+        if (nkh == 2) {
+          if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
+          tc_fence_after();
+          lsum += half_exp(me, 1, nmc);
+          tc_fence_before();
+          mbar_arrive(&sm.bar_pready[X]);
+          if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
+        }
+        if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
+        tc_fence_after();
+        const float inv = me.valid ? 1.f / lsum : 0.f;
+        float o[64];
+        tmem_ld32(tO, o);
+        tmem_ld32(tO + 32, o + 32);
+        tmem_ld_wait();
+        if (me.valid) {
           uint16_t* orow =
               p.O + (((static_cast<size_t>(l) * B + b) * L + i) * H + h) * kHeadDim;
-          float o[64];
-          tmem_ld32(tO + lane_off, o);
-          tmem_ld32(tO + lane_off + 32, o + 32);
-          tmem_ld_wait();
-          if (me.valid) {
 #pragma unroll
-            for (int k = 0; k < 64; k += 8) {
-              const uint4 v = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
-                                         pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
-                                         pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
-                                         pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
-              *reinterpret_cast<uint4*>(orow + k) = v;
-            }
+          for (int k = 0; k < 64; k += 8) {
+            const uint4 v = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
+                                       pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
+                                       pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
+                                       pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
+            *reinterpret_cast<uint4*>(orow + k) = v;
           }
         }
+        sm.nlse[i] = me.valid ? -(lg2(lsum) - nmc) : -INFINITY;
+        release();
       }
-      // this warpgroup has read its S, P and O: with two query tiles its
-      // columns take S^T of key tile X next
-      tc_fence_before();
-      mbar_arrive(&sm.bar_free[X]);
-      sm.nlse[i] = -lse;
+      // rows past the last query tile take no part in the column sums
+      for (int i = kTile * nq + (tid & 255); i < kTailMax; i += 256) sm.nlse[i] = -INFINITY;
       tail_named_sync();   // every LSE is written
 
-      // columns: key j = i of this thread, summed over the query rows
-      float acc = 0.f;
-      if (use && tail_wait(&sm.bar_st[X], ph, abort_flag)) {
-        tc_fence_after();
-        const uint32_t tST = nX == 1 ? tm + 256u : tS;
-        const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
+      // ---- columns: key tiles X and X + 2, summed over the query rows
+      for (int rr = 0; ok && rr < 2; ++rr) {
+        const int kt = X + 2 * rr;
+        if (kt >= nq) break;
+        const int j = kTile * kt + r;
+        const Partners me = partners_of(j);
+        const uint32_t tST = nq == 1 ? tm + 256u + lane_off : tR;
         uint64_t a2a = f2_pack(0.f, 0.f), a2b = a2a;
-        for (int q2 = 0; q2 < nc2; ++q2) {
-          float x[64];
-          tmem_ld32(tST + lane_off + 64 * q2, x);
-          tmem_ld32(tST + lane_off + 64 * q2 + 32, x + 32);
-          tmem_ld_wait();
+        for (int qh = 0; ok && qh < nkh; ++qh) {
+          if (!(ok = tail_wait(&sm.bar_stfull[X], (n_stfull++) & 1, abort_flag))) break;
+          tc_fence_after();
+          const int nh = min(256, n - 256 * qh);
+          for (int q2 = 0; q2 < (nh + 63) >> 6; ++q2) {
+            float x[64];
+            tmem_ld32(tST + 64 * q2, x);
+            tmem_ld32(tST + 64 * q2 + 32, x + 32);
+            tmem_ld_wait();
 #pragma unroll
-          for (int hq = 0; hq < 2; ++hq) {
-            float* xh = x + 32 * hq;
-            apply_mask(xh, partner_mask(me, sm, cur, 2 * q2 + hq, n));
-            const float* lw = sm.nlse + 64 * q2 + 32 * hq;
+            for (int hq = 0; hq < 2; ++hq) {
+              const int qa = 8 * qh + 2 * q2 + hq;   // chunk of query rows
+              float* xh = x + 32 * hq;
+              apply_mask(xh, partner_mask(me, sm, cur, qa, n));
+              const float* lw = sm.nlse + 32 * qa;
 #pragma unroll
-            for (int k = 0; k < 32; k += 4) {
-              const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
-              float e0, e1, e2, e3;
-              f2_unpack(f2_fma(f2_pack(xh[k], xh[k + 1]), c2, f2_pack(l4.x, l4.y)), e0, e1);
-              f2_unpack(f2_fma(f2_pack(xh[k + 2], xh[k + 3]), c2, f2_pack(l4.z, l4.w)), e2, e3);
-              a2a = f2_add(a2a, f2_pack(ex2(e0), ex2(e1)));
-              a2b = f2_add(a2b, f2_pack(ex2(e2), ex2(e3)));
+              for (int k = 0; k < 32; k += 4) {
+                const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
+                float e0, e1, e2, e3;
+                f2_unpack(f2_fma(f2_pack(xh[k], xh[k + 1]), c2, f2_pack(l4.x, l4.y)), e0, e1);
+                f2_unpack(f2_fma(f2_pack(xh[k + 2], xh[k + 3]), c2, f2_pack(l4.z, l4.w)), e2, e3);
+                a2a = f2_add(a2a, f2_pack(ex2(e0), ex2(e1)));
+                a2b = f2_add(a2b, f2_pack(ex2(e2), ex2(e3)));
+              }
             }
           }
+          if (nq > 1) release();
         }
         float a0, a1, a2, a3;
         f2_unpack(a2a, a0, a1);
         f2_unpack(a2b, a2, a3);
-        acc = (a0 + a2) + (a1 + a3);
+        sm.colsum[par][j] = me.valid ? (a0 + a2) + (a1 + a3) : 0.f;
       }
-      if (use) sm.colsum[par][i] = acc;
     }
 
     // ------------------------------------------------- heads, threshold, compaction
@@ -381,35 +476,48 @@ __global__ void __launch_bounds__(kTailThreads, 1)
     cluster_sync();
     tc_fence_after();
     const int nxt = cur ^ 1;
-    if (tid < kTailMax) {
-      const int j = tid;
-      bool keep = false;
-      if (j < n) {
-        const uint32_t la = smem_u32(&sm.colsum[par][j]);
-        float v[kTailMaxHeads];
+    if (tid < 256) {
+      bool keep[2] = {false, false};
 #pragma unroll
-        for (int hh = 0; hh < kTailMaxHeads; ++hh)
-          v[hh] = hh < H ? ld_dsmem_f32(dsmem_addr(la, hh)) : 0.f;
-        float a = 0.f;
+      for (int rd = 0; rd < 2; ++rd) {
+        const int j = tid + 256 * rd;
+        if (j < n) {
+          const uint32_t la = smem_u32(&sm.colsum[par][j]);
+          float v[kTailMaxHeads];
 #pragma unroll
-        for (int hh = 0; hh < kTailMaxHeads; ++hh)
-          if (hh < H) a += v[hh];
-        const float s = a / static_cast<float>(H * n);
-        keep = (j == 0) || (s >= p.alpha[l] / static_cast<float>(n));
-        if (h == 0) p.scores[(static_cast<size_t>(l) * B + b) * L + j] = s;
+          for (int hh = 0; hh < kTailMaxHeads; ++hh)
+            v[hh] = hh < H ? ld_dsmem_f32(dsmem_addr(la, hh)) : 0.f;
+          float a = 0.f;
+#pragma unroll
+          for (int hh = 0; hh < kTailMaxHeads; ++hh)
+            if (hh < H) a += v[hh];
+          const float s = a / static_cast<float>(H * n);
+          keep[rd] = (j == 0) || (s >= p.alpha[l] / static_cast<float>(n));
+          if (h == 0) p.scores[(static_cast<size_t>(l) * B + b) * L + j] = s;
+        }
+        const uint32_t kb = __ballot_sync(0xffffffffu, keep[rd]);
+        if (lane == 0) sm.kbits[rd][warp] = kb;
       }
-      const uint32_t kb = __ballot_sync(0xffffffffu, keep);
-      if (lane == 0) sm.wcnt[warp] = __popc(kb);
       tail_named_sync();
-      int off = 0, total = 0;
+      if (warp == 0) {
+        // exclusive prefix over (round, warp): 16 entries, one per lane
+        const int cnt = lane < 16 ? __popc(sm.kbits[lane >> 3][lane & 7]) : 0;
+        int x = cnt;
 #pragma unroll
-      for (int w8 = 0; w8 < 8; ++w8) {
-        const int c = sm.wcnt[w8];
-        off += (w8 < warp) ? c : 0;
-        total += c;
+        for (int off = 1; off < 32; off <<= 1) {
+          const int y = __shfl_up_sync(0xffffffffu, x, off);
+          if (lane >= off) x += y;
+        }
+        if (lane < 16) sm.kpre[lane >> 3][lane & 7] = x - cnt;
+        if (lane == 31) sm.total = x;
       }
-      if (keep) {
-        const int k = off + __popc(kb & ((1u << lane) - 1u));
+      tail_named_sync();
+      const int total = sm.total;
+#pragma unroll
+      for (int rd = 0; rd < 2; ++rd) {
+        if (!keep[rd]) continue;
+        const int j = tid + 256 * rd;
+        const int k = sm.kpre[rd][warp] + __popc(sm.kbits[rd][warp] & ((1u << lane) - 1u));
         const int ps = sm.pos[cur][j];
         sm.pos[nxt][k] = ps;
         if (h == 0) p.pos[(static_cast<size_t>(l + 1) * B + b) * L + k] = ps;
@@ -419,26 +527,32 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         if (h == 0) p.len[static_cast<size_t>(l + 1) * B + b] = total;
       }
       tail_named_sync();
-      const bool gk = tid < total && tail_is_global(sm, sm.pos[nxt][tid]);
-      const uint32_t gb = __ballot_sync(0xffffffffu, gk);
-      if (lane == 0) sm.gbits[nxt][warp] = gb;
+#pragma unroll
+      for (int rd = 0; rd < 2; ++rd) {
+        const int k = tid + 256 * rd;
+        const bool gk = k < total && tail_is_global(sm, sm.pos[nxt][k]);
+        const uint32_t gb = __ballot_sync(0xffffffffu, gk);
+        if (lane == 0 && (k >> 5) < kTailChunks) sm.gbits[nxt][k >> 5] = gb;
+      }
     }
-    cnt0 += 1;
-    cnt1 += (nX == 2) ? 1 : 0;
     cur = nxt;
   }
 
   // no CTA leaves while another may still read its column sums
   tc_fence_before();
   cluster_sync();
-  if (warp == 8) {
+  if (warp >= 8 && warp - 8 < 2) {
     if (lane == 0) {
       // after an expired wait, MMAs may still be in flight
-      umma_commit(&sm.bar_fin);
+      umma_commit(&sm.bar_fin[warp - 8]);
       int dummy = 0;
-      mbar_wait(&sm.bar_fin, 0, &dummy, 1000000000ull);
+      mbar_wait(&sm.bar_fin[warp - 8], 0, &dummy, 1000000000ull);
     }
     __syncwarp();
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 8) {
     tc_fence_after();
     tmem_dealloc(tm, 512);
   }

@@ -31,6 +31,13 @@ def test_header_declares_the_documented_calls():
     assert "sc_layer_forward" in names and "sc_stack_forward" in names
 
 
+def test_binding_constants_match_the_header():
+    text = open(HEADER).read()
+    defines = dict(re.findall(r"^#define\s+(SC_\w+)\s+(\d+)", text, re.M))
+    assert int(defines["SC_TAIL_MAX_LEN"]) == bd.TAIL_MAX_LEN
+    assert int(defines["SC_STACK_NO_TAIL"]) == bd.SC_STACK_NO_TAIL
+
+
 def test_every_declared_symbol_is_exported(lib):
     raw = ctypes.CDLL(bd.library_path())
     for name in declared_functions():

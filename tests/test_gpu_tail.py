@@ -1,12 +1,14 @@
 """GPU parity of the cluster kernel that runs the remaining layers of a
-sequence once at most 256 tokens are left (one cluster of H CTAs per sequence,
-all such layers in one launch), against the fp64 oracle.
+sequence once at most TAIL_MAX_LEN (384) tokens are left (one cluster of H CTAs
+per sequence, all such layers in one launch), against the fp64 oracle.
 
-Covered: every layer in the cluster kernel (L <= 256) with a window narrower
-than the sequence and global tokens (masked path), a window that covers every
-pair, cluster sizes H = 4, 12 and 16, more clusters than the GPU holds at once,
-the hand-over from the per-layer kernels in the middle of a stack, empty and
-one-token sequences, and the launch plan the library reports.
+Covered: every layer in the cluster kernel with a window narrower than the
+sequence and global tokens (masked path), a window that covers every pair,
+sequences of one, two and three 128-row tiles (above 256 tokens the keys and
+queries are processed in two halves), cluster sizes H = 4, 12 and 16, more
+clusters than the GPU holds at once, the hand-over from the per-layer kernels
+in the middle of a stack, empty and one-token sequences, and the launch plan the
+library reports.
 """
 import numpy as np
 import pytest
@@ -38,6 +40,12 @@ TAIL_STACKS = [
     wk.Workload("many_clusters_b20", n_layers=3, B=20, L=130, w=40, seed=15),
     wk.Workload("handover_1200", n_layers=5, B=2, L=1200, w=128, n_extra_global=6,
                 salient_frac=0.08, salient_scale=4.0, alpha_first=0.5, alpha_last=1.0, seed=16),
+    # above 256 tokens: two key / query halves per tile
+    wk.Workload("halves_384_w64", n_layers=4, B=2, L=384, w=64, n_extra_global=5, seed=19),
+    wk.Workload("halves_320_full", n_layers=3, B=3, L=320, w=256, n_extra_global=2,
+                ragged=(260, 320), seed=20),
+    wk.Workload("halves_theta_small", n_layers=6, B=2, L=380, w=100, n_extra_global=3,
+                alpha_first=0.05, alpha_last=0.2, seed=21),
 ]
 
 
@@ -48,12 +56,21 @@ def test_tail_stack_matches_oracle(sc, wl):
 
 
 def test_handover_happens_mid_stack(sc):
-    """The hand-over workload really uses both paths: layer 0 has > 256 tokens
-    and a later layer <= 256."""
-    wl = TAIL_STACKS[-1]
+    """The hand-over workload really uses both paths: layer 0 has more than
+    TAIL_MAX_LEN tokens and a later layer at most that many."""
+    wl = next(w for w in TAIL_STACKS if w.name == "handover_1200")
     inp, res, _ = resample_stack(wl)
-    assert (res["len"][0] > 256).all()
-    assert (res["len"][wl.n_layers - 1] <= 256).all()
+    assert (res["len"][0] > sc.TAIL_MAX_LEN).all()
+    assert (res["len"][wl.n_layers - 1] <= sc.TAIL_MAX_LEN).all()
+
+
+def test_halves_cases_have_more_than_two_tiles(sc):
+    """The 'halves' workloads keep more than 256 tokens in some layer, so the
+    two-half path of the cluster kernel runs."""
+    for w in TAIL_STACKS:
+        if w.name.startswith("halves"):
+            _, res, _ = resample_stack(w)
+            assert (res["len"][: w.n_layers] > 256).any(), w.name
 
 
 def test_tail_empty_and_single_token_sequences(sc):
@@ -84,6 +101,7 @@ def test_launch_plan(sc):
     g = [0, 5]
     # every sequence starts in the cluster kernel: global lookup + one launch
     assert sc.stack_launch_count(12, 2, 256, 12, 64, g, False) == 2
+    assert sc.stack_launch_count(12, 2, sc.TAIL_MAX_LEN, 12, 64, g, False) == 2
     # per-layer kernels (rows, cols, and a gather between layers) + the cluster kernel
     assert sc.stack_launch_count(12, 2, 700, 12, 64, g, False) == 1 + 12 * 2 + 11 + 1
     assert sc.stack_launch_count(12, 2, 700, 12, 64, g, True) == 2 + 12 * 2 + 11 + 1

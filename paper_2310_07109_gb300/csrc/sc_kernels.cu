@@ -304,8 +304,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       mbar_init(&sm.bar_sg[X], 1);
       mbar_init(&sm.bar_sgend[X], 1);
       mbar_init(&sm.bar_sfull[X], 1);
-      mbar_init(&sm.bar_sfree[X], 128);
-      mbar_init(&sm.bar_pready[X], 128);
+      mbar_init(&sm.bar_sfree[X], 4);   // one arrival per warp
+      mbar_init(&sm.bar_pready[X], 4);
       mbar_init(&sm.bar_pvdone[X], 1);
       mbar_init(&sm.bar_fin[X], 1);
     }
@@ -478,7 +478,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         tmem_st8(tP + 16, pk);            // P_G
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&sm.bar_pready[X]);
+        warp_arrive(&sm.bar_pready[X]);
         pv_issued = 1;
       }
     }
@@ -508,7 +508,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       }
       tmem_ld_wait();
       tc_fence_before();
-      mbar_arrive(&sm.bar_sfree[X]);   // S is in registers: the next S may overwrite it
+      warp_arrive(&sm.bar_sfree[X]);   // S is in registers: the next S may overwrite it
 #pragma unroll
       for (int ch = 0; ch < 4; ++ch) {
         if (ch < ch_lo || ch > ch_hi) continue;
@@ -576,7 +576,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       lsum += (sa + sb) + (sc2 + sd);
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&sm.bar_pready[X]);
+      warp_arrive(&sm.bar_pready[X]);
       ++pv_issued;
     }
 
@@ -587,23 +587,25 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       tc_fence_after();
       const float inv = 1.f / lsum;
       lse = valid ? m_ref + lg2(lsum) : INFINITY;
-      uint16_t* orow = v.O + ((static_cast<size_t>(b) * p.L + i) * p.H + h) * kHeadDim;
+      // O rows leave through this warp's quarter of its Q tile: every MMA that
+      // read the tile completed before the P V whose completion was awaited
+      uint8_t* stage = Qs + X * kTileBytes + wq * 4096;
 #pragma unroll
       for (int c = 0; c < 64; c += 32) {
         float o[32];
         tmem_ld32(tO + c, o);
         tmem_ld_wait();
-        if (valid) {
 #pragma unroll
-          for (int k = 0; k < 32; k += 8) {
-            uint4 u4 = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
-                                  pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
-                                  pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
-                                  pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
-            *reinterpret_cast<uint4*>(orow + c + k) = u4;
-          }
-        }
+        for (int k = 0; k < 32; k += 8)
+          stage_row_piece<8>(stage, (c + k) >> 3,
+                          make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
+                                     pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
+                                     pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
+                                     pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv)));
       }
+      flush_staged_rows<8>(stage,
+                        v.O + ((static_cast<size_t>(b) * p.L + r0 + 32 * wq) * p.H + h) * kHeadDim,
+                        static_cast<size_t>(p.H) * kHeadDim, __ballot_sync(0xffffffffu, valid));
     }
     if (active && i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
 
@@ -755,9 +757,9 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     }
     for (int X = 0; X < 2; ++X) {
       mbar_init(&sm.bar_sfull[X], 1);
-      mbar_init(&sm.bar_sfree[X], 128);
+      mbar_init(&sm.bar_sfree[X], 4);   // one arrival per warp
       mbar_init(&sm.bar_sg[X], 1);
-      mbar_init(&sm.bar_pg[X], 128);
+      mbar_init(&sm.bar_pg[X], 4);
       mbar_init(&sm.bar_og[X], 1);
     }
     mbar_init(&sm.bar_fin, 1);
@@ -923,7 +925,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
         tmem_ld_wait();
         if (hf == 1) {
           tc_fence_before();
-          mbar_arrive(&sm.bar_sfree[X]);
+          warp_arrive(&sm.bar_sfree[X]);
         }
 #pragma unroll
         for (int c2 = 0; c2 < 2; ++c2) {
@@ -977,7 +979,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
         *reinterpret_cast<uint16_t*>(col + sw128_offset(g, ch) + wi) = pb[g];
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&sm.bar_pg[X]);
+      warp_arrive(&sm.bar_pg[X]);
       bool ok3 = ok2 && warp_wait(&sm.bar_og[X], 0, abort_flag);
       if (wq == 0 && ok3) {
         tc_fence_after();

@@ -17,8 +17,9 @@
 //   columns  per 128-key tile: S^T = K Q^T over the queries in halves, and per
 //            key column j the sum over rows of exp2(S_ij - LSE_i): one thread
 //            per column, no cross-thread sums
-//   heads    the H CTAs exchange their column sums through distributed shared
-//            memory; every CTA adds the heads in the same fixed order, so all
+//   heads    each CTA writes its column sums into every CTA of the cluster
+//            (distributed shared memory) before the cluster barrier; every CTA
+//            then adds the heads in the same fixed order, so all
 //            take the same keep decisions (s_j >= alpha_l / n, j == 0 kept) and
 //            compact the token list the same way, without a second exchange
 //
@@ -44,11 +45,15 @@ constexpr int kTailTiles = (kTailMax + kTile - 1) / kTile;   // 128-row tiles (3
 constexpr uint32_t kTailOpBytes = kTailTiles * kTileBytes;   // rows of one tensor (48 KB)
 constexpr int kTailChunks = kTailMax / 32;                    // 32-token chunks (12)
 static_assert(kTailMax <= 384, "a second key half must fit beside O in tensor memory");
-// Q, K, V operands plus alignment; more than half of an SM's shared memory, so
-// a second CTA never shares the SM (each holds all 512 tensor-memory columns
-// while it waits at cluster barriers: two CTAs of different clusters on one SM
-// could otherwise wait on each other's allocation).
-constexpr uint32_t kTailDyn = 3 * kTailOpBytes + 1024;
+constexpr uint32_t kTailStageBytes = 8 * 2048;                // O row staging, 2 KB per softmax warp
+// column sums of every head, [layer parity][head][column], written by the
+// CTA of that head into every CTA of the cluster
+constexpr uint32_t kTailColBytes = 2 * kTailMaxHeads * kTailMax * 4;
+// Q, K, V operands, the O staging and alignment; more than half of an SM's
+// shared memory, so a second CTA never shares the SM (each holds all 512
+// tensor-memory columns while it waits at cluster barriers: two CTAs of
+// different clusters on one SM could otherwise wait on each other's allocation).
+constexpr uint32_t kTailDyn = 3 * kTailOpBytes + kTailStageBytes + kTailColBytes + 1024;
 static_assert(kTailDyn > 233472 / 2, "the tail kernel must occupy an SM alone");
 
 struct TailSmem {
@@ -56,14 +61,11 @@ struct TailSmem {
   uint32_t tmem_base;
   int abort;
   int n[2];
-  uint32_t kbits[2][8];               // compaction: ballot of kept tokens per (round, warp)
-  int kpre[2][8];                     // ... and the exclusive prefix of their counts
-  int total;
+  alignas(16) uint32_t kbits[2][8];   // compaction: ballot of kept tokens per (round, warp)
   int gpos[kMaxGlobal];               // global positions (sorted), -1 past n_global
   uint32_t gbits[2][kTailChunks];     // global flags of the current / next token list
   int32_t pos[2][kTailMax];           // original positions of the current / next tokens
   alignas(16) float nlse[kTailMax];   // -LSE of each query row (-inf past n)
-  float colsum[2][kTailMax];          // this head's column sums, by layer parity
 };
 
 __device__ __forceinline__ bool tail_is_global(const TailSmem& sm, int ps) {
@@ -147,8 +149,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   if (tid == 0) {
     for (int X = 0; X < 2; ++X) {
       mbar_init(&sm.bar_sfull[X], 1);
-      mbar_init(&sm.bar_sfree[X], 128);
-      mbar_init(&sm.bar_pready[X], 128);
+      mbar_init(&sm.bar_sfree[X], 4);   // one arrival per warp
+      mbar_init(&sm.bar_pready[X], 4);
       mbar_init(&sm.bar_odone[X], 1);
       mbar_init(&sm.bar_stfull[X], 1);
       mbar_init(&sm.bar_fin[X], 1);
@@ -169,9 +171,14 @@ __global__ void __launch_bounds__(kTailThreads, 1)
     const uint32_t bits = __ballot_sync(0xffffffffu, c < n0 && tail_is_global(sm, ps));
     if (lane == 0) sm.gbits[0][c >> 5] = bits;
   }
+  // the CTAs write into each other's shared memory from the first layer on:
+  // each announces that it runs here and waits for the others after its
+  // first gather
+  cluster_arrive_relaxed();
   const uint32_t tm = sm.tmem_base;
   volatile int* abort_flag = &sm.abort;
   const uint32_t q_a = smem_u32(base), k_a = q_a + kTailOpBytes, v_a = k_a + kTailOpBytes;
+  float* const colall = reinterpret_cast<float*>(base + 3 * kTailOpBytes + kTailStageBytes);
   const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
   const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
 
@@ -212,6 +219,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
       cp_async_wait_all();
       fence_proxy_async_smem();
     }
+    if (it == 0) cluster_wait();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -368,7 +376,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
       };
       auto release = [&]() {   // the warpgroup's columns are read
         tc_fence_before();
-        mbar_arrive(&sm.bar_sfree[X]);
+        warp_arrive(&sm.bar_sfree[X]);
       };
 
       // ---- rows: query tiles X and X + 2
@@ -393,13 +401,13 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         const float nmc = me.valid ? -mx * kLogitScale2 : 0.f;
         float lsum = half_exp(me, 0, nmc);
         tc_fence_before();
-        mbar_arrive(&sm.bar_pready[X]);
+        warp_arrive(&sm.bar_pready[X]);
         if (nkh == 2) {
           if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
           tc_fence_after();
           lsum += half_exp(me, 1, nmc);
           tc_fence_before();
-          mbar_arrive(&sm.bar_pready[X]);
+          warp_arrive(&sm.bar_pready[X]);
           if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
         }
         if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
@@ -409,17 +417,21 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         tmem_ld32(tO, o);
         tmem_ld32(tO + 32, o + 32);
         tmem_ld_wait();
-        if (me.valid) {
-          uint16_t* orow =
-              p.O + (((static_cast<size_t>(l) * B + b) * L + i) * H + h) * kHeadDim;
+        // the warp's 32 rows leave in two column halves of 64 bytes
+        uint8_t* stage = base + 3 * kTailOpBytes + warp * 2048;
+        uint16_t* row0 =
+            p.O + (((static_cast<size_t>(l) * B + b) * L + i - (r & 31)) * H + h) * kHeadDim;
+        const uint32_t rows = __ballot_sync(0xffffffffu, me.valid);
 #pragma unroll
-          for (int k = 0; k < 64; k += 8) {
-            const uint4 v = make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
-                                       pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
-                                       pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
-                                       pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv));
-            *reinterpret_cast<uint4*>(orow + k) = v;
-          }
+        for (int c = 0; c < 64; c += 32) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 8)
+            stage_row_piece<4>(stage, k >> 3,
+                               make_uint4(pack_bf16x2(o[c + k] * inv, o[c + k + 1] * inv),
+                                          pack_bf16x2(o[c + k + 2] * inv, o[c + k + 3] * inv),
+                                          pack_bf16x2(o[c + k + 4] * inv, o[c + k + 5] * inv),
+                                          pack_bf16x2(o[c + k + 6] * inv, o[c + k + 7] * inv)));
+          flush_staged_rows<4>(stage, row0 + c, static_cast<size_t>(H) * kHeadDim, rows);
         }
         sm.nlse[i] = me.valid ? -(lg2(lsum) - nmc) : -INFINITY;
         release();
@@ -467,7 +479,11 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         float a0, a1, a2, a3;
         f2_unpack(a2a, a0, a1);
         f2_unpack(a2b, a2, a3);
-        sm.colsum[par][j] = me.valid ? (a0 + a2) + (a1 + a3) : 0.f;
+        // this head's sum of column j goes to every CTA of the cluster; the
+        // cluster barrier below (release / acquire) makes it visible there
+        const float cs = me.valid ? (a0 + a2) + (a1 + a3) : 0.f;
+        const uint32_t la = smem_u32(colall + (par * kTailMaxHeads + h) * kTailMax + j);
+        for (int hh = 0; hh < H; ++hh) st_dsmem_f32(dsmem_addr(la, hh), cs);
       }
     }
 
@@ -482,11 +498,10 @@ __global__ void __launch_bounds__(kTailThreads, 1)
       for (int rd = 0; rd < 2; ++rd) {
         const int j = tid + 256 * rd;
         if (j < n) {
-          const uint32_t la = smem_u32(&sm.colsum[par][j]);
+          const float* cj = colall + par * kTailMaxHeads * kTailMax + j;
           float v[kTailMaxHeads];
 #pragma unroll
-          for (int hh = 0; hh < kTailMaxHeads; ++hh)
-            v[hh] = hh < H ? ld_dsmem_f32(dsmem_addr(la, hh)) : 0.f;
+          for (int hh = 0; hh < kTailMaxHeads; ++hh) v[hh] = hh < H ? cj[hh * kTailMax] : 0.f;
           float a = 0.f;
 #pragma unroll
           for (int hh = 0; hh < kTailMaxHeads; ++hh)
@@ -499,25 +514,29 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         if (lane == 0) sm.kbits[rd][warp] = kb;
       }
       tail_named_sync();
-      if (warp == 0) {
-        // exclusive prefix over (round, warp): 16 entries, one per lane
-        const int cnt = lane < 16 ? __popc(sm.kbits[lane >> 3][lane & 7]) : 0;
-        int x = cnt;
+      // every thread reads the 16 ballot words (round-major, then warp) and
+      // forms its own exclusive prefix and the total
+      int kpre[2] = {0, 0}, total = 0;
+      {
+        const uint4* kw = reinterpret_cast<const uint4*>(&sm.kbits[0][0]);
 #pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-          const int y = __shfl_up_sync(0xffffffffu, x, off);
-          if (lane >= off) x += y;
+        for (int q = 0; q < 4; ++q) {
+          const uint4 u = kw[q];
+          const uint32_t wv[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int idx = 4 * q + e;   // = 8 * round + warp
+            if (idx == warp) kpre[0] = total;
+            if (idx == 8 + warp) kpre[1] = total;
+            total += __popc(wv[e]);
+          }
         }
-        if (lane < 16) sm.kpre[lane >> 3][lane & 7] = x - cnt;
-        if (lane == 31) sm.total = x;
       }
-      tail_named_sync();
-      const int total = sm.total;
 #pragma unroll
       for (int rd = 0; rd < 2; ++rd) {
         if (!keep[rd]) continue;
         const int j = tid + 256 * rd;
-        const int k = sm.kpre[rd][warp] + __popc(sm.kbits[rd][warp] & ((1u << lane) - 1u));
+        const int k = kpre[rd] + __popc(sm.kbits[rd][warp] & ((1u << lane) - 1u));
         const int ps = sm.pos[cur][j];
         sm.pos[nxt][k] = ps;
         if (h == 0) p.pos[(static_cast<size_t>(l + 1) * B + b) * L + k] = ps;

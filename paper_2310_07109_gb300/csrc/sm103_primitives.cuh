@@ -56,6 +56,14 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
+// One arrival per warp (count warps, not threads, at init): the warp's lanes
+// synchronise first, so every lane's preceding fences are ordered before it.
+// Saves the shared-memory unit 31 of 32 atomic updates per warp.
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
 // The waiting thread is suspended until the phase completes or `hint_ns`
 // passes, so waiting warps do not compete for issue slots.
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity,
@@ -294,6 +302,15 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 
 // Every thread of every CTA of the cluster arrives (release) and waits
 // (acquire); called by whole, converged warps.
+// Split cluster barrier: arrive without ordering (only "this CTA is running"),
+// and the matching wait.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void cluster_sync() {
   asm volatile(
       "barrier.cluster.arrive.release.aligned;\n\t"
@@ -312,6 +329,10 @@ __device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
   float v;
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
   return v;
+}
+
+__device__ __forceinline__ void st_dsmem_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
 }
 
 // 16-byte global -> shared copy through the load/store path (no register
@@ -411,6 +432,38 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
+}
+
+// Coalesced store of a warp's 32 bf16 rows (one row per lane, kPieces 16-byte
+// pieces: 8 for 128-byte rows, 4 for 64-byte rows) through a 32 * kPieces * 16
+// byte shared-memory staging area.  Each lane first stages its pieces
+// (XOR-swizzled by row, so that every 8-lane phase of a 16-byte access covers
+// all 32 banks); the flush reads them back so that kPieces consecutive lanes
+// cover one row, and each store instruction writes whole rows of several
+// tokens instead of one piece of 32 different rows.
+template <int kPieces>
+__device__ __forceinline__ uint32_t stage_offset(int r, int c) {
+  static_assert(kPieces == 8 || kPieces == 4, "128- or 64-byte rows");
+  return kPieces == 8 ? r * 128 + ((c ^ (r & 7)) << 4) : r * 64 + ((c ^ ((r >> 1) & 3)) << 4);
+}
+template <int kPieces>
+__device__ __forceinline__ void stage_row_piece(uint8_t* stage, int c, uint4 v) {
+  *reinterpret_cast<uint4*>(stage + stage_offset<kPieces>(threadIdx.x & 31, c)) = v;
+}
+// Row r of the warp goes to row0 + r * row_stride (elements) when bit r of
+// rows_mask is set; rows whose bit is clear are not written.
+template <int kPieces>
+__device__ __forceinline__ void flush_staged_rows(const uint8_t* stage, uint16_t* row0,
+                                                  size_t row_stride, uint32_t rows_mask) {
+  __syncwarp();
+  const int lane = threadIdx.x & 31, c = lane % kPieces;
+#pragma unroll
+  for (int k = 0; k < kPieces; ++k) {
+    const int r = (32 / kPieces) * k + lane / kPieces;
+    const uint4 v = *reinterpret_cast<const uint4*>(stage + stage_offset<kPieces>(r, c));
+    if ((rows_mask >> r) & 1u) *reinterpret_cast<uint4*>(row0 + r * row_stride + 8 * c) = v;
+  }
+  __syncwarp();   // the staging area may be written again
 }
 
 // 128-byte swizzle: byte offset of 16-byte chunk `c` (0..7) of row `r` inside

@@ -231,6 +231,13 @@ __device__ __forceinline__ void mma_pv_ts(uint32_t d_tmem, uint32_t p_tmem, uint
                  (accumulate || k > 0) ? 1u : 0u);
 }
 
+// Bits lo..hi (inclusive, clipped to 0..31) of a 32-bit word; 0 when empty.
+__device__ __forceinline__ uint32_t bit_range32(int lo, int hi) {
+  lo = max(lo, 0);
+  hi = min(hi, 31);
+  return hi < lo ? 0u : ((0xffffffffu >> (31 - hi)) & (0xffffffffu << lo));
+}
+
 // Reduce 16 values per lane over the warp (butterfly reduce-scatter, 16
 // shuffles): lane L returns the warp-wide result for element L >> 1.
 template <typename Op>
@@ -443,9 +450,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     // is used for rows whose results are discarded (global rows, rows >= n)
     const int lo = max(0, i - p.w);
     const int hi = min(n - 1, i + p.w);
-    // union of the band over this warp's 32 rows: chunks outside it are skipped
-    const int wlo = max(0, r0 + 32 * wq - p.w);
-    const int whi = min(n - 1, r0 + 32 * wq + 31 + p.w);
 
     float m_ref = -INFINITY, lsum = 0.f;
     bool ok = active;
@@ -487,47 +491,48 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     // The tile's maximum is taken before its exponentials; when it exceeds the
     // reference by more than 8, the reference is raised and O (all earlier
     // P V complete) and the row sum are rescaled exactly.  P stays below 2^8.
+    // All exponentials of the tile are formed in registers before the previous
+    // P V is awaited: only the P store and a rescale of O depend on it.
     const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
     for (int t = 0; ok && t <= khiX - kloX; ++t) {
       const int j0 = (kloX + t) * kTile;
-      // 32-column chunks of this tile that intersect the warp's band
-      const int clo = max(0, wlo - j0), chi = min(kTile - 1, whi - j0);
-      const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
-      const int a = lo - j0, e = hi - j0;
+      const int a = lo - j0, e = hi - j0;   // this row's allowed columns of the tile
       if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
       float x[128];
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        if (ch >= ch_lo && ch <= ch_hi) {
-          tmem_ld32(tS + 32 * ch, x + 32 * ch);
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) x[32 * ch + k] = -INFINITY;
-        }
-      }
+      for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + 32 * ch, x + 32 * ch);
       tmem_ld_wait();
       tc_fence_before();
       warp_arrive(&sm.bar_sfree[X]);   // S is in registers: the next S may overwrite it
+      // keys outside a row's band take no part; tiles inside the band of all
+      // 32 rows of the warp (most of them) need no mask
+      if (!__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        if (ch < ch_lo || ch > ch_hi) continue;
-        if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
-          // edge chunk: keys outside this row's band take no part
+        for (int ch = 0; ch < 4; ++ch) {
+          // this row's allowed keys among the chunk's 32, as bits; chunks
+          // that every row of the warp takes whole are left alone
+          const uint32_t keep = bit_range32(a - 32 * ch, e - 32 * ch);
+          if (__any_sync(0xffffffffu, keep != 0xffffffffu)) {
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            const int c = 32 * ch + k;
-            x[32 * ch + k] = (c >= a && c <= e) ? x[32 * ch + k] : -INFINITY;
+            for (int k = 0; k < 32; ++k) {
+              const uint32_t out =
+                  ~static_cast<uint32_t>(static_cast<int32_t>(keep << (31 - k)) >> 31);
+              x[32 * ch + k] =
+                  __uint_as_float((__float_as_uint(x[32 * ch + k]) & ~out) | (0xff800000u & out));
+            }
           }
         }
       }
-      float m0 = x[0], m1 = x[1];
+      float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int k = 2; k < 128; k += 4) {
-        m0 = fmax3(m0, x[k], x[k + 1]);
-        m1 = fmax3(m1, x[k + 2], x[k + 3]);
+      for (int k = 0; k < kTile; k += 8) {
+        m4[0] = fmax3(m4[0], x[k], x[k + 1]);
+        m4[1] = fmax3(m4[1], x[k + 2], x[k + 3]);
+        m4[2] = fmax3(m4[2], x[k + 4], x[k + 5]);
+        m4[3] = fmax3(m4[3], x[k + 6], x[k + 7]);
       }
-      const float tmax = fmaxf(m0, m1) * kLogitScale2;
+      const float tmax = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * kLogitScale2;
       const bool raise = tmax > m_ref + 8.f;
       float f = 1.f;
       if (raise) {
@@ -535,6 +540,24 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         m_ref = tmax;
         lsum *= f;
       }
+      const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
+      const uint64_t n2 = f2_pack(nref, nref);
+      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+      uint32_t pk[64];
+#pragma unroll
+      for (int k = 0; k < kTile; k += 2) {
+        float u, w;
+        f2_unpack(f2_fma(f2_pack(x[k], x[k + 1]), c2, n2), u, w);
+        u = ex2(u);
+        w = ex2(w);
+        if (k & 2) s2b = f2_add(s2b, f2_pack(u, w));
+        else s2a = f2_add(s2a, f2_pack(u, w));
+        pk[k >> 1] = pack_bf16x2(u, w);
+      }
+      float sa, sb, sc2, sd;
+      f2_unpack(s2a, sa, sb);
+      f2_unpack(s2b, sc2, sd);
+      lsum += (sa + sb) + (sc2 + sd);
       // every earlier P V has completed: O is final for a rescale and the P
       // columns of this warpgroup are free again
       if (pv_issued > 0 && !(ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag)))
@@ -552,28 +575,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
           tmem_st_wait();   // o is reused
         }
       }
-      const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
-      const uint64_t n2 = f2_pack(nref, nref);
-      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {   // 32 keys = 16 columns of P per step
-        uint32_t pk[16];
-#pragma unroll
-        for (int k = 0; k < 32; k += 2) {
-          float u, w;
-          f2_unpack(f2_fma(f2_pack(x[32 * ch + k], x[32 * ch + k + 1]), c2, n2), u, w);
-          u = ex2(u);
-          w = ex2(w);
-          if (k & 2) s2b = f2_add(s2b, f2_pack(u, w));
-          else s2a = f2_add(s2a, f2_pack(u, w));
-          pk[k >> 1] = pack_bf16x2(u, w);
-        }
-        tmem_st16(tP + 16 * ch, pk);
-      }
-      float sa, sb, sc2, sd;
-      f2_unpack(s2a, sa, sb);
-      f2_unpack(s2b, sc2, sd);
-      lsum += (sa + sb) + (sc2 + sd);
+      for (int ch = 0; ch < 4; ++ch) tmem_st16(tP + 16 * ch, pk + 16 * ch);
       tmem_st_wait();
       tc_fence_before();
       warp_arrive(&sm.bar_pready[X]);

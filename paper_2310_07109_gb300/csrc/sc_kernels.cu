@@ -689,7 +689,7 @@ struct ColsSmem {
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  alignas(16) float lse[kPairTiles * kTile];  // read as float4
+  alignas(16) float nlse[kPairTiles * kTile];  // -LSE of the band's query rows, read as float4
   float gsum[kMaxGlobal];
   int flag;
   float wpart[kColsThreads / 32];
@@ -882,7 +882,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
 #pragma unroll
     for (int u = 0; u < 3; ++u) {
       const int k = tid + 256 * u;
-      if (k < nq * kTile) sm.lse[k] = lv[u];
+      if (k < nq * kTile) sm.nlse[k] = -lv[u];
     }
 #pragma unroll
     for (int gg = 0; gg < 2; ++gg) {
@@ -899,61 +899,54 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     }
     asm volatile("bar.sync 3, 256;" ::: "memory");
 
-    // union of the band over this warp's 32 key columns
-    const int wlo = max(0, j0 + 32 * wq - p.w);
-    const int whi = min(n - 1, j0 + 32 * wq + 31 + p.w);
     float acc = 0.f;
     bool ok = active;
-    float x[64];
+    float x[128];
+    const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
     for (int t = 0; ok && t <= qhiX - qloX; ++t) {
       const int i0 = (qloX + t) * kTile;            // first query row of this tile
-      const int clo = max(0, wlo - i0), chi = min(kTile - 1, whi - i0);
-      const int ch_lo = clo >> 5, ch_hi = chi >= clo ? (chi >> 5) : -1;
+      // rows i0+a .. i0+e are in j's band (and in the sequence)
+      const int a = j - p.w - i0, e = min(j + p.w, n - 1) - i0;
       if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
       tc_fence_after();
-      const float* lw = sm.lse + (qloX + t - qt_lo) * kTile;
-      const int a = j - p.w - i0, e = j + p.w - i0;  // rows i0+a .. i0+e are in j's band
-      float ps[8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
-      // two halves of 64 columns: load both chunks of a half, then use them;
-      // S^T is released to the next MMA once the second half is in registers
+      for (int ch = 0; ch < 4; ++ch) tmem_ld32(tST + lane_off + 32 * ch, x + 32 * ch);
+      tmem_ld_wait();
+      tc_fence_before();
+      warp_arrive(&sm.bar_sfree[X]);   // S^T is in registers: the next may overwrite it
+      // rows outside this key's band contribute nothing; tiles inside the band
+      // of all 32 keys of the warp (most of them) need no mask
+      if (!__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-#pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          const int ch = 2 * hf + c2;
-          if (ch >= ch_lo && ch <= ch_hi) tmem_ld32(tST + lane_off + 32 * ch, x + 32 * c2);
-        }
-        tmem_ld_wait();
-        if (hf == 1) {
-          tc_fence_before();
-          warp_arrive(&sm.bar_sfree[X]);
-        }
-#pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          const int ch = 2 * hf + c2;
-          if (ch < ch_lo || ch > ch_hi) continue;
-          if (!__all_sync(0xffffffffu, a <= 32 * ch && e >= 32 * ch + 31)) {
-            // edge chunk: rows outside this key's band contribute nothing
+        for (int ch = 0; ch < 4; ++ch) {
+          const uint32_t keep = bit_range32(a - 32 * ch, e - 32 * ch);
+          if (__any_sync(0xffffffffu, keep != 0xffffffffu)) {
 #pragma unroll
             for (int k = 0; k < 32; ++k) {
-              const int c = 32 * ch + k;
-              x[32 * c2 + k] = (c >= a && c <= e) ? x[32 * c2 + k] : -INFINITY;
+              const uint32_t out =
+                  ~static_cast<uint32_t>(static_cast<int32_t>(keep << (31 - k)) >> 31);
+              x[32 * ch + k] =
+                  __uint_as_float((__float_as_uint(x[32 * ch + k]) & ~out) | (0xff800000u & out));
             }
-          }
-#pragma unroll
-          for (int k = 0; k < 32; k += 4) {
-            const float4 l4 = *reinterpret_cast<const float4*>(lw + 32 * ch + k);
-            const int u = (k >> 2) & 1;
-            ps[4 * u + 0] += ex2(fmaf(x[32 * c2 + k + 0], kLogitScale2, -l4.x));
-            ps[4 * u + 1] += ex2(fmaf(x[32 * c2 + k + 1], kLogitScale2, -l4.y));
-            ps[4 * u + 2] += ex2(fmaf(x[32 * c2 + k + 2], kLogitScale2, -l4.z));
-            ps[4 * u + 3] += ex2(fmaf(x[32 * c2 + k + 3], kLogitScale2, -l4.w));
           }
         }
       }
-      acc += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      // sum over the tile's rows of exp2(S^T scaled - LSE_i)
+      const float* lw = sm.nlse + (qloX + t - qt_lo) * kTile;
+      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+#pragma unroll
+      for (int k = 0; k < kTile; k += 4) {
+        const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
+        float e0, e1, e2, e3;
+        f2_unpack(f2_fma(f2_pack(x[k], x[k + 1]), c2, f2_pack(l4.x, l4.y)), e0, e1);
+        f2_unpack(f2_fma(f2_pack(x[k + 2], x[k + 3]), c2, f2_pack(l4.z, l4.w)), e2, e3);
+        s2a = f2_add(s2a, f2_pack(ex2(e0), ex2(e1)));
+        s2b = f2_add(s2b, f2_pack(ex2(e2), ex2(e3)));
+      }
+      float sa, sb, sc2, sd;
+      f2_unpack(s2a, sa, sb);
+      f2_unpack(s2b, sc2, sd);
+      acc += (sa + sc2) + (sb + sd);
     }
 
     if (active && ngp) {

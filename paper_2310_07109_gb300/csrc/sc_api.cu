@@ -47,7 +47,8 @@ int fail_cuda(const char* what, cudaError_t e) {
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
-  size_t status, lse, acc, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident, tail_from,
+  size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident,
+      tail_from,
       loop_layer, qkv, total;
 };
 
@@ -61,8 +62,8 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
     return at;
   };
   w->status = take(kAlign);
-  w->lse = take(sizeof(float) * B * H * (size_t)L);
   w->acc = take(sizeof(float) * B * H * (size_t)L);
+  w->colpart = take(sizeof(float) * B * H * (size_t)L * kMaxBandTiles);
   w->gpart = take(sizeof(float) * B * H * T * 4 * kMaxGlobal);
   w->gstat = take(sizeof(float) * B * H * T * 4 * kMaxGlobal * 2);
   w->og = take(sizeof(float) * B * H * kMaxGlobal * kHeadDim);
@@ -236,8 +237,8 @@ int check_common(int B, int L, int H, int w, const int32_t* gpos, int ngl) {
 
 void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->status = reinterpret_cast<int*>(ws + lay.status);
-  p->lse = reinterpret_cast<float*>(ws + lay.lse);
   p->acc = reinterpret_cast<float*>(ws + lay.acc);
+  p->colpart = reinterpret_cast<float*>(ws + lay.colpart);
   p->gpart = reinterpret_cast<float*>(ws + lay.gpart);
   p->gstat = reinterpret_cast<float*>(ws + lay.gstat);
   p->og = reinterpret_cast<float*>(ws + lay.og);

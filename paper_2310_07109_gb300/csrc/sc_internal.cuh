@@ -62,8 +62,9 @@ struct LayerParams {
   float alpha;           // theta_b = alpha / n_b unless theta != nullptr
   const float* theta;    // [B] absolute thresholds or nullptr
   // workspace
-  float* lse;            // [B][H][L] per-row log2-sum-exp2 (+inf for global rows)
   float* acc;            // [B][H][L] per-head column sums: band rows + global rows
+  float* colpart;        // [B][H][L][kMaxBandTiles] band-row column sums per query tile
+                         //   (slot = query tile mod kMaxBandTiles)
   float* gpart;          // [B][H][T][4][kMaxGlobal] column sums of global keys over far rows,
                          //   per (query tile, 32-row warp slice)
   float* gstat;          // [B][H][T][4][kMaxGlobal][2] (max, sum) of global rows per

@@ -40,6 +40,11 @@ namespace sc {
 // ---------------------------------------------------------------------------
 // small helpers
 // ---------------------------------------------------------------------------
+// Barrier over the four warps of softmax warpgroup X (ids 2 and 3).
+__device__ __forceinline__ void named_sync_wg(int X) {
+  asm volatile("bar.sync %0, 128;" ::"r"(2 + X) : "memory");
+}
+
 __device__ __forceinline__ void named_sync_softmax() {
   asm volatile("bar.sync 1, 128;" ::: "memory");
 }
@@ -155,11 +160,12 @@ __device__ __forceinline__ void mma_qk(uint32_t d_tmem, uint32_t a_smem, uint32_
 // Issue D[128 x 64] (+)= P[128 x 16*ksteps] * V[16*ksteps x 64]: P is a K-major
 // 128B-swizzled tile in two 64-key halves of 16 KB, V an MN-major tile of
 // 128-byte key rows.
-__device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_t v_smem,
-                                       int ksteps, bool accumulate) {
+// P (A, K-major, 64-key blocks p_block bytes apart) from shared memory.
+__device__ __forceinline__ void mma_pv(uint32_t d_tmem, uint32_t p_smem, uint32_t p_block,
+                                       uint32_t v_smem, int ksteps, bool accumulate) {
   const uint32_t idesc = idesc_bf16(128, 64, false, true);
   for (int k = 0; k < ksteps; ++k)
-    umma_bf16(d_tmem, sdesc_sw128(p_smem + (k >> 2) * 16384 + (k & 3) * 32),
+    umma_bf16(d_tmem, sdesc_sw128(p_smem + (k >> 2) * p_block + (k & 3) * 32),
               sdesc_sw128(v_smem + k * 2048), idesc, (accumulate || k > 0) ? 1u : 0u);
 }
 
@@ -207,6 +213,7 @@ __host__ __device__ constexpr uint32_t col_p(int X) { return 256u * X + 128u; }
 __host__ __device__ constexpr uint32_t col_o(int X) { return 256u * X + 192u; }
 
 struct RowsSmem {
+  alignas(16) float nlse[2][kTile];   // -LSE of each query tile's rows (read as float4)
   uint64_t bar_q;
   uint64_t bar_kfull[kPairTiles];
   uint64_t bar_vfull[kVStages], bar_vempty[kVStages];
@@ -424,6 +431,16 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         if (k + kVStages < nk) umma_commit(&sm.bar_vempty[k % kVStages]);   // slot reused
         umma_commit(&sm.bar_pvdone[X]);
       }
+      // band pass: S^T = K Q^T of each key tile of the band against this
+      // query tile, into the S columns once they are read (after the S_G /
+      // S_Gt of the epilogue, when there are global keys)
+      for (int a = kloX; ok && a <= khiX; ++a) {
+        if ((a > kloX || ngp) && !(ok = mbar_wait(&sm.bar_sfree[X], (nfree++) & 1, abort_flag)))
+          break;
+        tc_fence_after();
+        mma_qk(tS, k_a + (a - kt_lo) * kTileBytes, q_a, 128);
+        umma_commit(&sm.bar_sfull[X]);
+      }
       umma_commit(&sm.bar_fin[X]);
       drain_wait(&sm.bar_fin[X], 0);
     }
@@ -583,34 +600,13 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       ++pv_issued;
     }
 
-    // ---- epilogue: O, LSE
+    // ---- epilogue: LSE, the global keys and queries, the band's column
+    // sums, O
     float lse = INFINITY;
-    if (ok && pv_issued > 0 &&
-        (ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag))) {
-      tc_fence_after();
-      const float inv = 1.f / lsum;
-      lse = valid ? m_ref + lg2(lsum) : INFINITY;
-      // O rows leave through this warp's quarter of its Q tile: every MMA that
-      // read the tile completed before the P V whose completion was awaited
-      uint8_t* stage = Qs + X * kTileBytes + wq * 4096;
-#pragma unroll
-      for (int c = 0; c < 64; c += 32) {
-        float o[32];
-        tmem_ld32(tO + c, o);
-        tmem_ld_wait();
-#pragma unroll
-        for (int k = 0; k < 32; k += 8)
-          stage_row_piece<8>(stage, (c + k) >> 3,
-                          make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
-                                     pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
-                                     pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
-                                     pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv)));
-      }
-      flush_staged_rows<8>(stage,
-                        v.O + ((static_cast<size_t>(b) * p.L + r0 + 32 * wq) * p.H + h) * kHeadDim,
-                        static_cast<size_t>(p.H) * kHeadDim, __ballot_sync(0xffffffffu, valid));
-    }
-    if (active && i < n) p.lse[(static_cast<size_t>(b) * p.H + h) * p.L + i] = lse;
+    const bool have_o = ok && pv_issued > 0 &&
+                        (ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag));
+    if (have_o) lse = valid ? m_ref + lg2(lsum) : INFINITY;
+    if (active) sm.nlse[X][r] = -lse;
 
     if (active && ngp) {
       // Per-warp partial results (32 rows / 32 keys each), reduced with
@@ -659,6 +655,88 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
         for (int k = r; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
       }
+      // S_G and S_Gt are read: the S columns take the band pass
+      tc_fence_before();
+      warp_arrive(&sm.bar_sfree[X]);
+    }
+
+    // Band pass (the column sums of Sec. "Extractor of Attention Scores"):
+    // for each key j of the band, the sum over this tile's rows i of
+    // exp2(S_ij scaled - LSE_i); global rows (LSE = +inf) and rows past the
+    // end add nothing.  One thread per key column of S^T; written per query
+    // tile, summed over query tiles and heads in a fixed order by the
+    // finalisation.
+    if (active) named_sync_wg(X);   // every -LSE of the tile is in shared memory
+    const int nt = khiX - kloX + 1;
+    const uint64_t c2b = f2_pack(kLogitScale2, kLogitScale2);
+    for (int u = 0; ok && u < nt; ++u) {
+      const int j = (kloX + u) * kTile + r;   // key of this thread
+      if (!(ok = warp_wait(&sm.bar_sfull[X], (nt + u) & 1, abort_flag))) break;
+      tc_fence_after();
+      float x[128];
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch) tmem_ld32(tS + 32 * ch, x + 32 * ch);
+      tmem_ld_wait();
+      tc_fence_before();
+      warp_arrive(&sm.bar_sfree[X]);   // S^T is in registers
+      // query columns r0 + a .. r0 + e are in j's band (and in the sequence)
+      const int a = j - p.w - r0, e = min(j + p.w, n - 1) - r0;
+      if (!__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          const uint32_t keep = bit_range32(a - 32 * ch, e - 32 * ch);
+          if (__any_sync(0xffffffffu, keep != 0xffffffffu)) {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) {
+              const uint32_t out =
+                  ~static_cast<uint32_t>(static_cast<int32_t>(keep << (31 - k)) >> 31);
+              x[32 * ch + k] =
+                  __uint_as_float((__float_as_uint(x[32 * ch + k]) & ~out) | (0xff800000u & out));
+            }
+          }
+        }
+      }
+      const float* lw = sm.nlse[X];
+      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+#pragma unroll
+      for (int k = 0; k < kTile; k += 4) {
+        const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
+        float e0, e1, e2, e3;
+        f2_unpack(f2_fma(f2_pack(x[k], x[k + 1]), c2b, f2_pack(l4.x, l4.y)), e0, e1);
+        f2_unpack(f2_fma(f2_pack(x[k + 2], x[k + 3]), c2b, f2_pack(l4.z, l4.w)), e2, e3);
+        s2a = f2_add(s2a, f2_pack(ex2(e0), ex2(e1)));
+        s2b = f2_add(s2b, f2_pack(ex2(e2), ex2(e3)));
+      }
+      float sa, sb, sc2, sd;
+      f2_unpack(s2a, sa, sb);
+      f2_unpack(s2b, sc2, sd);
+      if (j < n)
+        p.colpart[((static_cast<size_t>(b) * p.H + h) * p.L + j) * kMaxBandTiles + qt % kMaxBandTiles] =
+            (sa + sc2) + (sb + sd);
+    }
+
+    // ---- O: its rows leave through this warp's quarter of its Q tile; every
+    // MMA that read the tile completed before the last S^T was awaited
+    if (ok && have_o) {
+      tc_fence_after();
+      const float inv = 1.f / lsum;
+      uint8_t* stage = Qs + X * kTileBytes + wq * 4096;
+#pragma unroll
+      for (int c = 0; c < 64; c += 32) {
+        float o[32];
+        tmem_ld32(tO + c, o);
+        tmem_ld_wait();
+#pragma unroll
+        for (int k = 0; k < 32; k += 8)
+          stage_row_piece<8>(stage, (c + k) >> 3,
+                          make_uint4(pack_bf16x2(o[k] * inv, o[k + 1] * inv),
+                                     pack_bf16x2(o[k + 2] * inv, o[k + 3] * inv),
+                                     pack_bf16x2(o[k + 4] * inv, o[k + 5] * inv),
+                                     pack_bf16x2(o[k + 6] * inv, o[k + 7] * inv)));
+      }
+      flush_staged_rows<8>(stage,
+                        v.O + ((static_cast<size_t>(b) * p.L + r0 + 32 * wq) * p.H + h) * kHeadDim,
+                        static_cast<size_t>(p.H) * kHeadDim, __ballot_sync(0xffffffffu, valid));
     }
   }
 
@@ -675,21 +753,26 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 // cols kernel
 // ---------------------------------------------------------------------------
 // One CTA per pair of 128-key tiles (2p, 2p+1) of one (sequence, head), one
-// softmax warpgroup per key tile; the two share the query tiles of their band.
-// Tensor memory per warpgroup X: S^T [128 X, 128 X + 128), S^T against the
-// global queries [256 + 16 X, +16), the global rows' P V [320 + 64 X, +64).
+// warpgroup per key tile.  The band rows' column sums come from the rows
+// kernel (one partial per query tile); here: the global rows' P over the
+// pair's keys and their P V, the keys' column sums, and the finalisation.
+// Tensor memory (256 columns, so that two CTAs share an SM) per warpgroup X:
+// S^T against the global queries [16 X, +16), the global rows' P V
+// [64 + 64 X, +64).
 constexpr int kColsThreads = 320;
-constexpr int kColsStages = 4;      // Q ring depth
+// The global rows' P is the A operand of an M = 128 MMA whose rows past the 16
+// global rows are never used: each 64-key block of that A tile holds its 16
+// valid rows (2 KB) and lets the MMA read the following rows from whatever
+// shared memory comes next (the K and V tiles), so only 2 KB is reserved.
+constexpr uint32_t kPgBlock = 2 * 1024;
 
 struct ColsSmem {
   uint64_t bar_kv;
-  uint64_t bar_qfull[kColsStages], bar_qempty[kColsStages];
   uint64_t bar_sfull[2], bar_sfree[2], bar_sg[2], bar_pg[2], bar_og[2], bar_fin;
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  alignas(16) float nlse[kPairTiles * kTile];  // -LSE of the band's query rows, read as float4
   float gsum[kMaxGlobal];
   int flag;
   float wpart[kColsThreads / 32];
@@ -702,14 +785,16 @@ struct ColsSmem {
   int total;
 };
 
-// dynamic shared memory: K and V of both key tiles, the Q ring, the global
-// queries, and one A tile (32 KB) per warpgroup for the global rows' P V
-constexpr uint32_t kColsDyn = kTileBytes * (4 + kColsStages) + kGTileBytes + 4 * kTileBytes + 1024;
+// dynamic shared memory: the global rows' P blocks (2 per warpgroup), K and V
+// of both key tiles, the global queries
+constexpr uint32_t kColsDyn = 4 * kPgBlock + kTileBytes * 4 + kGTileBytes + 1024;
+static_assert(3 * kPgBlock + kTileBytes <= 4 * kPgBlock + 4 * kTileBytes,
+              "the A operand's unused rows stay inside the shared memory");
 
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
                                   ColsSmem& sm);
 
-__global__ void __launch_bounds__(kColsThreads, 1)
+__global__ void __launch_bounds__(kColsThreads, 2)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
   const LayerView v = layer_view(p);
@@ -733,11 +818,10 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   extern __shared__ uint8_t dyn_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* Ks = base;                              // 2 tiles
+  uint8_t* Pg = base;                              // 2 x 2 blocks of 16 rows
+  uint8_t* Ks = Pg + 4 * kPgBlock;                 // 2 tiles
   uint8_t* Vs = Ks + 2 * kTileBytes;               // 2 tiles
-  uint8_t* Pg = Vs + 2 * kTileBytes;               // 2 x 32 KB A tiles
-  uint8_t* Qs = Pg + 4 * kTileBytes;               // kColsStages tiles
-  uint8_t* QG = Qs + kColsStages * kTileBytes;
+  uint8_t* QG = Vs + 2 * kTileBytes;
   __shared__ ColsSmem sm;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -748,16 +832,9 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     qlo[X] = max(0, j0 - p.w) / kTile;
     qhi[X] = min(n - 1, j1 + p.w) / kTile;
   }
-  const int qt_lo = qlo[0];
-  const int qt_hi = hasB ? qhi[1] : qhi[0];
-  const int nq = qt_hi - qt_lo + 1;
 
   if (tid == 0) {
     mbar_init(&sm.bar_kv, 1);
-    for (int s = 0; s < kColsStages; ++s) {
-      mbar_init(&sm.bar_qfull[s], 1);
-      mbar_init(&sm.bar_qempty[s], 1);
-    }
     for (int X = 0; X < 2; ++X) {
       mbar_init(&sm.bar_sfull[X], 1);
       mbar_init(&sm.bar_sfree[X], 4);   // one arrival per warp
@@ -770,7 +847,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldcg(v.gcur + b * kMaxGlobal + tid) : -1;
-  if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
+  if (warp == 9) tmem_alloc(&sm.tmem_base, 256);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -788,54 +865,25 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     }
     __syncwarp();
     if (ngp) load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_kv, lane);
-    if (lane == 0) {
-      bool ok = true;
-      for (int q = 0; ok && q < nq; ++q) {
-        const int s = q % kColsStages;
-        if (q >= kColsStages &&
-            !(ok = mbar_wait(&sm.bar_qempty[s], ((q / kColsStages) - 1) & 1, abort_flag)))
-          break;
-        mbar_arrive_expect_tx(&sm.bar_qfull[s], kTileBytes);
-        load_tile(maps, 0, rs, h, (qt_lo + q) * kTile, Qs + s * kTileBytes, &sm.bar_qfull[s]);
-      }
-      drain_wait(&sm.bar_kv, 0);
-      for (int s = 0; s < kColsStages && s < nq; ++s) {
-        const int last = s + kColsStages * ((nq - 1 - s) / kColsStages);
-        drain_wait(&sm.bar_qfull[s], (last / kColsStages) & 1);
-      }
-    }
+    if (lane == 0) drain_wait(&sm.bar_kv, 0);
   } else if (warp == 9) {
     if (lane == 0) {
-      const uint32_t k_a = smem_u32(Ks), q_a = smem_u32(Qs), v_a = smem_u32(Vs);
+      const uint32_t k_a = smem_u32(Ks), v_a = smem_u32(Vs);
       const int nX = hasB ? 2 : 1;
-      int su[2] = {0, 0};   // S^T tiles issued per warpgroup
       bool ok = mbar_wait(&sm.bar_kv, 0, abort_flag);
       if (ok) {
         tc_fence_after();
         if (ngp)
           for (int X = 0; X < nX; ++X) {
-            mma_qk(tm + 256 + 16 * X, k_a + X * kTileBytes, smem_u32(QG), 16);
+            mma_qk(tm + 16 * X, k_a + X * kTileBytes, smem_u32(QG), 16);
             umma_commit(&sm.bar_sg[X]);
           }
-      }
-      for (int q = 0; ok && q < nq; ++q) {
-        const int s = q % kColsStages, a = qt_lo + q;
-        if (!(ok = mbar_wait(&sm.bar_qfull[s], (q / kColsStages) & 1, abort_flag))) break;
-        for (int X = 0; ok && X < nX; ++X) {
-          if (a < (X ? qlo[1] : qlo[0]) || a > (X ? qhi[1] : qhi[0])) continue;
-          if (su[X] > 0 && !(ok = mbar_wait(&sm.bar_sfree[X], (su[X] - 1) & 1, abort_flag))) break;
-          tc_fence_after();
-          mma_qk(tm + 128 * X, k_a + X * kTileBytes, q_a + s * kTileBytes, 128);
-          umma_commit(&sm.bar_sfull[X]);
-          ++su[X];
-        }
-        if (ok) umma_commit(&sm.bar_qempty[s]);
       }
       if (ok && ngp)
         for (int X = 0; ok && X < nX; ++X) {
           if (!(ok = mbar_wait(&sm.bar_pg[X], 0, abort_flag))) break;
           tc_fence_after();
-          mma_pv(tm + 320 + 64 * X, smem_u32(Pg) + X * 2 * kTileBytes, v_a + X * kTileBytes,
+          mma_pv(tm + 64 + 64 * X, smem_u32(Pg) + X * 2 * kPgBlock, kPgBlock, v_a + X * kTileBytes,
                  kTile / 16, false);
           umma_commit(&sm.bar_og[X]);
         }
@@ -852,17 +900,18 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     const int j = j0 + r;             // key column owned by this thread
     const bool active = X == 0 || hasB;
     const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
-    const uint32_t tST = tm + 128 * X, tSG = tm + 256 + 16 * X, tOG = tm + 320 + 64 * X;
-    // every load of the prologue is issued before any is used: the LSE of the
-    // query rows of the band (at most kPairTiles * 128 = 3 * 256) and, per
-    // warp, the (max, sum) pieces of global rows warp and warp + 8
-    static_assert(kPairTiles * kTile <= 3 * 256, "LSE window exceeds three loads a thread");
-    const float* lse_src = p.lse + (static_cast<size_t>(b) * p.H + h) * p.L;
-    float lv[3];
+    const uint32_t tSG = tm + 16 * X, tOG = tm + 64 + 64 * X;
+    // every load of the prologue is issued before any is used: this key's
+    // band-row column sums of the query tiles of its band (one per tile, from
+    // the rows kernel) and, per warp, the (max, sum) pieces of global rows
+    // warp and warp + 8
+    float part[kMaxBandTiles];
+    const float* cp =
+        p.colpart + ((static_cast<size_t>(b) * p.H + h) * p.L + j) * kMaxBandTiles;
 #pragma unroll
-    for (int u = 0; u < 3; ++u) {
-      const int k = tid + 256 * u, row = qt_lo * kTile + k;
-      lv[u] = (k < nq * kTile && row < n) ? __ldcg(lse_src + row) : INFINITY;
+    for (int u = 0; u < kMaxBandTiles; ++u) {
+      const int q = qloX + u;
+      part[u] = (active && j < n && q <= qhiX) ? __ldcg(cp + q % kMaxBandTiles) : 0.f;
     }
     // lane k takes entries k, k+32, k+64, k+96 of the 4 Tn (key tile, warp
     // slice) pieces; the warp combines them in a fixed order
@@ -880,11 +929,6 @@ __global__ void __launch_bounds__(kColsThreads, 1)
       }
     }
 #pragma unroll
-    for (int u = 0; u < 3; ++u) {
-      const int k = tid + 256 * u;
-      if (k < nq * kTile) sm.nlse[k] = -lv[u];
-    }
-#pragma unroll
     for (int gg = 0; gg < 2; ++gg) {
       const int g = warp + 8 * gg;
       if (!ngp || g >= ng) continue;   // warp-uniform
@@ -899,55 +943,12 @@ __global__ void __launch_bounds__(kColsThreads, 1)
     }
     asm volatile("bar.sync 3, 256;" ::: "memory");
 
+    // band rows: the query tiles' sums in tile order
     float acc = 0.f;
-    bool ok = active;
-    float x[128];
-    const uint64_t c2 = f2_pack(kLogitScale2, kLogitScale2);
-    for (int t = 0; ok && t <= qhiX - qloX; ++t) {
-      const int i0 = (qloX + t) * kTile;            // first query row of this tile
-      // rows i0+a .. i0+e are in j's band (and in the sequence)
-      const int a = j - p.w - i0, e = min(j + p.w, n - 1) - i0;
-      if (!(ok = warp_wait(&sm.bar_sfull[X], t & 1, abort_flag))) break;
-      tc_fence_after();
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) tmem_ld32(tST + lane_off + 32 * ch, x + 32 * ch);
-      tmem_ld_wait();
-      tc_fence_before();
-      warp_arrive(&sm.bar_sfree[X]);   // S^T is in registers: the next may overwrite it
-      // rows outside this key's band contribute nothing; tiles inside the band
-      // of all 32 keys of the warp (most of them) need no mask
-      if (!__all_sync(0xffffffffu, a <= 0 && e >= kTile - 1)) {
-#pragma unroll
-        for (int ch = 0; ch < 4; ++ch) {
-          const uint32_t keep = bit_range32(a - 32 * ch, e - 32 * ch);
-          if (__any_sync(0xffffffffu, keep != 0xffffffffu)) {
-#pragma unroll
-            for (int k = 0; k < 32; ++k) {
-              const uint32_t out =
-                  ~static_cast<uint32_t>(static_cast<int32_t>(keep << (31 - k)) >> 31);
-              x[32 * ch + k] =
-                  __uint_as_float((__float_as_uint(x[32 * ch + k]) & ~out) | (0xff800000u & out));
-            }
-          }
-        }
-      }
-      // sum over the tile's rows of exp2(S^T scaled - LSE_i)
-      const float* lw = sm.nlse + (qloX + t - qt_lo) * kTile;
-      uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
-#pragma unroll
-      for (int k = 0; k < kTile; k += 4) {
-        const float4 l4 = *reinterpret_cast<const float4*>(lw + k);
-        float e0, e1, e2, e3;
-        f2_unpack(f2_fma(f2_pack(x[k], x[k + 1]), c2, f2_pack(l4.x, l4.y)), e0, e1);
-        f2_unpack(f2_fma(f2_pack(x[k + 2], x[k + 3]), c2, f2_pack(l4.z, l4.w)), e2, e3);
-        s2a = f2_add(s2a, f2_pack(ex2(e0), ex2(e1)));
-        s2b = f2_add(s2b, f2_pack(ex2(e2), ex2(e3)));
-      }
-      float sa, sb, sc2, sd;
-      f2_unpack(s2a, sa, sb);
-      f2_unpack(s2b, sc2, sd);
-      acc += (sa + sc2) + (sb + sd);
-    }
+    for (int u = 0; u < kMaxBandTiles; ++u) acc += part[u];
+    const bool ok = active;
+    float x[16];
 
     if (active && ngp) {
       bool ok2 = ok && warp_wait(&sm.bar_sg[X], 0, abort_flag);
@@ -968,7 +969,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
       acc += s;
       // P of the global rows, transposed into this warpgroup's A tile: row g,
       // column (key) r
-      uint8_t* col = Pg + X * 2 * kTileBytes + (r >> 6) * 16384;
+      uint8_t* col = Pg + X * 2 * kPgBlock + (r >> 6) * kPgBlock;
       const int ch = (r & 63) >> 3, wi = (r & 7) * 2;
 #pragma unroll
       for (int g = 0; g < kMaxGlobal; ++g)
@@ -999,7 +1000,7 @@ __global__ void __launch_bounds__(kColsThreads, 1)
   __syncthreads();
   if (warp == 9) {
     tc_fence_after();
-    tmem_dealloc(tm, 512);
+    tmem_dealloc(tm, 256);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 

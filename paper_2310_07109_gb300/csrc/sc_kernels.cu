@@ -29,6 +29,7 @@
 // order-preserving removal) is Sec. "Sparse Attention", Sec. "Extractor of
 // Attention Scores in Sparse Attention Matrix" and Sec. "Token Pruning".
 #include <cuda_runtime.h>
+#include <utility>
 #include <cuda_bf16.h>
 #include <cstdint>
 
@@ -272,6 +273,8 @@ struct OpMax {
 
 __global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
+  pdl_launch_dependents();
+  pdl_wait();
   // grid: x = (sequence, head), y = pair of query tiles, so that low tiles (the
   // ones every sequence has) are dispatched first
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
@@ -796,6 +799,8 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
 
 __global__ void __launch_bounds__(kColsThreads, 2)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
   const LayerView v = layer_view(p);
   if (owned_by_tail(p, v, b)) return;
@@ -1202,6 +1207,8 @@ constexpr int kGatherThreads = 256;
 // 16-byte vectors, all loads issued before any store.
 __global__ void __launch_bounds__(kGatherThreads)
     sc_gather_kernel(const GatherParams g) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.y;
   int layer = g.layer;
   long long src_base = g.src_base;
@@ -1257,6 +1264,8 @@ constexpr int kPrepThreads = 1024;
 
 __global__ void __launch_bounds__(kPrepThreads)
     sc_prep_kernel(const PrepParams pp) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   __shared__ int wsum[kPrepThreads / 32];
   __shared__ int spos[kMaxLen];
@@ -1356,6 +1365,8 @@ __global__ void __launch_bounds__(kPrepThreads)
 // advance kernel: one step of the device-driven layer loop
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) sc_advance_kernel(const AdvanceParams a) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ int s_layer;
   if (threadIdx.x == 0) s_layer = __ldcg(a.dev_layer) + 1;
   __syncthreads();
@@ -1376,9 +1387,27 @@ __global__ void __launch_bounds__(256) sc_advance_kernel(const AdvanceParams a) 
 // ---------------------------------------------------------------------------
 namespace sc {
 
+// Every kernel of the chain is launched with programmatic stream serialisation:
+// it may be scheduled while its predecessor finishes and waits for it on the
+// device (pdl_wait) before touching global memory.
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_chained(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                  cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st) {
-  sc_prep_kernel<<<pp.B, kPrepThreads, 0, st>>>(pp);
-  return cudaGetLastError();
+  return launch_chained(sc_prep_kernel, dim3(pp.B), dim3(kPrepThreads), 0, st, pp);
 }
 
 cudaError_t configure_kernels() {
@@ -1399,25 +1428,21 @@ cudaError_t configure_kernels() {
 
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
   dim3 grid(p.B * p.H, (p.T + 1) / 2);
-  sc_rows_kernel<<<grid, kRowsThreads, kRowsDyn, st>>>(m, p);
-  return cudaGetLastError();
+  return launch_chained(sc_rows_kernel, grid, dim3(kRowsThreads), kRowsDyn, st, m, p);
 }
 
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
   dim3 grid(p.B * p.H, (p.T + 1) / 2);
-  sc_cols_kernel<<<grid, kColsThreads, kColsDyn, st>>>(m, p);
-  return cudaGetLastError();
+  return launch_chained(sc_cols_kernel, grid, dim3(kColsThreads), kColsDyn, st, m, p);
 }
 
 cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st) {
-  sc_advance_kernel<<<1, 256, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_chained(sc_advance_kernel, dim3(1), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {
   dim3 grid((g.L + kGatherTokens - 1) / kGatherTokens, g.B);
-  sc_gather_kernel<<<grid, kGatherThreads, 0, st>>>(g);
-  return cudaGetLastError();
+  return launch_chained(sc_gather_kernel, grid, dim3(kGatherThreads), 0, st, g);
 }
 
 }  // namespace sc

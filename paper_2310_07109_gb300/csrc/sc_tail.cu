@@ -121,6 +121,8 @@ __device__ __forceinline__ int round16(int x) { return (x + 15) & ~15; }
 
 __global__ void __launch_bounds__(kTailThreads, 1)
     sc_tail_kernel(const __grid_constant__ TailParams p) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int H = p.H, w = p.w, L = p.L, B = p.B, n_layers = p.n_layers;
   const int h = static_cast<int>(blockIdx.x) % H, b = static_cast<int>(blockIdx.x) / H;
   // every CTA of the cluster reads the same values: the exits below are uniform
@@ -615,8 +617,13 @@ cudaError_t tail_max_clusters(int H, int* out) {
 }
 
 cudaError_t launch_tail(const TailParams& p, cudaStream_t st) {
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg = tail_config(p.B, p.H, st, attr);
+  // chained like the per-layer kernels: scheduled while its predecessor
+  // finishes, waiting for it on the device
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, sc_tail_kernel, p);
 }
 

@@ -112,6 +112,19 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
 }
 
 // ---------------------------------------------------------------------------
+// Programmatic dependent launch.  Each kernel of the chain lets the next one
+// be scheduled at once (its CTAs take only free SM resources: every CTA of
+// this grid is already resident when the trigger takes effect) and, before
+// touching any global memory, waits until the preceding grid has completed
+// and its writes are visible.  Both are no-ops for a launch without the
+// programmatic attribute.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
 // TMA: gather four 128-byte rows of a 2-D tensor map (box = 64 bf16 x 1 row)
 // into 512 contiguous bytes of shared memory, completing on an mbarrier.
 // ---------------------------------------------------------------------------

@@ -13,8 +13,9 @@ Functions
 layer(Q, K, V, is_global, w, theta)          one layer, every output
 layer_sampled(Q, K, V, is_global, w, rows, cols)
                                              O rows / scores of chosen rows/cols
-stack(Q, K, V, pad_mask, global_pos, w, alpha)
+stack(Q, K, V, pad_mask, global_pos, w, alpha, keep_rule)
                                              the pruned layer stack (bf16 bits in)
+top_count(rho, n), keep_top(scores, k)       the top-ratio keep rule
 """
 from __future__ import annotations
 
@@ -64,7 +65,12 @@ def _load():
                 _ip, _ip, ctypes.c_int, _dp, _ip, ctypes.c_int, _dp]
             lib.sco_stack.restype = ctypes.c_int
             lib.sco_stack.argtypes = [ctypes.c_int] * 6 + [_u16p] * 3 + [
-                _u8p, _ip, ctypes.c_int, _dp, _dp, _dp, _ip, _ip, ctypes.c_int]
+                _u8p, _ip, ctypes.c_int, _dp, ctypes.c_int, _dp, _dp, _ip, _ip,
+                ctypes.c_int]
+            lib.sco_top_count.restype = ctypes.c_int
+            lib.sco_top_count.argtypes = [ctypes.c_double, ctypes.c_int]
+            lib.sco_keep_top.restype = ctypes.c_int
+            lib.sco_keep_top.argtypes = [ctypes.c_int, _dp, ctypes.c_int, _ip]
             _lib = lib
     return _lib
 
@@ -103,6 +109,27 @@ def layer(Q, K, V, is_global, w, theta, nthreads=None):
     return O, s[:n], keep[:n].astype(bool)
 
 
+# keep rules of the stack (the value per layer is alpha_l, theta_l or rho_l)
+KEEP_RELATIVE = 0   # theta = alpha_l / n_l
+KEEP_ABSOLUTE = 1   # theta = theta_l
+KEEP_TOP_RATIO = 2  # k = ceil(rho_l n_l) tokens: the first and the k-1 best others
+
+
+def top_count(rho, n):
+    """k = ceil(rho * n) clamped to 1..n (0 for n = 0); rho is taken as the
+    float32 value a caller of the library passes."""
+    return int(_load().sco_top_count(float(np.float32(rho)), int(n)))
+
+
+def keep_top(scores, k):
+    """keep mask of the top-ratio rule for ``k`` kept tokens (token 0 always)."""
+    s = _c(np.asarray(scores, dtype=np.float64).reshape(-1), np.float64)
+    keep = np.zeros(max(len(s), 1), np.int32)
+    if _load().sco_keep_top(len(s), s.ctypes.data_as(_dp), int(k), keep.ctypes.data_as(_ip)) < 0:
+        raise ValueError("oracle keep_top rejected its arguments")
+    return keep[:len(s)].astype(bool)
+
+
 def layer_sampled(Q, K, V, is_global, w, rows=(), cols=()):
     """O rows for ``rows`` ([len(rows), H, d]) and scores for ``cols`` ([len(cols)])."""
     Q, K, V = _c(Q, np.float64), _c(K, np.float64), _c(V, np.float64)
@@ -124,13 +151,17 @@ def layer_sampled(Q, K, V, is_global, w, rows=(), cols=()):
     return O[:len(rows)], s[:len(cols)]
 
 
-def stack(Q, K, V, pad_mask, global_pos, w, alpha, want_O=True, nthreads=None):
+def stack(Q, K, V, pad_mask, global_pos, w, alpha, want_O=True, nthreads=None,
+          keep_rule=KEEP_RELATIVE):
     """The pruned layer stack.
 
     Q, K, V: bf16 bit patterns (uint16) [n_layers, B, L, H, d], original order.
     pad_mask: uint8/bool [B, L] (1 = real token) or None.
     global_pos: sorted original positions of the global tokens.
-    alpha: [n_layers]; theta_l = alpha_l / n_l per sequence.
+    alpha: [n_layers], the keep rule's value per layer: theta_l = alpha_l / n_l
+    per sequence (KEEP_RELATIVE), theta_l = alpha_l (KEEP_ABSOLUTE), or the
+    kept ratio rho_l = alpha_l (KEEP_TOP_RATIO; taken as float32, as the
+    library receives it).
     Returns dict with O ([nl,B,L,H,d] float64 or None), scores ([nl,B,L]),
     pos ([nl+1,B,L] int32), len ([nl+1,B] int32).  Slots at or past the
     current length hold -1 (pos) / NaN (scores, O).
@@ -140,6 +171,8 @@ def stack(Q, K, V, pad_mask, global_pos, w, alpha, want_O=True, nthreads=None):
     assert K.shape == Q.shape and V.shape == Q.shape
     alpha = _c(np.asarray(alpha, dtype=np.float64).reshape(-1), np.float64)
     assert alpha.shape[0] == nl
+    if keep_rule == KEEP_TOP_RATIO:
+        alpha = alpha.astype(np.float32).astype(np.float64)
     gp = _c(np.asarray(global_pos, dtype=np.int32).reshape(-1), np.int32)
     mask = None if pad_mask is None else _c(np.asarray(pad_mask).astype(np.uint8), np.uint8)
     O = np.full((nl, B, L, H, d), np.nan) if want_O else None
@@ -151,7 +184,7 @@ def stack(Q, K, V, pad_mask, global_pos, w, alpha, want_O=True, nthreads=None):
                       K.ctypes.data_as(_u16p), V.ctypes.data_as(_u16p),
                       None if mask is None else mask.ctypes.data_as(_u8p),
                       gp.ctypes.data_as(_ip), len(gp), alpha.ctypes.data_as(_dp),
-                      None if O is None else O.ctypes.data_as(_dp),
+                      int(keep_rule), None if O is None else O.ctypes.data_as(_dp),
                       scores.ctypes.data_as(_dp), pos.ctypes.data_as(_ip),
                       lens.ctypes.data_as(_ip), int(nthreads or default_threads()))
     if r < 0:

@@ -26,6 +26,12 @@
  *   5. Binarised keep mask (Sec. "Token Pruning", Step 2): token j is kept when
  *      s_j >= theta; the first current token (the CLS token) is always kept.
  *      Kept tokens are removed/compacted in order (Step 3, hard pruning).
+ *      Two alternatives to the per-layer threshold alpha_l / n_l, both from the
+ *      paper: an absolute threshold theta_l per layer (Sec. "RQ4": the
+ *      thresholds of the layers are scaled linearly up to the last one), and
+ *      the "top-k of the sequence length" family of Sec. "Pruning": a layer
+ *      keeps k = ceil(rho_l n) tokens (clamped to 1..n), the first token and
+ *      the k-1 others with the largest scores, ties going to the lower index.
  *
  * Everything is double precision and loops over the definition directly; no
  * blocking, no online softmax, no reordering.  The stack driver reads the
@@ -182,6 +188,42 @@ SCO_EXPORT int sco_layer(int n, int H, int d, int w, const double *Q,
     return kept;
 }
 
+/* ------------------------------------------------------------------------ */
+/* top-ratio keep rule (Sec. "Pruning", second family)                      */
+/* ------------------------------------------------------------------------ */
+/* k = ceil(rho * n), clamped to 1..n.  rho * n is exact in double for a rho
+ * that came from a float and n < 2^24. */
+SCO_EXPORT int sco_top_count(double rho, int n)
+{
+    if (n <= 0) return 0;
+    double c = ceil(rho * (double)n);
+    if (!(c >= 1.0)) return 1;   /* also a NaN ratio */
+    if (c >= (double)n) return n;
+    return (int)c;
+}
+
+/*
+ * keep[j] for the top-ratio rule: token 0, and each other token whose rank
+ * among tokens 1..n-1 (larger score first, ties by lower index) is below k-1.
+ * The rank is counted directly: the number of other tokens that come first.
+ * Returns the number kept (k), or -1 on bad arguments.
+ */
+SCO_EXPORT int sco_keep_top(int n, const double *scores, int k, int *keep)
+{
+    if (n < 0 || k < 0) return -1;
+    if (n == 0) return 0;
+    if (k < 1) k = 1;
+    if (k > n) k = n;
+    keep[0] = 1;
+    for (int j = 1; j < n; ++j) {
+        int rank = 0;
+        for (int i = 1; i < n; ++i)
+            if (scores[i] > scores[j] || (scores[i] == scores[j] && i < j)) ++rank;
+        keep[j] = rank < k - 1;
+    }
+    return k;
+}
+
 /*
  * Sampled evaluation of one layer, for sizes where the full layer is too slow:
  * O rows of the listed query rows, and s_j of the listed key columns, each
@@ -284,7 +326,10 @@ static int is_global_position(const int *g, int ng, int p)
  *             before the first layer (Fig. "experiment" caption: inputs are
  *             padded to max_length; padding carries no content).
  * gpos, ngpos global original positions.
- * alpha       [n_layers]: theta_l = alpha_l / n_l for each sequence.
+ * alpha       [n_layers]: the keep rule's value per layer.
+ * rule        0: theta_l = alpha_l / n_l for each sequence;
+ *             1: theta_l = alpha_l (absolute);
+ *             2: top ratio rho_l = alpha_l (see sco_keep_top).
  * O           [n_layers][B][L][H][d] doubles at current slots, or NULL.
  * scores      [n_layers][B][L] doubles at current slots.
  * pos         [n_layers+1][B][L] original positions of the current tokens.
@@ -295,10 +340,11 @@ SCO_EXPORT int sco_stack(int n_layers, int B, int L, int H, int d, int w,
                          const uint16_t *Qb, const uint16_t *Kb,
                          const uint16_t *Vb, const uint8_t *pad_mask,
                          const int *gpos, int ngpos, const double *alpha,
-                         double *O, double *scores, int *pos, int *len,
-                         int nthreads)
+                         int rule, double *O, double *scores, int *pos,
+                         int *len, int nthreads)
 {
     if (n_layers < 1 || B < 1 || L < 1 || H < 1 || d < 1 || w < 0) return -1;
+    if (rule < 0 || rule > 2) return -1;
     const size_t row = (size_t)H * d;
     double *q = (double *)malloc(sizeof(double) * (size_t)L * row);
     double *k = (double *)malloc(sizeof(double) * (size_t)L * row);
@@ -330,8 +376,9 @@ SCO_EXPORT int sco_stack(int n_layers, int B, int L, int H, int d, int w,
                 }
                 isg[c] = is_global_position(gpos, ngpos, pl[c]);
             }
-            double theta = n > 0 ? alpha[l] / (double)n : 0.0;
+            double theta = rule == 1 ? alpha[l] : (n > 0 ? alpha[l] / (double)n : 0.0);
             sco_layer(n, H, d, w, q, k, v, isg, theta, o, s, keep, nthreads);
+            if (rule == 2) sco_keep_top(n, s, sco_top_count(alpha[l], n), keep);
             int m = 0;
             for (int c = 0; c < n; ++c) {
                 scores[base * L + c] = s[c];

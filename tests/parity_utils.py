@@ -29,24 +29,46 @@ def near_threshold(scores, n, theta):
     return [int(j) for j in bad if j != 0]
 
 
+def near_cut(scores, n, k):
+    """Top-ratio rule: current indices j >= 1 whose oracle score lies within
+    MARGIN / n of the midpoint between the lowest kept and the highest dropped
+    score (token 0 is kept regardless and takes no part in the ranking)."""
+    s = np.asarray(scores[1:n])
+    if k - 1 <= 0 or k - 1 >= len(s):
+        return []
+    srt = np.sort(s)[::-1]
+    cut = 0.5 * (srt[k - 2] + srt[k - 1])
+    return [int(j) + 1 for j in np.nonzero(np.abs(s - cut) < MARGIN / n)[0]]
+
+
+def near_boundary(wl, scores, n, value):
+    """Tokens of one (layer, sequence) too close to the keep decision of ``wl``'s rule."""
+    if wl.keep_rule == oracle.KEEP_TOP_RATIO:
+        return near_cut(scores, n, oracle.top_count(value, n))
+    theta = value if wl.keep_rule == oracle.KEEP_ABSOLUTE else value / n
+    return near_threshold(scores, n, theta)
+
+
 def resample_stack(wl: wk.Workload, max_rounds: int = 50, nthreads=None, overrides=None):
     """Draw ``wl`` and redraw (layer, token) Q/K rows until no oracle score of any
-    layer lies within MARGIN / n of its threshold.  Layers interact only through
-    the kept set, so fixing the first offending layer and re-running converges.
-    ``overrides`` replaces entries of the drawn inputs (e.g. global_pos, pad_mask)."""
+    layer lies within MARGIN / n of its keep decision (the threshold, or the cut
+    between kept and dropped scores of the top-ratio rule).  Layers interact
+    only through the kept set, so fixing the first offending layer and
+    re-running converges.  ``overrides`` replaces entries of the drawn inputs
+    (e.g. global_pos, pad_mask)."""
     redraws = {}
     for _ in range(max_rounds):
         inp = wk.make_inputs(wl, redraws)
         inp.update(overrides or {})
         res = oracle.stack(inp["Q"], inp["K"], inp["V"], inp["pad_mask"], inp["global_pos"],
-                           wl.w, inp["alpha"], nthreads=nthreads)
+                           wl.w, inp["alpha"], nthreads=nthreads, keep_rule=wl.keep_rule)
         bad = []
         for l in range(wl.n_layers):
             for b in range(wl.B):
                 n = int(res["len"][l, b])
                 if n == 0:
                     continue
-                for j in near_threshold(res["scores"][l, b], n, inp["alpha"][l] / n):
+                for j in near_boundary(wl, res["scores"][l, b], n, inp["alpha"][l]):
                     bad.append((l, b, int(res["pos"][l, b, j])))
             if bad:
                 break

@@ -298,3 +298,115 @@ def test_generator_is_deterministic_and_redraw_is_local():
     diff = np.argwhere((a["Q"] != c["Q"]).any(axis=(3, 4)))
     assert diff.tolist() == [[1, 0, 7]]
     assert (a["V"] == c["V"]).all()
+
+
+# --------------------------------------------------------------------------
+# the other keep rules: an absolute threshold per layer (RQ4's schedule) and
+# a kept ratio per layer (the "top-k of the sequence length" family of the
+# Pruning section)
+# --------------------------------------------------------------------------
+def test_top_count_closed_forms():
+    assert oracle.top_count(1.0, 37) == 37
+    assert oracle.top_count(0.0, 37) == 1
+    assert oracle.top_count(0.5, 7) == 4
+    assert oracle.top_count(0.5, 8) == 4
+    assert oracle.top_count(2.0, 5) == 5
+    assert oracle.top_count(0.25, 0) == 0
+    # the ratio is the float32 a library caller passes: float32(0.3) is a
+    # little above 0.3, so 10 tokens keep 4
+    assert float(np.float32(0.3)) > 0.3
+    assert oracle.top_count(0.3, 10) == 4
+
+
+@pytest.mark.parametrize("n,k,seed", [(1, 1, 0), (2, 1, 1), (2, 2, 2), (50, 1, 3),
+                                      (50, 17, 4), (50, 50, 5), (300, 123, 6)])
+def test_keep_top_matches_stable_sort(n, k, seed):
+    rng = np.random.default_rng(seed)
+    s = rng.random(n)
+    if n > 10:
+        s[5:9] = s[20 % n]          # ties, resolved by the lower index
+    keep = oracle.keep_top(s, k)
+    order = 1 + np.argsort(-s[1:], kind="stable")   # numpy's stable sort
+    expect = np.zeros(n, bool)
+    expect[0] = True
+    expect[order[:k - 1]] = True
+    np.testing.assert_array_equal(keep, expect)
+    assert keep.sum() == k
+
+
+def test_keep_top_ignores_token0_score():
+    s = np.array([0.0, 0.3, 0.1, 0.3, 0.2])
+    assert list(np.nonzero(oracle.keep_top(s, 3))[0]) == [0, 1, 3]
+    s[0] = 9.0   # a large first score takes no other token's place
+    assert list(np.nonzero(oracle.keep_top(s, 3))[0]) == [0, 1, 3]
+
+
+def test_uniform_attention_keeps_the_first_k():
+    # zero queries with a window covering the sequence: every probability is
+    # 1/n, every score the same, so the ties keep the lowest indices
+    n, H, d = 40, 3, 8
+    rng = np.random.default_rng(2)
+    Q = np.zeros((n, H, d))
+    K = rng.standard_normal((n, H, d))
+    V = rng.standard_normal((n, H, d))
+    _, s, _ = oracle.layer(Q, K, V, _globals_mask(n, [0]), n, 0.0)
+    assert (s == s[0]).all()
+    k = oracle.top_count(0.3, n)
+    assert list(np.nonzero(oracle.keep_top(s, k))[0]) == list(range(k))
+
+
+def test_stack_top_ratio_lengths_and_sets():
+    wl, inp = _small_stack(ragged=(40, 96), extra=2, nl=5)
+    rho = np.array([0.9, 0.75, 0.6, 0.5, 0.35])
+    res = oracle.stack(inp["Q"], inp["K"], inp["V"], inp["pad_mask"], inp["global_pos"],
+                       wl.w, rho, keep_rule=oracle.KEEP_TOP_RATIO)
+    for b in range(wl.B):
+        for l in range(wl.n_layers):
+            n = int(res["len"][l, b])
+            k = int(np.ceil(float(np.float32(rho[l])) * n))   # closed form of the chain
+            assert res["len"][l + 1, b] == min(max(k, 1), n)
+            s = res["scores"][l, b, :n]
+            keep = oracle.keep_top(s, k)
+            cur = res["pos"][l, b, :n]
+            assert list(res["pos"][l + 1, b, :res["len"][l + 1, b]]) == list(cur[keep])
+
+
+def test_stack_absolute_threshold():
+    wl, inp = _small_stack(L=128, nl=4)
+    theta = np.array([0.002, 0.004, 0.006, 0.008])
+    res = oracle.stack(inp["Q"], inp["K"], inp["V"], None, inp["global_pos"], wl.w, theta,
+                       keep_rule=oracle.KEEP_ABSOLUTE)
+    for b in range(wl.B):
+        for l in range(wl.n_layers):
+            n0, n1 = res["len"][l, b], res["len"][l + 1, b]
+            s = res["scores"][l, b, :n0]
+            cur = res["pos"][l, b, :n0]
+            assert list(res["pos"][l + 1, b, :n1]) == [
+                p for c, p in enumerate(cur) if c == 0 or s[c] >= theta[l]]
+    # one layer without padding: theta = alpha / L is the relative rule
+    one = {k: inp[k][:1] for k in ("Q", "K", "V")}
+    a = oracle.stack(one["Q"], one["K"], one["V"], None, inp["global_pos"], wl.w, [0.8])
+    t = oracle.stack(one["Q"], one["K"], one["V"], None, inp["global_pos"], wl.w, [0.8 / wl.L],
+                     keep_rule=oracle.KEEP_ABSOLUTE)
+    for key in ("pos", "len"):
+        np.testing.assert_array_equal(a[key], t[key])
+
+
+@pytest.mark.parametrize("rule,values", [(oracle.KEEP_TOP_RATIO, (0.9, 0.6)),
+                                         (oracle.KEEP_ABSOLUTE, (0.004, 0.012))])
+def test_resampling_clears_the_keep_decision(rule, values):
+    from parity_utils import MARGIN, resample_stack
+    wl = wk.Workload("t", n_layers=3, B=2, L=160, H=2, w=12, alpha_first=values[0],
+                     alpha_last=values[1], keep_rule=rule, seed=21)
+    inp, res, _ = resample_stack(wl)
+    for l in range(wl.n_layers):
+        for b in range(wl.B):
+            n = int(res["len"][l, b])
+            s = res["scores"][l, b, 1:n]
+            kept = res["len"][l + 1, b] - 1
+            if rule == oracle.KEEP_TOP_RATIO:
+                srt = np.sort(s)[::-1]
+                if 0 < kept < len(s):
+                    assert srt[kept - 1] - srt[kept] >= 2 * MARGIN / n
+            else:
+                assert (np.abs(s - inp["alpha"][l]) >= MARGIN / n).all()

@@ -57,9 +57,11 @@ def _rng(*key: int) -> np.random.Generator:
 class Workload:
     """One synthetic workload.
 
-    alpha schedule: theta_l = alpha_l / n_l, alpha linear from ``alpha_first``
-    (layer 1) to ``alpha_last`` (layer n_layers), endpoints included; the paper
-    scales its per-layer thresholds linearly with depth (RQ4 discussion).
+    alpha schedule: linear from ``alpha_first`` (layer 1) to ``alpha_last``
+    (layer n_layers), endpoints included; the paper scales its per-layer
+    thresholds linearly with depth (RQ4 discussion).  ``keep_rule`` says what
+    the per-layer value is: 0 = alpha_l with theta_l = alpha_l / n_l, 1 = an
+    absolute threshold theta_l, 2 = the ratio of tokens a layer keeps.
     """
     name: str
     n_layers: int
@@ -75,6 +77,7 @@ class Workload:
     alpha_last: float = 0.9
     ragged: Optional[Tuple[int, int]] = None
     seed: int = 1
+    keep_rule: int = 0
 
     def alphas(self) -> np.ndarray:
         if self.n_layers == 1:
@@ -89,7 +92,8 @@ class Workload:
         s = (f"{self.name}: {self.n_layers} layers, B={self.B}, L={self.L}, H={self.H}, "
              f"d={self.d}, window +-{self.w}, globals 1+{self.n_extra_global}, "
              f"salient {self.salient_frac:.0%} x{self.salient_scale:g}, "
-             f"alpha {self.alpha_first:g}->{self.alpha_last:g}")
+             + ("alpha", "theta", "kept ratio")[self.keep_rule]
+             + f" {self.alpha_first:g}->{self.alpha_last:g}")
         if self.ragged:
             s += f", true lengths U[{self.ragged[0]},{self.ragged[1]}]"
         return s + f", seed {self.seed}"
@@ -115,6 +119,27 @@ def cfg5(L: int, control: bool = False) -> Workload:
 
 
 CONFIGS = {"cfg1": CFG1, "cfg2": CFG2, "cfg3": CFG3, "cfg4": CFG4}
+
+
+def window_sweep(w: int) -> Workload:
+    """The window-size ablation (Table "window_size", RQ3): sparse attention
+    alone (nothing pruned) over inputs of maximum length 1024, one-sided window
+    ``w`` in {16, 32, 64, 128, 256, 512}; 12 layers, B = 8."""
+    assert w in (16, 32, 64, 128, 256, 512)
+    return Workload(f"window_w{w}_L1024_B8", n_layers=12, B=8, L=1024, w=w,
+                    alpha_first=0.0, alpha_last=0.0)
+
+
+# The paper's own threshold schedule (RQ4): absolute thresholds scaled
+# linearly with depth up to 0.01 at the 12th layer (0.01 l / 12), over the
+# config-2 shape.
+ABS_THETA = Workload("abs_theta_L1024_B8", n_layers=12, B=8, L=1024,
+                     alpha_first=0.01 / 12, alpha_last=0.01, keep_rule=1)
+
+# The top-k family of Sec. "Pruning": each layer keeps a fixed ratio of its
+# current tokens (0.95 at layer 1 down to 0.8 at layer 12), config-2 shape.
+TOP_RATIO = Workload("top_ratio_L1024_B8", n_layers=12, B=8, L=1024,
+                     alpha_first=0.95, alpha_last=0.8, keep_rule=2)
 
 
 def global_positions(wl: Workload) -> np.ndarray:

@@ -36,6 +36,12 @@
  *   keep_j = (j == 0) || s_j >= theta  (Sec. "Token Pruning", Step 2, the
  *   binarised mask, read as >= and with the first token always kept);
  *   kept tokens are compacted in order (Step 3, hard pruning).
+ *   Keep rules (sc_keep_rule): theta = alpha / n per sequence (default),
+ *   an absolute theta (the schedule of Sec. "RQ4": thresholds scaled linearly
+ *   with depth), or the "top-k of the sequence length" family of Sec.
+ *   "Pruning": a layer keeps k = ceil(rho n) tokens, clamped to 1..n, the
+ *   first token and the k-1 others with the largest s_j, ties to the lower
+ *   current index.
  */
 #ifndef SPARSECODER_H
 #define SPARSECODER_H
@@ -62,6 +68,14 @@ typedef enum {
   SC_ERR_WORKSPACE = 5    /* workspace missing, too small or misaligned */
 } sc_status;
 
+/* What decides that a token survives a layer (the value `alpha` of a layer). */
+typedef enum {
+  SC_KEEP_RELATIVE = 0,  /* s_j >= alpha / n (theta = alpha / n per sequence) */
+  SC_KEEP_ABSOLUTE = 1,  /* s_j >= alpha (an absolute threshold) */
+  SC_KEEP_TOP_RATIO = 2  /* the ceil(alpha n) best tokens (alpha = kept ratio; k is
+                            computed in double from the float alpha, so exactly) */
+} sc_keep_rule;
+
 /*
  * One layer on tokens already in current (compacted) order.
  *
@@ -74,15 +88,19 @@ typedef enum {
  * w          one-sided window (>= 0).
  * global_pos HOST int32 [n_global]: sorted, distinct original positions,
  *            0 <= g < L, n_global <= SC_MAX_GLOBAL (may be 0).
- * alpha      theta_b = alpha / n_b for every sequence (threshold schedule of
- *            Sec. "RQ4": thresholds scaled linearly across layers; the caller
- *            supplies alpha for this layer).  Ignored when theta != NULL.
- * theta      optional float [B]: absolute thresholds per sequence.
+ * alpha      the keep rule's value: theta_b = alpha / n_b (SC_KEEP_RELATIVE;
+ *            the threshold schedule of Sec. "RQ4" scales it linearly across
+ *            layers, the caller supplies this layer's), theta_b = alpha
+ *            (SC_KEEP_ABSOLUTE), or the kept ratio (SC_KEEP_TOP_RATIO; finite).
+ *            Ignored when theta != NULL.
+ * theta      optional float [B]: absolute thresholds per sequence (threshold
+ *            rules only; must be NULL under SC_KEEP_TOP_RATIO).
  * O          bf16 [B][L][H][64] out: attention output of every current token
  *            (all n_b tokens, before pruning) at its current slot.
  * scores     float [B][L] out: s_j at current slot j.
  * pos_out    int32 [B][L] out: original positions of the kept tokens, in order.
  * len_out    int32 [B] out: number of kept tokens.
+ * keep_rule  an sc_keep_rule (0 = SC_KEEP_RELATIVE).
  * Slots at or beyond the current (resp. kept) length are left untouched.
  * pos_out/len_out must not alias pos/len.
  */
@@ -101,6 +119,7 @@ typedef struct {
   float* scores;
   int32_t* pos_out;
   int32_t* len_out;
+  int keep_rule;
 } sc_layer_args;
 
 /*
@@ -112,7 +131,10 @@ typedef struct {
  *            tokens are removed before layer 0 (Fig. "experiment" caption:
  *            shorter inputs are padded to max_length).
  * w, global_pos, n_global   as for sc_layer_args.
- * alpha      HOST float [n_layers]: theta_{l,b} = alpha[l] / n_{l,b}.
+ * alpha      HOST float [n_layers]: the keep rule's value per layer:
+ *            theta_{l,b} = alpha[l] / n_{l,b} (SC_KEEP_RELATIVE), theta_l =
+ *            alpha[l] (SC_KEEP_ABSOLUTE) or the kept ratio rho_l
+ *            (SC_KEEP_TOP_RATIO; finite).
  * O          bf16 [n_layers][B][L][H][64] out (current slots of each layer).
  * scores     float [n_layers][B][L] out.
  * pos        int32 [n_layers+1][B][L] out: pos[0] = real tokens after padding
@@ -120,6 +142,7 @@ typedef struct {
  * len        int32 [n_layers+1][B] out.
  * flags      0, or SC_STACK_NO_TAIL: run every layer of every sequence through
  *            the per-layer kernels (see sc_stack_forward).
+ * keep_rule  an sc_keep_rule (0 = SC_KEEP_RELATIVE), the same for every layer.
  */
 #define SC_STACK_NO_TAIL 1
 
@@ -137,6 +160,7 @@ typedef struct {
   int32_t* pos;
   int32_t* len;
   int flags;
+  int keep_rule;
 } sc_stack_args;
 
 /*

@@ -38,7 +38,8 @@ class LayerArgs(ctypes.Structure):
                 ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
                 ("alpha", ctypes.c_float), ("theta", ctypes.c_void_p),
                 ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
-                ("pos_out", ctypes.c_void_p), ("len_out", ctypes.c_void_p)]
+                ("pos_out", ctypes.c_void_p), ("len_out", ctypes.c_void_p),
+                ("keep_rule", ctypes.c_int)]
 
 
 class StackArgs(ctypes.Structure):
@@ -49,10 +50,15 @@ class StackArgs(ctypes.Structure):
                 ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
                 ("alpha", ctypes.POINTER(ctypes.c_float)),
                 ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
-                ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p), ("flags", ctypes.c_int)]
+                ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p), ("flags", ctypes.c_int),
+                ("keep_rule", ctypes.c_int)]
 
 
 SC_STACK_NO_TAIL = 1
+# keep rules (sc_keep_rule): what a layer's value alpha means
+SC_KEEP_RELATIVE = 0   # theta = alpha / n
+SC_KEEP_ABSOLUTE = 1   # theta = alpha
+SC_KEEP_TOP_RATIO = 2  # keep ceil(alpha n) tokens: the first and the best others
 # sequences with at most this many current tokens finish in the cluster kernel
 # (SC_TAIL_MAX_LEN of include/sparsecoder.h)
 TAIL_MAX_LEN = 384
@@ -148,10 +154,12 @@ def _int32_host(values):
 
 
 def layer_forward(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *, O=None,
-                  scores=None, pos_out=None, len_out=None, workspace=None, stream=None):
+                  scores=None, pos_out=None, len_out=None, workspace=None, stream=None,
+                  keep_rule=SC_KEEP_RELATIVE):
     """One layer on current-order inputs (``sc_layer_forward``).
 
     Q, K, V: bf16 [B, L, H, 64] cuda tensors; length: int32 [B]; pos: int32 [B, L].
+    keep_rule: an SC_KEEP_* value saying what ``alpha`` is.
     Returns (O, scores, pos_out, len_out).
     """
     B, L, H, D = Q.shape
@@ -164,30 +172,33 @@ def layer_forward(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *,
     garr, ng = _int32_host(global_pos)
     a = LayerArgs(B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(length), _ptr(pos),
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, float(alpha),
-                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out))
+                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out),
+                  int(keep_rule))
     _check(load().sc_layer_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
     return O, scores, pos_out, len_out
 
 
 def layer_forward_noalloc(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=None, *, O,
-                          scores, pos_out, len_out, stream=None):
+                          scores, pos_out, len_out, stream=None, keep_rule=SC_KEEP_RELATIVE):
     """One layer through ``sc_layer_forward_noalloc``: no device memory is
     allocated, by this call or the library; every output tensor is passed in."""
     B, L, H, D = Q.shape
     garr, ng = _int32_host(global_pos)
     a = LayerArgs(B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(length), _ptr(pos),
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, float(alpha),
-                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out))
+                  _ptr(theta), _ptr(O), _ptr(scores), _ptr(pos_out), _ptr(len_out),
+                  int(keep_rule))
     _check(load().sc_layer_forward_noalloc(ctypes.byref(a), _stream_handle(stream)))
     return O, scores, pos_out, len_out
 
 
 def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
-                  stream=None, events=None, no_tail=False):
+                  stream=None, events=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE):
     """The pruned layer stack (``sc_stack_forward``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
-    pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers].
+    pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers],
+    the value of the keep rule ``keep_rule`` (an SC_KEEP_* value) per layer.
     events: optional list of >= 3 + 3 * n_layers torch.cuda.Event(enable_timing=True),
     recorded around every kernel on the launching stream (sc_stack_forward_profiled).
     no_tail: run every layer through the per-layer kernels (SC_STACK_NO_TAIL).
@@ -207,7 +218,7 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
                   _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
-                  SC_STACK_NO_TAIL if no_tail else 0)
+                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule))
     if events is None:
         _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
                                        _stream_handle(stream)))

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <cmath>
 #include <cstdint>
 #include <cstdio>
 #include <cstring>
@@ -235,6 +236,19 @@ int check_common(int B, int L, int H, int w, const int32_t* gpos, int ngl) {
   return SC_OK;
 }
 
+// The keep rule and its per-layer values (one value for a layer call): the
+// top-ratio rule takes no per-sequence thresholds and needs finite ratios.
+int check_keep(int rule, const float* values, int count, const float* theta) {
+  if (rule != SC_KEEP_RELATIVE && rule != SC_KEEP_ABSOLUTE && rule != SC_KEEP_TOP_RATIO)
+    return fail(SC_ERR_INVALID_ARG, "keep_rule", "not an sc_keep_rule");
+  if (rule == SC_KEEP_TOP_RATIO) {
+    if (theta) return fail(SC_ERR_INVALID_ARG, "theta", "the top-ratio rule takes no thresholds");
+    for (int l = 0; l < count; ++l)
+      if (!std::isfinite(values[l])) return fail(SC_ERR_INVALID_ARG, "alpha", "ratio not finite");
+  }
+  return SC_OK;
+}
+
 void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->status = reinterpret_cast<int*>(ws + lay.status);
   p->acc = reinterpret_cast<float*>(ws + lay.acc);
@@ -304,6 +318,7 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
     return SC_ERR_INVALID_ARG;
   if (a->pos_out == a->pos || a->len_out == a->len) return SC_ERR_INVALID_ARG;
+  if ((rc = check_keep(a->keep_rule, &a->alpha, 1, a->theta)) != SC_OK) return rc;
   WsLayout lay;
   ws_layout(a->B, a->L, a->H, &lay);
   if (!workspace || ws_bytes < lay.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
@@ -332,6 +347,7 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   p.len_out = a->len_out;
   p.alpha = a->alpha;
   p.theta = a->theta;
+  p.keep_rule = a->keep_rule;
   fill_workspace(&p, ws, lay, 0);
 
   PrepParams pp{};
@@ -373,6 +389,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   if (rc != SC_OK) return rc;
   if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
     return SC_ERR_INVALID_ARG;
+  if ((rc = check_keep(a->keep_rule, a->alpha, a->n_layers, nullptr)) != SC_OK) return rc;
   if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
     return SC_ERR_INVALID_ARG;
   const long long rows = static_cast<long long>(a->n_layers) * a->B * a->L * a->H;
@@ -402,6 +419,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   p.B = a->B; p.L = a->L; p.H = a->H; p.w = a->w;
   p.T = (a->L + kTile - 1) / kTile;
   p.theta = nullptr;
+  p.keep_rule = a->keep_rule;
   p.tail_from = tail_from;
   p.tail_max = use_tail ? kTailMax : 0;
   fill_workspace(&p, ws, lay, 0);
@@ -594,6 +612,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     tp.n_global = a->n_global;
     for (int g = 0; g < a->n_global; ++g) tp.global_pos[g] = a->global_pos[g];
     for (int l = 0; l < a->n_layers; ++l) tp.alpha[l] = a->alpha[l];
+    tp.keep_rule = a->keep_rule;
     if ((e = launch_tail(tp, st)) != cudaSuccess) return fail_cuda("launch tail kernel", e);
   }
   if (!mark(2 + 3 * a->n_layers)) return fail(SC_ERR_CUDA, "event record", "");
@@ -694,6 +713,7 @@ extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
   if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
     return SC_ERR_INVALID_ARG;
   if (a->pos_out == a->pos || a->len_out == a->len) return SC_ERR_INVALID_ARG;
+  if ((rc = check_keep(a->keep_rule, &a->alpha, 1, a->theta)) != SC_OK) return rc;
   // a single layer reads its rows in place, so the compacted copies that the
   // layout reserves last are not needed: everything before them must fit
   WsLayout lay;
@@ -734,6 +754,7 @@ extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
   p.len_out = a->len_out;
   p.alpha = a->alpha;
   p.theta = a->theta;
+  p.keep_rule = a->keep_rule;
   fill_workspace(&p, ws, lay, 0);
 
   PrepParams pp{};

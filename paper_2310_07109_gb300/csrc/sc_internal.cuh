@@ -29,6 +29,11 @@ constexpr int kTailMaxLayers = 64;
 constexpr int kTailMaxHeads = 16;   // largest (non-portable) cluster
 
 // log2(e) / sqrt(64): logits are kept in base-2 units, x = (q.k) * kLogitScale2.
+// keep rules (the SC_KEEP_* values of the C interface)
+constexpr int kKeepRelative = SC_KEEP_RELATIVE;
+constexpr int kKeepAbsolute = SC_KEEP_ABSOLUTE;
+constexpr int kKeepTopRatio = SC_KEEP_TOP_RATIO;
+
 constexpr float kLogitScale2 = 0.125f * 1.4426950408889634f;
 
 // TMA descriptors of Q, K, V (index 0, 1, 2) for both row sources: [0] the
@@ -59,8 +64,9 @@ struct LayerParams {
   int32_t* gcur_out;     // [B][kMaxGlobal] out (next layer)
   int32_t* ng_out;       // [B] out
   int32_t* ident_out;    // [B] out (next layer)
-  float alpha;           // theta_b = alpha / n_b unless theta != nullptr
-  const float* theta;    // [B] absolute thresholds or nullptr
+  float alpha;           // the keep rule's value (alpha, theta or kept ratio)
+  const float* theta;    // [B] absolute thresholds or nullptr (threshold rules)
+  int keep_rule;         // kKeepRelative, kKeepAbsolute or kKeepTopRatio
   // workspace
   float* acc;            // [B][H][L] per-head column sums: band rows + global rows
   float* colpart;        // [B][H][L][kMaxBandTiles] band-row column sums per query tile
@@ -172,7 +178,8 @@ struct TailParams {
   const uint16_t* src[3];      // Q, K, V [n_layers][B][L][H][64]
   int n_global;
   int global_pos[kMaxGlobal];
-  float alpha[kTailMaxLayers];
+  float alpha[kTailMaxLayers];   // the keep rule's value per layer
+  int keep_rule;
 };
 
 }  // namespace sc

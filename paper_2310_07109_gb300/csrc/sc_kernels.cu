@@ -34,6 +34,7 @@
 #include <cstdint>
 
 #include "sc_internal.cuh"
+#include "sc_select.cuh"
 #include "sm103_primitives.cuh"
 
 namespace sc {
@@ -795,7 +796,7 @@ static_assert(3 * kPgBlock + kTileBytes <= 4 * kPgBlock + 4 * kTileBytes,
               "the A operand's unused rows stay inside the shared memory");
 
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
-                                  ColsSmem& sm);
+                                  ColsSmem& sm, uint8_t* scratch);
 
 __global__ void __launch_bounds__(kColsThreads, 2)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
@@ -1079,8 +1080,12 @@ __global__ void __launch_bounds__(kColsThreads, 2)
       if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
     v.scores[static_cast<size_t>(b) * p.L + jj] = s;
-    const float theta = p.theta ? __ldg(p.theta + b) : v.alpha / static_cast<float>(n);
-    p.keep[static_cast<size_t>(b) * p.L + jj] = (jj == 0 || s >= theta) ? 1 : 0;
+    if (p.keep_rule != kKeepTopRatio) {   // the top-ratio cut needs every score first
+      const float theta = p.theta ? __ldg(p.theta + b)
+                          : p.keep_rule == kKeepAbsolute ? v.alpha
+                                                         : v.alpha / static_cast<float>(n);
+      p.keep[static_cast<size_t>(b) * p.L + jj] = (jj == 0 || s >= theta) ? 1 : 0;
+    }
   }
   if (tid == 0) p.cnt_tile[b * p.T + pr] = 0u;
   __threadfence();
@@ -1089,16 +1094,22 @@ __global__ void __launch_bounds__(kColsThreads, 2)
   __syncthreads();
   if (!sm.flag) return;
   __threadfence();
-  finalize_sequence(p, v, b, n, sm);
+  finalize_sequence(p, v, b, n, sm, base);
 }
+
+struct BlockSync {
+  __device__ __forceinline__ void operator()() const { __syncthreads(); }
+};
 
 // Order-preserving compaction of sequence b's kept tokens, the next layer's
 // global list, and the bf16 outputs of the global rows.  One CTA; token c is
 // handled by thread c % kColsThreads in round c / kColsThreads (coalesced
 // loads, all issued at once); output slots come from warp ballots and a
-// fixed-order prefix over (round, warp).
+// fixed-order prefix over (round, warp).  Under the top-ratio rule the keep
+// flags come from the cut over all n scores, found here (`scratch`: shared
+// memory the CTA no longer uses, for the selection's histogram and tie flags).
 __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int b, int n,
-                                  ColsSmem& sm) {
+                                  ColsSmem& sm, uint8_t* scratch) {
   constexpr int kRounds = (kMaxLen + kColsThreads - 1) / kColsThreads;
   constexpr int kWarps = kColsThreads / 32;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -1107,11 +1118,35 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
   int32_t* pos_out = v.pos_out + static_cast<size_t>(b) * p.L;
   bool kf[kRounds];
   int32_t ps[kRounds];
+  if (p.keep_rule == kKeepTopRatio) {
+    const float* sc = v.scores + static_cast<size_t>(b) * p.L;
+    uint32_t key[kRounds];
 #pragma unroll
-  for (int r = 0; r < kRounds; ++r) {
-    const int c = r * kColsThreads + tid;
-    kf[r] = c < n && __ldcg(keep + c) != 0;
-    ps[r] = c < n ? __ldcg(pos + c) : 0;
+    for (int r = 0; r < kRounds; ++r) {
+      const int c = r * kColsThreads + tid;
+      key[r] = (c >= 1 && c < n) ? select_key(__ldcg(sc + c)) : 0u;
+      ps[r] = c < n ? __ldcg(pos + c) : 0;
+    }
+    SelectSmem& ss = *reinterpret_cast<SelectSmem*>(scratch);
+    uint8_t* tie = scratch + sizeof(SelectSmem);
+    uint32_t cut;
+    int ties, eq;
+    radix_cut<kColsThreads, kRounds>(key, top_count(v.alpha, n) - 1, n - 1, ss, tid, BlockSync(),
+                                     cut, ties, eq);
+    const bool split = eq > ties;   // an exact tie straddles the cut
+    if (split) rank_ties<kColsThreads, kRounds>(key, cut, ties, n, tie, tid, BlockSync());
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) {
+      const int c = r * kColsThreads + tid;
+      kf[r] = c < n && (c == 0 || key[r] > cut || (key[r] == cut && (!split || tie[c] == 2)));
+    }
+  } else {
+#pragma unroll
+    for (int r = 0; r < kRounds; ++r) {
+      const int c = r * kColsThreads + tid;
+      kf[r] = c < n && __ldcg(keep + c) != 0;
+      ps[r] = c < n ? __ldcg(pos + c) : 0;
+    }
   }
 #pragma unroll
   for (int r = 0; r < kRounds; ++r) {

@@ -36,6 +36,7 @@
 #include <cstdint>
 
 #include "sc_internal.cuh"
+#include "sc_select.cuh"
 #include "sm103_primitives.cuh"
 
 namespace sc {
@@ -66,6 +67,8 @@ struct TailSmem {
   uint32_t gbits[2][kTailChunks];     // global flags of the current / next token list
   int32_t pos[2][kTailMax];           // original positions of the current / next tokens
   alignas(16) float nlse[kTailMax];   // -LSE of each query row (-inf past n)
+  SelectSmem sel;                     // top-ratio rule: the cut's histogram
+  uint8_t tie[kTailMax];              // ... and the ranks of exact ties at the cut
 };
 
 __device__ __forceinline__ bool tail_is_global(const TailSmem& sm, int ps) {
@@ -78,6 +81,10 @@ __device__ __forceinline__ bool tail_is_global(const TailSmem& sm, int ps) {
 __device__ __forceinline__ void tail_named_sync() {
   asm volatile("bar.sync 1, 256;" ::: "memory");
 }
+
+struct TailSync {   // the 256 softmax threads
+  __device__ __forceinline__ void operator()() const { tail_named_sync(); }
+};
 
 __device__ __forceinline__ bool tail_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
@@ -495,7 +502,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
     tc_fence_after();
     const int nxt = cur ^ 1;
     if (tid < 256) {
-      bool keep[2] = {false, false};
+      float sj[2] = {0.f, 0.f};
 #pragma unroll
       for (int rd = 0; rd < 2; ++rd) {
         const int j = tid + 256 * rd;
@@ -508,10 +515,43 @@ __global__ void __launch_bounds__(kTailThreads, 1)
 #pragma unroll
           for (int hh = 0; hh < kTailMaxHeads; ++hh)
             if (hh < H) a += v[hh];
-          const float s = a / static_cast<float>(H * n);
-          keep[rd] = (j == 0) || (s >= p.alpha[l] / static_cast<float>(n));
-          if (h == 0) p.scores[(static_cast<size_t>(l) * B + b) * L + j] = s;
+          sj[rd] = a / static_cast<float>(H * n);
+          if (h == 0) p.scores[(static_cast<size_t>(l) * B + b) * L + j] = sj[rd];
         }
+      }
+      // keep flags: the threshold (relative or absolute), or the top-ratio cut
+      // over the n scores (every CTA of the cluster finds the same cut)
+      bool keep[2];
+      if (p.keep_rule == kKeepTopRatio) {
+        uint32_t key[2];
+#pragma unroll
+        for (int rd = 0; rd < 2; ++rd) {
+          const int j = tid + 256 * rd;
+          key[rd] = (j >= 1 && j < n) ? select_key(sj[rd]) : 0u;
+        }
+        uint32_t cut;
+        int ties, eq;
+        radix_cut<256, 2>(key, top_count(p.alpha[l], n) - 1, n - 1, sm.sel, tid, TailSync(), cut,
+                          ties, eq);
+        const bool split = eq > ties;
+        if (split) rank_ties<256, 2>(key, cut, ties, n, sm.tie, tid, TailSync());
+#pragma unroll
+        for (int rd = 0; rd < 2; ++rd) {
+          const int j = tid + 256 * rd;
+          keep[rd] = j < n && (j == 0 || key[rd] > cut ||
+                               (key[rd] == cut && (!split || sm.tie[j] == 2)));
+        }
+      } else {
+        const float thr = p.keep_rule == kKeepAbsolute ? p.alpha[l]
+                                                       : p.alpha[l] / static_cast<float>(n);
+#pragma unroll
+        for (int rd = 0; rd < 2; ++rd) {
+          const int j = tid + 256 * rd;
+          keep[rd] = j < n && (j == 0 || sj[rd] >= thr);
+        }
+      }
+#pragma unroll
+      for (int rd = 0; rd < 2; ++rd) {
         const uint32_t kb = __ballot_sync(0xffffffffu, keep[rd]);
         if (lane == 0) sm.kbits[rd][warp] = kb;
       }

@@ -36,6 +36,10 @@ def test_binding_constants_match_the_header():
     defines = dict(re.findall(r"^#define\s+(SC_\w+)\s+(\d+)", text, re.M))
     assert int(defines["SC_TAIL_MAX_LEN"]) == bd.TAIL_MAX_LEN
     assert int(defines["SC_STACK_NO_TAIL"]) == bd.SC_STACK_NO_TAIL
+    rules = dict(re.findall(r"^\s*(SC_KEEP_\w+)\s*=\s*(\d+)", text, re.M))
+    assert {k: int(v) for k, v in rules.items()} == {
+        "SC_KEEP_RELATIVE": bd.SC_KEEP_RELATIVE, "SC_KEEP_ABSOLUTE": bd.SC_KEEP_ABSOLUTE,
+        "SC_KEEP_TOP_RATIO": bd.SC_KEEP_TOP_RATIO}
 
 
 def test_every_declared_symbol_is_exported(lib):
@@ -96,6 +100,14 @@ def test_layer_rejects_bad_arguments(lib):
     far = (ctypes.c_int32 * 2)(0, 256)                                    # outside [0, L)
     assert _call_layer(lib, global_pos=ctypes.cast(far, ctypes.POINTER(ctypes.c_int32))) \
         == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, keep_rule=3) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, keep_rule=-1) == bd.SC_ERR_INVALID_ARG
+    # the top-ratio rule takes no per-sequence thresholds and a finite ratio
+    assert _call_layer(lib, keep_rule=bd.SC_KEEP_TOP_RATIO, theta=FAKE) == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, keep_rule=bd.SC_KEEP_TOP_RATIO, alpha=float("nan")) \
+        == bd.SC_ERR_INVALID_ARG
+    assert _call_layer(lib, keep_rule=bd.SC_KEEP_TOP_RATIO, alpha=float("inf")) \
+        == bd.SC_ERR_INVALID_ARG
 
 
 def test_stack_rejects_bad_arguments(lib):
@@ -118,6 +130,10 @@ def test_stack_rejects_bad_arguments(lib):
     assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
     assert call(w=512) == bd.SC_ERR_UNSUPPORTED
     assert call(flags=2) == bd.SC_ERR_INVALID_ARG
+    assert call(keep_rule=7) == bd.SC_ERR_INVALID_ARG
+    bad = (ctypes.c_float * 12)(*([0.5] * 11 + [float("nan")]))
+    assert call(keep_rule=bd.SC_KEEP_TOP_RATIO,
+                alpha=ctypes.cast(bad, ctypes.POINTER(ctypes.c_float))) == bd.SC_ERR_INVALID_ARG
 
 
 def test_launch_count_rejects_bad_arguments(lib):

@@ -78,7 +78,7 @@ def _run_stack(sc, wl, inp, no_tail=False):
     mask = None if inp["pad_mask"] is None else torch.from_numpy(inp["pad_mask"]).to(dev)
     ws = sc.new_workspace(wl.B, wl.L, wl.H, dev)
     out = sc.stack_forward(Q, K, V, mask, inp["global_pos"], wl.w, inp["alpha"], workspace=ws,
-                           no_tail=no_tail)
+                           no_tail=no_tail, keep_rule=wl.keep_rule)
     assert sc.workspace_status(ws) == 0
     return {"O": torch_bf16_to_f64(out["O"]), "scores": out["scores"].cpu().numpy(),
             "pos": out["pos"].cpu().numpy(), "len": out["len"].cpu().numpy()}

@@ -3,7 +3,13 @@
 12-layer pruned sparse-attention stack at L = 4096 (and its roofline fraction).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
-                    [--workload cfg4|cfg2|cfg3|cfg5_L512|...|cfg5_L4096[_theta0]]
+                    [--workload cfg4|cfg2|cfg3|cfg5_L512|...|cfg5_L4096[_theta0]
+                                |abs_theta|top_ratio|window_w16|...|window_w256]
+
+Besides the default, the workloads cover the other keep rules (abs_theta: the
+absolute per-layer thresholds 0.01 l / 12 of RQ4; top_ratio: a kept ratio per
+layer, 0.95 -> 0.8) and the window-size ablation of RQ3 (window_wNN: sparse
+attention alone, nothing pruned, L = 1024, B = 8); each prints its own line.
 
 One step = one call of sc_stack_forward over the whole workload: padding removal,
 then per layer the rows kernel (band + global attention, O, row LSE) and the
@@ -41,6 +47,12 @@ if ROOT not in sys.path:
 import workloads as wk  # noqa: E402
 
 METRIC = "kept-tokens/sec per 12-layer pruned stack at L=4096; fraction of roofline"
+
+
+def metric_name(wl: wk.Workload) -> str:
+    """The metric's name for a workload (the default's is METRIC)."""
+    return "kept-tokens/sec per %d-layer pruned stack at L=%d; fraction of roofline" % (
+        wl.n_layers, wl.L)
 UNIT = "kept-tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 BYTES_PER_TOKEN = 6152      # Q,K,V read (3*12*64*2) + O write (12*64*2) + score (4) + position (4)
@@ -54,6 +66,12 @@ def pick_workload(name: str) -> wk.Workload:
         rest = name[len("cfg5_L"):]
         control = rest.endswith("_theta0")
         return wk.cfg5(int(rest.replace("_theta0", "")), control=control)
+    if name == "abs_theta":
+        return wk.ABS_THETA
+    if name == "top_ratio":
+        return wk.TOP_RATIO
+    if name.startswith("window_w"):
+        return wk.window_sweep(int(name[len("window_w"):]))
     raise SystemExit("unknown workload %s" % name)
 
 
@@ -302,7 +320,7 @@ def oracle_sample(wl, inp, b, n_layers, threads):
     Q, K, V = (np.ascontiguousarray(inp[k][:n_layers, sl]) for k in ("Q", "K", "V"))
     t0 = time.perf_counter()
     res = oracle.stack(Q, K, V, mask, inp["global_pos"], wl.w, inp["alpha"][:n_layers],
-                       want_O=True, nthreads=threads)
+                       want_O=True, nthreads=threads, keep_rule=wl.keep_rule)
     dt = time.perf_counter() - t0
     return dt, int(res["len"][:n_layers].sum()), min(threads, wl.H)
 
@@ -325,7 +343,7 @@ def run_reference(args, wl):
         tot_tok += tok
     value = tot_tok / tot_t
     sample = "one sequence of the workload, first %d layer(s), per step" % layers
-    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+    line = {"impl": "reference", "metric": metric_name(wl), "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -370,7 +388,7 @@ def run_native(args, wl):
     def step(events=None):
         nonlocal out
         out = sc.stack_forward(dQKV["Q"], dQKV["K"], dQKV["V"], mask, gpos, wl.w, alpha,
-                               out=out, workspace=ws, events=events)
+                               out=out, workspace=ws, events=events, keep_rule=wl.keep_rule)
 
     def barrier():
         if world > 1:
@@ -535,7 +553,7 @@ def run_native(args, wl):
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
            "ms_per_step": e2e_ms}
 
-    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+    line = {"metric": metric_name(wl), "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",

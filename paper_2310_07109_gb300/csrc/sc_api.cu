@@ -48,7 +48,8 @@ int fail_cuda(const char* what, cudaError_t e) {
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
-  size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, gcur, ng, ident,
+  size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, rows_done, gcur, ng,
+      ident,
       tail_from,
       loop_layer, qkv, total;
 };
@@ -71,6 +72,7 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->keep = take(sizeof(uint8_t) * B * (size_t)L);
   w->cnt_tile = take(sizeof(uint32_t) * B * T);
   w->cnt_seq = take(sizeof(uint32_t) * B);
+  w->rows_done = take(sizeof(uint32_t) * B * H);
   w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
   w->ng = take(sizeof(int32_t) * 2 * B);
   w->ident = take(sizeof(int32_t) * 2 * B);
@@ -259,6 +261,7 @@ void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->keep = reinterpret_cast<uint8_t*>(ws + lay.keep);
   p->cnt_tile = reinterpret_cast<uint32_t*>(ws + lay.cnt_tile);
   p->cnt_seq = reinterpret_cast<uint32_t*>(ws + lay.cnt_seq);
+  p->rows_done = reinterpret_cast<uint32_t*>(ws + lay.rows_done);
   int32_t* gcur = reinterpret_cast<int32_t*>(ws + lay.gcur);
   int32_t* ng = reinterpret_cast<int32_t*>(ws + lay.ng);
   int32_t* ident = reinterpret_cast<int32_t*>(ws + lay.ident);

@@ -79,6 +79,7 @@ struct LayerParams {
   uint8_t* keep;         // [B][L]
   uint32_t* cnt_tile;    // [B][T]
   uint32_t* cnt_seq;     // [B]
+  uint32_t* rows_done;   // [B][H]: rows CTAs of (sequence, head) whose results are visible
   int* status;
   // hand-over to the cluster kernel: sequence b is skipped here once
   // tail_from[b] <= layer; the finalize of a layer sets tail_from[b] = layer + 1

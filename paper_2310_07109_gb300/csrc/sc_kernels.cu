@@ -122,7 +122,7 @@ struct RowSource {
 };
 
 __device__ __forceinline__ RowSource row_source(const LayerParams& p, const LayerView& v, int b) {
-  const bool id = __ldg(v.ident + b) != 0;
+  const bool id = __ldcg(v.ident + b) != 0;
   return {id ? 0 : 1, (id ? v.src_base : 0) + static_cast<long long>(b) * p.L};
 }
 
@@ -274,11 +274,15 @@ struct OpMax {
 
 __global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
-  pdl_launch_dependents();
+  // the cols kernel is scheduled once every CTA here has passed this wait, so
+  // what the kernels before this one wrote is complete when it starts
   pdl_wait();
-  // grid: x = (sequence, head), y = pair of query tiles, so that low tiles (the
-  // ones every sequence has) are dispatched first
-  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
+  pdl_launch_dependents();
+  // grid: pairs of query tiles, (sequence, head)-major, so that the CTAs of a
+  // (sequence, head) finish together and its cols CTAs can start early
+  const int T2 = (p.T + 1) / 2;
+  const int pr = blockIdx.x % T2, bh = blockIdx.x / T2;
+  const int h = bh % p.H, b = bh / p.H;
   const LayerView v = layer_view(p);
   if (owned_by_tail(p, v, b)) return;
   const int n = __ldcg(v.len + b);
@@ -745,12 +749,16 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   }
 
   tc_fence_before();
+  __threadfence();   // O, the partial sums and statistics of this CTA ...
   __syncthreads();
   if (warp == 9) {
     tc_fence_after();
     tmem_dealloc(tm, 512);
   }
-  if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
+  if (tid == 0) {
+    if (sm.abort) atomicOr(p.status, kStatusTimeout);
+    red_release_add_u32(p.rows_done + b * p.H + h, 1u);   // ... are visible to the cols CTAs
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -800,9 +808,14 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
 
 __global__ void __launch_bounds__(kColsThreads, 2)
     sc_cols_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
+  // No grid-wide wait on the rows kernel: this kernel is scheduled only after
+  // every rows CTA has passed its own wait (so the earlier kernels' results
+  // are complete), and each CTA waits below for the rows CTAs of its own
+  // (sequence, head) only, so that it can run beside the rows kernel's last CTAs.
   pdl_launch_dependents();
-  pdl_wait();
-  const int h = blockIdx.x % p.H, b = blockIdx.x / p.H, pr = blockIdx.y;
+  const int T2 = (p.T + 1) / 2;
+  const int pr = blockIdx.x % T2, bh = blockIdx.x / T2;
+  const int h = bh % p.H, b = bh / p.H;
   const LayerView v = layer_view(p);
   if (owned_by_tail(p, v, b)) return;
   const int n = __ldcg(v.len + b);
@@ -907,6 +920,10 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     const bool active = X == 0 || hasB;
     const uint32_t lane_off = static_cast<uint32_t>(wq * 32) << 16;
     const uint32_t tSG = tm + 16 * X, tOG = tm + 64 + 64 * X;
+    // the rows CTAs of this (sequence, head) have finished (their partial
+    // sums, statistics and the cleared global-row outputs are read below)
+    if (tid == 0) wait_count(p.rows_done + b * p.H + h, static_cast<uint32_t>(Tp), abort_flag);
+    asm volatile("bar.sync 3, 256;" ::: "memory");
     // every load of the prologue is issued before any is used: this key's
     // band-row column sums of the query tiles of its band (one per tile, from
     // the rows kernel) and, per warp, the (max, sum) pieces of global rows
@@ -1229,6 +1246,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
     v.ident_out[b] = (total == 0 || sm.last_pos == total - 1) ? 1 : 0;
     p.cnt_seq[b] = 0u;
+    for (int hh = 0; hh < p.H; ++hh) p.rows_done[b * p.H + hh] = 0u;
   }
 }
 
@@ -1462,12 +1480,12 @@ cudaError_t configure_kernels() {
 }
 
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.B * p.H, (p.T + 1) / 2);
+  dim3 grid(p.B * p.H * ((p.T + 1) / 2));
   return launch_chained(sc_rows_kernel, grid, dim3(kRowsThreads), kRowsDyn, st, m, p);
 }
 
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.B * p.H, (p.T + 1) / 2);
+  dim3 grid(p.B * p.H * ((p.T + 1) / 2));
   return launch_chained(sc_cols_kernel, grid, dim3(kColsThreads), kColsDyn, st, m, p);
 }
 

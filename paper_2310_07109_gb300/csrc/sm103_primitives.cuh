@@ -111,6 +111,34 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// A counter in global memory that other CTAs raise once their results are
+// visible (release), waited for with acquire loads, bounded like mbar_wait.
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* ptr) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void red_release_add_u32(uint32_t* ptr, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ bool wait_count(const uint32_t* ctr, uint32_t target,
+                                           volatile int* abort,
+                                           uint64_t limit_ns = 2000000000ull) {
+  if (ld_acquire_u32(ctr) >= target) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    __nanosleep(100);
+    if (ld_acquire_u32(ctr) >= target) return true;
+    if (*abort) return false;
+    if (global_timer_ns() - t0 > limit_ns) {
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
 // Programmatic dependent launch.  Each kernel of the chain lets the next one
 // be scheduled at once (its CTAs take only free SM resources: every CTA of

@@ -284,10 +284,14 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   const int pr = blockIdx.x % T2, bh = blockIdx.x / T2;
   const int h = bh % p.H, b = bh / p.H;
   const LayerView v = layer_view(p);
-  if (owned_by_tail(p, v, b)) return;
+  // the sequence's state, loaded together
+  const bool tailed = owned_by_tail(p, v, b);
   const int n = __ldcg(v.len + b);
+  const int ng_raw = __ldcg(v.ng + b);
+  const int gc_raw = threadIdx.x < kMaxGlobal ? __ldcg(v.gcur + b * kMaxGlobal + threadIdx.x) : -1;
+  if (tailed) return;
   if (2 * pr * kTile >= n) return;
-  const int ng = min(__ldcg(v.ng + b), kMaxGlobal);
+  const int ng = min(ng_raw, kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
   const bool hasB = (2 * pr + 1) * kTile < n;
 
@@ -334,7 +338,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? __ldcg(v.gcur + b * kMaxGlobal + tid) : -1;
+  if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? gc_raw : -1;
   if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
@@ -348,9 +352,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     // ------------------------------------------------------------- Q, globals, K
     const RowSource rs = row_source(p, v, b);
     if (lane == 0) {
+      // Q, then the first two K tiles (the first S needs Q and K), then the
+      // global rows, then the other K tiles
       mbar_arrive_expect_tx(&sm.bar_q, (hasB ? 2 : 1) * kTileBytes + 3 * ngp * 128);
       load_tile(maps, 0, rs, h, 2 * pr * kTile, Qs, &sm.bar_q);
       if (hasB) load_tile(maps, 0, rs, h, (2 * pr + 1) * kTile, Qs + kTileBytes, &sm.bar_q);
+      for (int k = 0; k < nk && k < 2; ++k) {
+        mbar_arrive_expect_tx(&sm.bar_kfull[k], kTileBytes);
+        load_tile(maps, 1, rs, h, (kt_lo + k) * kTile, Ks + k * kTileBytes, &sm.bar_kfull[k]);
+      }
     }
     __syncwarp();
     if (ngp) {
@@ -359,7 +369,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       load_globals(maps, 0, rs, h, p.H, sm.gc, ng, QG, &sm.bar_q, lane);
     }
     if (lane == 0) {
-      for (int k = 0; k < nk; ++k) {
+      for (int k = 2; k < nk; ++k) {
         mbar_arrive_expect_tx(&sm.bar_kfull[k], kTileBytes);
         load_tile(maps, 1, rs, h, (kt_lo + k) * kTile, Ks + k * kTileBytes, &sm.bar_kfull[k]);
       }

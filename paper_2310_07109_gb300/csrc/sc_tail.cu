@@ -426,6 +426,9 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         tmem_ld32(tO, o);
         tmem_ld32(tO + 32, o + 32);
         tmem_ld_wait();
+        sm.nlse[i] = me.valid ? -(lg2(lsum) - nmc) : -INFINITY;
+        // O is in registers: the columns may take S^T while O is stored
+        release();
         // the warp's 32 rows leave in two column halves of 64 bytes
         uint8_t* stage = base + 3 * kTailOpBytes + warp * 2048;
         uint16_t* row0 =
@@ -442,8 +445,6 @@ __global__ void __launch_bounds__(kTailThreads, 1)
                                           pack_bf16x2(o[c + k + 6] * inv, o[c + k + 7] * inv)));
           flush_staged_rows<4>(stage, row0 + c, static_cast<size_t>(H) * kHeadDim, rows);
         }
-        sm.nlse[i] = me.valid ? -(lg2(lsum) - nmc) : -INFINITY;
-        release();
       }
       // rows past the last query tile take no part in the column sums
       for (int i = kTile * nq + (tid & 255); i < kTailMax; i += 256) sm.nlse[i] = -INFINITY;

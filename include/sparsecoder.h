@@ -56,7 +56,7 @@ extern "C" {
 #define SC_HEAD_DIM 64
 #define SC_MAX_LEN 4096   /* longest supported (padded) sequence */
 #define SC_MAX_GLOBAL 16  /* most global positions per call */
-#define SC_MAX_WINDOW 256 /* widest one-sided window when L > 640 */
+#define SC_MAX_WINDOW 512 /* widest one-sided window when L > 640 */
 #define SC_TAIL_MAX_LEN 384 /* sequences this short finish in the cluster kernel (see sc_stack_forward) */
 
 typedef enum {
@@ -173,10 +173,10 @@ typedef struct {
  * counterpart; this is an interface convenience.
  *
  * Same arguments, semantics and results as sc_layer_forward (the caller still
- * passes every input and output).  The scratch comes from a 4 MiB array
+ * passes every input and output).  The scratch comes from a 6 MiB array
  * compiled into the library, which every GPU that loads it holds until the
- * process exits; sizes whose scratch does not fit (from roughly B*L*H = 300k
- * (sequence, token, head) rows on, e.g. B=2, L=4096, H=12 fits) return
+ * process exits; sizes whose scratch does not fit (from roughly B*L*H = 130k
+ * (sequence, token, head) rows on; B=2, L=4096, H=12 is 98k and fits) return
  * SC_ERR_UNSUPPORTED with the detail in sc_last_error().  The first call
  * on each device looks up the array's device address (cudaGetSymbolAddress);
  * make that first call before any stream capture.  All calls share the array:

@@ -20,7 +20,7 @@ _lib = None
 SC_HEAD_DIM = 64
 SC_MAX_LEN = 4096
 SC_MAX_GLOBAL = 16
-SC_MAX_WINDOW = 256
+SC_MAX_WINDOW = 512
 
 SC_OK, SC_ERR_INVALID_ARG, SC_ERR_UNSUPPORTED, SC_ERR_CUDA, SC_ERR_TIMEOUT, SC_ERR_WORKSPACE = range(6)
 

@@ -65,7 +65,7 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   };
   w->status = take(kAlign);
   w->acc = take(sizeof(float) * B * H * (size_t)L);
-  w->colpart = take(sizeof(float) * B * H * (size_t)L * kMaxBandTiles);
+  w->colpart = take(sizeof(float) * B * H * (size_t)L * kWideBandTiles);
   w->gpart = take(sizeof(float) * B * H * T * 4 * kMaxGlobal);
   w->gstat = take(sizeof(float) * B * H * T * 4 * kMaxGlobal * 2);
   w->og = take(sizeof(float) * B * H * kMaxGlobal * kHeadDim);
@@ -232,7 +232,7 @@ int check_common(int B, int L, int H, int w, const int32_t* gpos, int ngl) {
     if (gpos[g] < 0 || gpos[g] >= L) return SC_ERR_INVALID_ARG;
     if (g > 0 && gpos[g] <= gpos[g - 1]) return SC_ERR_INVALID_ARG;
   }
-  // one 128-row tile must reach at most five 128-key tiles
+  // one 128-row tile must reach at most nine 128-key tiles
   if (L > kMaxBandTiles * kTile && w > SC_MAX_WINDOW) return SC_ERR_UNSUPPORTED;
   if (static_cast<long long>(B) * L * H > (1ll << 30)) return SC_ERR_UNSUPPORTED;
   return SC_OK;
@@ -271,6 +271,10 @@ void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->ng_out = ng + (1 - slot) * p->B;
   p->ident = ident + slot * p->B;
   p->ident_out = ident + (1 - slot) * p->B;
+  // rows kernel layout: pairs of query tiles, or single tiles when a tile's
+  // band reaches more than five key tiles
+  p->wide = (p->w > kPairWindow && p->T > kMaxBandTiles) ? 1 : 0;
+  p->band_slots = p->wide ? kWideBandTiles : kMaxBandTiles;
 }
 
 void compacted_qkv(char* ws, const WsLayout& lay, int B, int L, int H, uint16_t* out[3]) {
@@ -675,7 +679,7 @@ int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {
 // the library until the process exits.
 namespace {
 
-constexpr size_t kStaticWorkspaceBytes = size_t(4) << 20;  // 4 MiB
+constexpr size_t kStaticWorkspaceBytes = size_t(6) << 20;  // 6 MiB
 
 }  // namespace
 

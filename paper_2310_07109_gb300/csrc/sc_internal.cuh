@@ -11,7 +11,9 @@ namespace sc {
 
 constexpr int kHeadDim = 64;
 constexpr int kTile = 128;         // rows (queries or keys) per tile
-constexpr int kMaxBandTiles = 5;   // key (query) tiles touched by one 128-row tile
+constexpr int kMaxBandTiles = 5;   // key (query) tiles touched by one 128-row tile, w <= 256
+constexpr int kWideBandTiles = 9;  // ... with a wide window, 256 < w <= 512
+constexpr int kPairWindow = 256;   // widest window of the paired rows layout on long sequences
 constexpr int kMaxGlobal = 16;     // global tokens per sequence (one 16-wide MMA tile)
 constexpr int kMaxLen = 4096;
 constexpr int kMaxTiles = kMaxLen / kTile;
@@ -69,8 +71,10 @@ struct LayerParams {
   int keep_rule;         // kKeepRelative, kKeepAbsolute or kKeepTopRatio
   // workspace
   float* acc;            // [B][H][L] per-head column sums: band rows + global rows
-  float* colpart;        // [B][H][L][kMaxBandTiles] band-row column sums per query tile
-                         //   (slot = query tile mod kMaxBandTiles)
+  float* colpart;        // [B][H][L][band_slots] band-row column sums per query tile
+                         //   (slot = query tile mod band_slots)
+  int band_slots;        // kMaxBandTiles, or kWideBandTiles with wide
+  int wide;              // rows kernel: one query tile per CTA (256 < w on long sequences)
   float* gpart;          // [B][H][T][4][kMaxGlobal] column sums of global keys over far rows,
                          //   per (query tile, 32-row warp slice)
   float* gstat;          // [B][H][T][4][kMaxGlobal][2] (max, sum) of global rows per

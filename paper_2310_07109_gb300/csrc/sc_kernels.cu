@@ -209,6 +209,12 @@ constexpr int kPairTiles = kMaxBandTiles + 1;
 // the first is used by query tile 0 alone and the sixth by query tile 1 alone
 // (each query tile's band spans at most five key tiles).
 constexpr int kVStages = kPairTiles - 1;
+// Wide windows (256 < w <= 512 on sequences of more than five tiles): one
+// query tile per CTA, up to nine resident key tiles and a three-slot V ring in
+// the same shared memory (one Q tile + 9 + 3 = two Q tiles + 6 + 5).
+constexpr int kWideVStages = 3;
+static_assert(1 + kWideBandTiles + kWideVStages == 2 + kPairTiles + kVStages,
+              "both layouts fill the same shared memory");
 
 __host__ __device__ constexpr uint32_t col_s(int X) { return 256u * X; }
 __host__ __device__ constexpr uint32_t col_p(int X) { return 256u * X + 128u; }
@@ -217,7 +223,7 @@ __host__ __device__ constexpr uint32_t col_o(int X) { return 256u * X + 192u; }
 struct RowsSmem {
   alignas(16) float nlse[2][kTile];   // -LSE of each query tile's rows (read as float4)
   uint64_t bar_q;
-  uint64_t bar_kfull[kPairTiles];
+  uint64_t bar_kfull[kWideBandTiles];
   uint64_t bar_vfull[kVStages], bar_vempty[kVStages];
   uint64_t bar_sg[2], bar_sgend[2], bar_sfull[2], bar_sfree[2], bar_pready[2], bar_pvdone[2];
   uint64_t bar_fin[2];
@@ -272,17 +278,23 @@ struct OpMax {
   __device__ __forceinline__ float operator()(float a, float b) const { return fmaxf(a, b); }
 };
 
+// kWide: one query tile per CTA (see kWideVStages); otherwise pairs of tiles.
+template <bool kWide>
 __global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
   // the cols kernel is scheduled once every CTA here has passed this wait, so
   // what the kernels before this one wrote is complete when it starts
   pdl_wait();
   pdl_launch_dependents();
-  // grid: pairs of query tiles, (sequence, head)-major, so that the CTAs of a
-  // (sequence, head) finish together and its cols CTAs can start early
-  const int T2 = (p.T + 1) / 2;
-  const int pr = blockIdx.x % T2, bh = blockIdx.x / T2;
+  // grid: pairs of query tiles (single tiles with a wide window),
+  // (sequence, head)-major, so that the CTAs of a (sequence, head) finish
+  // together and its cols CTAs can start early
+  constexpr bool wide = kWide;
+  constexpr int band_slots = wide ? kWideBandTiles : kMaxBandTiles;
+  const int per_bh = wide ? p.T : (p.T + 1) / 2;
+  const int pr = blockIdx.x % per_bh, bh = blockIdx.x / per_bh;
   const int h = bh % p.H, b = bh / p.H;
+  const int q_first = wide ? pr : 2 * pr;   // first query tile of this CTA
   const LayerView v = layer_view(p);
   // the sequence's state, loaded together
   const bool tailed = owned_by_tail(p, v, b);
@@ -290,18 +302,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   const int ng_raw = __ldcg(v.ng + b);
   const int gc_raw = threadIdx.x < kMaxGlobal ? __ldcg(v.gcur + b * kMaxGlobal + threadIdx.x) : -1;
   if (tailed) return;
-  if (2 * pr * kTile >= n) return;
+  if (q_first * kTile >= n) return;
   const int ng = min(ng_raw, kMaxGlobal);
   const int ngp = ng > 0 ? kMaxGlobal : 0;
-  const bool hasB = (2 * pr + 1) * kTile < n;
+  const bool hasB = !wide && (q_first + 1) * kTile < n;
+  constexpr int nvs = wide ? kWideVStages : kVStages;   // V ring slots
 
   extern __shared__ uint8_t dyn_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* Qs = base;                                // 2 tiles
-  uint8_t* Ks = Qs + 2 * kTileBytes;                 // kPairTiles tiles (all resident)
-  uint8_t* Vs = Ks + kPairTiles * kTileBytes;        // kVStages tiles
-  uint8_t* KG = Vs + kVStages * kTileBytes;
+  uint8_t* Qs = base;                                        // 2 tiles (wide: 1)
+  uint8_t* Ks = Qs + (wide ? 1 : 2) * kTileBytes;            // all resident: 6 (wide: 9)
+  uint8_t* Vs = Ks + (wide ? kWideBandTiles : kPairTiles) * kTileBytes;   // nvs slots
+  uint8_t* KG = Vs + nvs * kTileBytes;
   uint8_t* VG = KG + kGTileBytes;
   uint8_t* QG = VG + kGTileBytes;
   __shared__ RowsSmem sm;
@@ -311,17 +324,17 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
   int klo[2], khi[2];
 #pragma unroll
   for (int X = 0; X < 2; ++X) {
-    const int q0 = (2 * pr + X) * kTile, q1 = min(q0 + kTile - 1, n - 1);
+    const int q0 = (q_first + X) * kTile, q1 = min(q0 + kTile - 1, n - 1);
     klo[X] = max(0, q0 - p.w) / kTile;
     khi[X] = min(n - 1, q1 + p.w) / kTile;
   }
   const int kt_lo = klo[0];
   const int kt_hi = hasB ? khi[1] : khi[0];
-  const int nk = kt_hi - kt_lo + 1;   // <= kPairTiles (window checked on the host)
+  const int nk = kt_hi - kt_lo + 1;   // <= 6 (wide: 9); window checked on the host
 
   if (tid == 0) {
     mbar_init(&sm.bar_q, 1);
-    for (int k = 0; k < kPairTiles; ++k) mbar_init(&sm.bar_kfull[k], 1);
+    for (int k = 0; k < kWideBandTiles; ++k) mbar_init(&sm.bar_kfull[k], 1);
     for (int s = 0; s < kVStages; ++s) {
       mbar_init(&sm.bar_vfull[s], 1);
       mbar_init(&sm.bar_vempty[s], 1);
@@ -355,8 +368,8 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       // Q, then the first two K tiles (the first S needs Q and K), then the
       // global rows, then the other K tiles
       mbar_arrive_expect_tx(&sm.bar_q, (hasB ? 2 : 1) * kTileBytes + 3 * ngp * 128);
-      load_tile(maps, 0, rs, h, 2 * pr * kTile, Qs, &sm.bar_q);
-      if (hasB) load_tile(maps, 0, rs, h, (2 * pr + 1) * kTile, Qs + kTileBytes, &sm.bar_q);
+      load_tile(maps, 0, rs, h, q_first * kTile, Qs, &sm.bar_q);
+      if (hasB) load_tile(maps, 0, rs, h, (q_first + 1) * kTile, Qs + kTileBytes, &sm.bar_q);
       for (int k = 0; k < nk && k < 2; ++k) {
         mbar_arrive_expect_tx(&sm.bar_kfull[k], kTileBytes);
         load_tile(maps, 1, rs, h, (kt_lo + k) * kTile, Ks + k * kTileBytes, &sm.bar_kfull[k]);
@@ -382,17 +395,19 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     if (lane == 0) {
       const RowSource rs = row_source(p, v, b);
       bool ok = true;
-      for (int k = 0; ok && k < nk; ++k) {
-        const int s = k % kVStages;
-        if (k >= kVStages &&
-            !(ok = mbar_wait(&sm.bar_vempty[s], ((k / kVStages) - 1) & 1, abort_flag)))
-          break;
+      // slot s = k mod nvs and its use count, advanced without division
+      for (int k = 0, s = 0, use = 0; ok && k < nk; ++k) {
+        if (k >= nvs && !(ok = mbar_wait(&sm.bar_vempty[s], (use - 1) & 1, abort_flag))) break;
         mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
         load_tile(maps, 2, rs, h, (kt_lo + k) * kTile, Vs + s * kTileBytes, &sm.bar_vfull[s]);
+        if (++s == nvs) {
+          s = 0;
+          ++use;
+        }
       }
-      for (int s = 0; s < kVStages && s < nk; ++s) {
-        const int last = s + kVStages * ((nk - 1 - s) / kVStages);
-        drain_wait(&sm.bar_vfull[s], (last / kVStages) & 1);
+      for (int s = 0; s < nvs && s < nk; ++s) {
+        const int last = s + nvs * ((nk - 1 - s) / nvs);
+        drain_wait(&sm.bar_vfull[s], (last / nvs) & 1);
       }
     }
    } else if (warp == 9 || warp == 11) {
@@ -422,6 +437,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         return true;
       };
       uint32_t nfree = 0, nready = 0;
+      // V slot of key tile k = a - kt_lo (k mod nvs) and its use count, advanced
+      // without division
+      int vslot = (kloX - kt_lo) % nvs, vuse = (kloX - kt_lo) / nvs;
       if (ok) ok = issue_s(kloX);
       if (ok && ngp) {
         if ((ok = mbar_wait(&sm.bar_pready[X], (nready++) & 1, abort_flag))) {
@@ -439,14 +457,18 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
           // the last S is read: its columns take S_G and S_Gt for the epilogue
           tc_fence_after();
           mma_qk(tS, q_a, smem_u32(KG), 16);
-          mma_qk(tS + 16, k_a + (2 * pr + X - kt_lo) * kTileBytes, smem_u32(QG), 16);
+          mma_qk(tS + 16, k_a + (q_first + X - kt_lo) * kTileBytes, smem_u32(QG), 16);
           umma_commit(&sm.bar_sgend[X]);
         }
         if (!(ok = mbar_wait(&sm.bar_pready[X], (nready++) & 1, abort_flag))) break;
-        if (!(ok = mbar_wait(&sm.bar_vfull[k % kVStages], (k / kVStages) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait(&sm.bar_vfull[vslot], vuse & 1, abort_flag))) break;
         tc_fence_after();
-        mma_pv_ts(tO, tP, v_a + (k % kVStages) * kTileBytes, kTile / 16, ngp > 0 || a > kloX);
-        if (k + kVStages < nk) umma_commit(&sm.bar_vempty[k % kVStages]);   // slot reused
+        mma_pv_ts(tO, tP, v_a + vslot * kTileBytes, kTile / 16, ngp > 0 || a > kloX);
+        if (k + nvs < nk) umma_commit(&sm.bar_vempty[vslot]);   // slot reused
+        if (++vslot == nvs) {
+          vslot = 0;
+          ++vuse;
+        }
         umma_commit(&sm.bar_pvdone[X]);
       }
       // band pass: S^T = K Q^T of each key tile of the band against this
@@ -471,7 +493,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     const int kloX = X ? klo[1] : klo[0], khiX = X ? khi[1] : khi[0];
     const int wq = warp & 3;              // TMEM lane quarter of this warp
     const int r = tid & 127;              // row inside the tile == TMEM lane
-    const int qt = 2 * pr + X;
+    const int qt = q_first + X;
     const int r0 = qt * kTile;
     const bool active = X == 0 || hasB;
     const int i = r0 + r;                 // current index of this query row
@@ -729,7 +751,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       f2_unpack(s2a, sa, sb);
       f2_unpack(s2b, sc2, sd);
       if (j < n)
-        p.colpart[((static_cast<size_t>(b) * p.H + h) * p.L + j) * kMaxBandTiles + qt % kMaxBandTiles] =
+        p.colpart[((static_cast<size_t>(b) * p.H + h) * p.L + j) * band_slots + qt % band_slots] =
             (sa + sc2) + (sb + sd);
     }
 
@@ -781,6 +803,17 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 // Tensor memory (256 columns, so that two CTAs share an SM) per warpgroup X:
 // S^T against the global queries [16 X, +16), the global rows' P V
 // [64 + 64 X, +64).
+// The band rows' column sums of key j from the rows kernel, one per query tile
+// qlo..qhi in tile order (slot = tile mod kSlots); entries past qhi are 0.
+template <int kSlots>
+__device__ __forceinline__ void load_band_parts(float (&part)[kWideBandTiles], const LayerParams& p,
+                                                int b, int h, int j, int qlo, int qhi, bool use) {
+  const float* cp = p.colpart + ((static_cast<size_t>(b) * p.H + h) * p.L + j) * kSlots;
+#pragma unroll
+  for (int u = 0; u < kWideBandTiles; ++u)
+    part[u] = (u < kSlots && use && qlo + u <= qhi) ? __ldcg(cp + (qlo + u) % kSlots) : 0.f;
+}
+
 constexpr int kColsThreads = 320;
 // The global rows' P is the A operand of an M = 128 MMA whose rows past the 16
 // global rows are never used: each 64-key block of that A tile holds its 16
@@ -932,20 +965,18 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     const uint32_t tSG = tm + 16 * X, tOG = tm + 64 + 64 * X;
     // the rows CTAs of this (sequence, head) have finished (their partial
     // sums, statistics and the cleared global-row outputs are read below)
-    if (tid == 0) wait_count(p.rows_done + b * p.H + h, static_cast<uint32_t>(Tp), abort_flag);
+    if (tid == 0)
+      wait_count(p.rows_done + b * p.H + h, static_cast<uint32_t>(p.wide ? Tn : Tp), abort_flag);
     asm volatile("bar.sync 3, 256;" ::: "memory");
     // every load of the prologue is issued before any is used: this key's
     // band-row column sums of the query tiles of its band (one per tile, from
     // the rows kernel) and, per warp, the (max, sum) pieces of global rows
     // warp and warp + 8
-    float part[kMaxBandTiles];
-    const float* cp =
-        p.colpart + ((static_cast<size_t>(b) * p.H + h) * p.L + j) * kMaxBandTiles;
-#pragma unroll
-    for (int u = 0; u < kMaxBandTiles; ++u) {
-      const int q = qloX + u;
-      part[u] = (active && j < n && q <= qhiX) ? __ldcg(cp + q % kMaxBandTiles) : 0.f;
-    }
+    float part[kWideBandTiles];
+    if (p.band_slots == kMaxBandTiles)
+      load_band_parts<kMaxBandTiles>(part, p, b, h, j, qloX, qhiX, active && j < n);
+    else
+      load_band_parts<kWideBandTiles>(part, p, b, h, j, qloX, qhiX, active && j < n);
     // lane k takes entries k, k+32, k+64, k+96 of the 4 Tn (key tile, warp
     // slice) pieces; the warp combines them in a fixed order
     const size_t base_slot = (static_cast<size_t>(b) * p.H + h) * p.T * 4 * kMaxGlobal;
@@ -979,7 +1010,7 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     // band rows: the query tiles' sums in tile order
     float acc = 0.f;
 #pragma unroll
-    for (int u = 0; u < kMaxBandTiles; ++u) acc += part[u];
+    for (int u = 0; u < kWideBandTiles; ++u) acc += part[u];
     const bool ok = active;
     float x[16];
 
@@ -1475,11 +1506,15 @@ cudaError_t launch_prep(const PrepParams& pp, cudaStream_t st) {
 
 cudaError_t configure_kernels() {
   // the attention kernels use most of an SM's shared memory
-  cudaError_t e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(kRowsDyn));
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(sc_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                             cudaSharedmemCarveoutMaxShared);
+  cudaError_t e = cudaSuccess;
+  for (auto k : {sc_rows_kernel<false>, sc_rows_kernel<true>}) {
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(kRowsDyn));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared);
+  }
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(sc_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(kColsDyn));
@@ -1490,8 +1525,11 @@ cudaError_t configure_kernels() {
 }
 
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {
-  dim3 grid(p.B * p.H * ((p.T + 1) / 2));
-  return launch_chained(sc_rows_kernel, grid, dim3(kRowsThreads), kRowsDyn, st, m, p);
+  if (p.wide)
+    return launch_chained(sc_rows_kernel<true>, dim3(p.B * p.H * p.T), dim3(kRowsThreads),
+                          kRowsDyn, st, m, p);
+  return launch_chained(sc_rows_kernel<false>, dim3(p.B * p.H * ((p.T + 1) / 2)),
+                        dim3(kRowsThreads), kRowsDyn, st, m, p);
 }
 
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st) {

@@ -36,6 +36,7 @@ def test_binding_constants_match_the_header():
     defines = dict(re.findall(r"^#define\s+(SC_\w+)\s+(\d+)", text, re.M))
     assert int(defines["SC_TAIL_MAX_LEN"]) == bd.TAIL_MAX_LEN
     assert int(defines["SC_STACK_NO_TAIL"]) == bd.SC_STACK_NO_TAIL
+    assert int(defines["SC_MAX_WINDOW"]) == bd.SC_MAX_WINDOW
     rules = dict(re.findall(r"^\s*(SC_KEEP_\w+)\s*=\s*(\d+)", text, re.M))
     assert {k: int(v) for k, v in rules.items()} == {
         "SC_KEEP_RELATIVE": bd.SC_KEEP_RELATIVE, "SC_KEEP_ABSOLUTE": bd.SC_KEEP_ABSOLUTE,
@@ -84,7 +85,7 @@ def test_layer_rejects_bad_arguments(lib):
     assert _call_layer(lib, B=0) == bd.SC_ERR_INVALID_ARG
     assert _call_layer(lib, w=-1) == bd.SC_ERR_INVALID_ARG
     assert _call_layer(lib, L=5000) == bd.SC_ERR_UNSUPPORTED
-    assert _call_layer(lib, L=2048, w=300) == bd.SC_ERR_UNSUPPORTED
+    assert _call_layer(lib, L=2048, w=513) == bd.SC_ERR_UNSUPPORTED
     assert _call_layer(lib, n_global=17) == bd.SC_ERR_UNSUPPORTED
     assert _call_layer(lib, Q=FAKE + 8) == bd.SC_ERR_INVALID_ARG        # not 16-byte aligned
     assert _call_layer(lib, pos_out=FAKE) == bd.SC_ERR_INVALID_ARG      # aliases pos
@@ -128,7 +129,7 @@ def test_stack_rejects_bad_arguments(lib):
     assert call(O=None) == bd.SC_ERR_INVALID_ARG
     assert call(V=FAKE + 2) == bd.SC_ERR_INVALID_ARG
     assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
-    assert call(w=512) == bd.SC_ERR_UNSUPPORTED
+    assert call(w=513) == bd.SC_ERR_UNSUPPORTED
     assert call(flags=2) == bd.SC_ERR_INVALID_ARG
     assert call(keep_rule=7) == bd.SC_ERR_INVALID_ARG
     bad = (ctypes.c_float * 12)(*([0.5] * 11 + [float("nan")]))

@@ -60,6 +60,10 @@ LAYER_CASES = [
     (2, 900, [0, 900], 256, [0, 450], 0.9, False),           # an empty sequence
     (2, 400, [400, 333], 32, [0], 1.0, True),                # gaps in original positions
     (1, 1024, [1024], 0, [0, 1, 2, 1023], 0.5, False),       # w = 0: diagonal + globals
+    # wide windows on long sequences: one query tile per rows CTA, up to nine
+    # key tiles per band
+    (2, 1024, [1024, 700], 512, [0, 300], 0.6, False),
+    (1, 2048, [2048], 300, [0, 1000, 2047], 0.7, False),
 ]
 
 
@@ -108,6 +112,8 @@ STACKS = [
     wk.Workload("salient4_4x1000", n_layers=4, B=1, L=1000, w=256, n_extra_global=8,
                 salient_frac=0.05, salient_scale=4.0, alpha_first=0.4, alpha_last=1.0, seed=5),
     wk.CFG1,
+    wk.Workload("wide_w512_4x1024", n_layers=4, B=2, L=1024, w=512, n_extra_global=2,
+                alpha_first=0.2, alpha_last=0.6, seed=6),
 ]
 
 

@@ -290,16 +290,13 @@ __global__ void __launch_bounds__(kTailThreads, 1)
             if (!(ok = ready())) break;
             issue_pv(0, false);
           } else {
-            if (!(ok = region())) break;   // pass 1, key half 0
-            issue_s(qt, 0);
-            if (!(ok = region())) break;   // pass 1, key half 1
-            issue_s(qt, 1);
-            if (!(ok = region())) break;   // pass 2, key half 0
+            if (!(ok = region())) break;
             issue_s(qt, 0);
             if (!(ok = ready())) break;
             issue_pv(0, false);
-            // key half 1 has at most 128 columns: S lands beside O, and after
-            // P V of half 0 in issue order, so it may be issued at once
+            // key half 1 has at most 128 columns: its S lands on P of half 0
+            // (not on O) after that half's P V in issue order, so it may be
+            // issued at once
             issue_s(qt, 1);
             if (!(ok = ready())) break;
             issue_pv(1, true);
@@ -394,30 +391,48 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         if (qt >= nq) break;
         const int i = kTile * qt + r;
         const Partners me = partners_of(i);
-        float mx = -INFINITY;
         if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
         tc_fence_after();
-        mx = half_max(me, 0, mx);
-        if (nkh == 2) {
-          release();
-          if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
-          tc_fence_after();
-          mx = half_max(me, 1, mx);
-          release();
-          if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
-          tc_fence_after();
-        }
-        const float nmc = me.valid ? -mx * kLogitScale2 : 0.f;
-        float lsum = half_exp(me, 0, nmc);
+        // half 0: P = exp2(S - max of half 0), exact when there is one half
+        const float m0 = half_max(me, 0, -INFINITY);
+        const float nmc0 = (me.valid && m0 != -INFINITY) ? -m0 * kLogitScale2 : 0.f;
+        float nmc = nmc0;
+        float lsum = half_exp(me, 0, nmc0);
         tc_fence_before();
         warp_arrive(&sm.bar_pready[X]);
         if (nkh == 2) {
+          // half 1 (at most 128 keys; its S lands on P of half 0 after that
+          // half's P V, so O of half 0 is complete once S is): the reference
+          // rises to its maximum when that exceeds the reference by more than
+          // 8 (base 2, P below 2^8 otherwise), and O and the row sum are
+          // rescaled exactly
           if (!(ok = tail_wait(&sm.bar_sfull[X], (n_sfull++) & 1, abort_flag))) break;
+          if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
           tc_fence_after();
+          const float m1 = half_max(me, 1, -INFINITY);
+          const bool raise = me.valid && m1 != -INFINITY &&
+                             (m0 == -INFINITY || (m1 - m0) * kLogitScale2 > 8.f);
+          float f = 1.f;
+          if (raise) {
+            f = m0 == -INFINITY ? 0.f : ex2((m0 - m1) * kLogitScale2);
+            nmc = -m1 * kLogitScale2;
+            lsum *= f;
+          }
+          if (__any_sync(0xffffffffu, raise)) {
+#pragma unroll 1
+            for (int c = 0; c < 64; c += 16) {
+              float o[16];
+              tmem_ld16(tO + c, o);
+              tmem_ld_wait();
+#pragma unroll
+              for (int k = 0; k < 16; ++k) o[k] *= f;
+              tmem_st16(tO + c, reinterpret_cast<const uint32_t*>(o));
+              tmem_st_wait();   // o is reused
+            }
+          }
           lsum += half_exp(me, 1, nmc);
           tc_fence_before();
           warp_arrive(&sm.bar_pready[X]);
-          if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
         }
         if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
         tc_fence_after();

@@ -663,6 +663,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         tmem_ld16(tS + 16, xt);             // S_Gt
         tmem_ld_wait();
       }
+      // S_G and S_Gt are in registers: the S columns take the band pass while
+      // the global keys and queries are evaluated
+      tc_fence_before();
+      warp_arrive(&sm.bar_sfree[X]);
       // far-row column sums of the global keys: rows outside the key's band
       float e16[kMaxGlobal];
 #pragma unroll
@@ -695,9 +699,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
         for (int k = r; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
       }
-      // S_G and S_Gt are read: the S columns take the band pass
-      tc_fence_before();
-      warp_arrive(&sm.bar_sfree[X]);
     }
 
     // Band pass (the column sums of Sec. "Extractor of Attention Scores"):

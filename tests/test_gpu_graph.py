@@ -42,7 +42,7 @@ def _capture(sc, wl, inp):
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.stream(side):
         out = sc.stack_forward(t["Q"], t["K"], t["V"], mask, inp["global_pos"], wl.w, inp["alpha"],
-                               workspace=ws)
+                               workspace=ws, keep_rule=wl.keep_rule)
         torch.cuda.synchronize()
         # eager result of the same call, then clobber the outputs
         eager = _host(out)
@@ -50,7 +50,7 @@ def _capture(sc, wl, inp):
             v.fill_(0 if v.dtype != torch.float32 else float("nan"))
         with torch.cuda.graph(graph, stream=side):
             sc.stack_forward(t["Q"], t["K"], t["V"], mask, inp["global_pos"], wl.w, inp["alpha"],
-                             out=out, workspace=ws)
+                             out=out, workspace=ws, keep_rule=wl.keep_rule)
     torch.cuda.current_stream().wait_stream(side)
     return graph, t, mask, out, ws, eager
 
@@ -72,6 +72,9 @@ CASES = [
     wk.Workload("small_12x700", n_layers=12, B=2, L=700, w=64, n_extra_global=3, seed=3),
     wk.Workload("all_tail_w64", n_layers=4, B=3, L=256, w=64, n_extra_global=4, ragged=(40, 256),
                 seed=11),
+    # the wide rows layout and the top-ratio rule inside the captured loop
+    wk.Workload("wide_top_ratio_768", n_layers=3, B=2, L=768, w=400, n_extra_global=2,
+                alpha_first=0.6, alpha_last=0.5, keep_rule=2, seed=23),
 ]
 
 

@@ -16,6 +16,9 @@ layer_sampled(Q, K, V, is_global, w, rows, cols)
 stack(Q, K, V, pad_mask, global_pos, w, alpha, keep_rule)
                                              the pruned layer stack (bf16 bits in)
 top_count(rho, n), keep_top(scores, k)       the top-ratio keep rule
+
+oracle.encoder: the rest of the encoder layer around the path (projections,
+layer norms, GELU), float64 numpy.
 """
 from __future__ import annotations
 

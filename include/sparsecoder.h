@@ -232,6 +232,104 @@ int sc_stack_launch_count(const sc_stack_args* args, int* count);
  * the status word. */
 int sc_workspace_status(void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * The encoder layer around the path (SURVEY "next": the steps either side of
+ * the attention, Fig. "sparsecoder"): a RoBERTa-style post-LN layer whose
+ * self-attention is the sparse attention with token pruning above, and whose
+ * output projection and feed-forward block run on the kept tokens only.  D = 64 H.
+ *
+ *   Q, K, V = X W_qkv^T + b_qkv            (W_qkv rows: the D outputs of Q, then K, then V)
+ *   O, s, keep = sc_layer_forward(Q, K, V)
+ *   S1 = X[kept] + O[kept] W_o^T + b_o;  H1 = LN1(S1)
+ *   Y  = LN2(H1 + GELU(H1 W_1^T + b_1) W_2^T + b_2)
+ * LN(x) = (x - mean) / sqrt(var + 1e-5) * gamma + beta over the D features
+ * (population variance); GELU(x) = x/2 (1 + erf(x / sqrt 2)).  Stored as bf16:
+ * Q, K, V, O, H1, GELU's output, Y; S1 and the second sum stay fp32.
+ *
+ * X          bf16 [B][L][D] hidden states in current order (row c of sequence b
+ *            is current token c; rows at or beyond len[b] are never read).
+ * len, pos, w, global_pos, n_global, keep_rule, alpha, theta: as sc_layer_args.
+ * W_qkv bf16 [3D][D], b_qkv fp32 [3D]; W_o bf16 [D][D], b_o [D];
+ * ln1_gamma, ln1_beta fp32 [D]; W_1 bf16 [4D][D], b_1 [4D]; W_2 bf16 [D][4D],
+ * b_2 [D]; ln2_gamma, ln2_beta [D].  Weights are [out][in] (row per output).
+ * Y          bf16 [B][L][D] out: the kept tokens' outputs, compacted (row k of
+ *            sequence b is its k-th kept token): the next layer's X, with
+ *            len_out and pos_out as its len and pos.
+ * O          bf16 [B][L][D] out: the attention output of every current token.
+ * scores, pos_out, len_out: as sc_layer_args.
+ * H must be even (D a multiple of 128) and at most 16.
+ */
+typedef struct {
+  int B, L, H, w;
+  const uint16_t* X;
+  const int32_t* len;
+  const int32_t* pos;
+  const int32_t* global_pos;
+  int n_global;
+  int keep_rule;
+  float alpha;
+  const float* theta;
+  const uint16_t* W_qkv;
+  const float* b_qkv;
+  const uint16_t* W_o;
+  const float* b_o;
+  const float* ln1_gamma;
+  const float* ln1_beta;
+  const uint16_t* W_1;
+  const float* b_1;
+  const uint16_t* W_2;
+  const float* b_2;
+  const float* ln2_gamma;
+  const float* ln2_beta;
+  uint16_t* Y;
+  uint16_t* O;
+  float* scores;
+  int32_t* pos_out;
+  int32_t* len_out;
+} sc_encoder_args;
+
+/* Bytes of workspace sc_encoder_layer_forward needs (0 on invalid sizes). */
+size_t sc_encoder_workspace_size(int B, int L, int H);
+
+/* One encoder layer (see sc_encoder_args).  Errors: see sc_status. */
+int sc_encoder_layer_forward(const sc_encoder_args* args, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+/*
+ * The GEMM of the encoder layer on its own: for every sequence b and row
+ * r < rows[b] (rows == NULL: all L rows),
+ *   out[b L + r][n] = act(sum_k A[b L + g(r)][k] W[n][k] + bias[n]) (+ res[...][n])
+ * with g(r) = gidx[b L + r] (gidx == NULL: r), act = GELU when gelu != 0, and
+ * res (bf16, NULL for none) read at row b L + g(r) when res_gathered, else at
+ * b L + r.  A bf16 [B L][K], W bf16 [N][K] ([out][in]), bias fp32 [N] or NULL,
+ * out [B L][N] bf16, or fp32 when out_f32.  N % 128 == 0, K % 64 == 0, K <= 8192;
+ * A and W 16-byte aligned.  `workspace` (>= 256 bytes, 256-byte aligned) holds
+ * the status word read by sc_workspace_status.
+ */
+typedef struct {
+  int B, L, N, K;
+  const uint16_t* A;
+  const int32_t* rows;
+  const int32_t* gidx;
+  const uint16_t* W;
+  const float* bias;
+  int gelu;
+  const uint16_t* res;
+  int res_gathered;
+  void* out;
+  int out_f32;
+} sc_linear_args;
+
+int sc_linear_forward(const sc_linear_args* args, void* workspace, size_t workspace_bytes,
+                      void* stream);
+
+/* Layer norm of the rows (b, r), r < rows[b] (rows == NULL: all): in fp32
+ * [B L][D], out bf16 [B L][D], gamma/beta fp32 [D], eps as given; D % 32 == 0,
+ * D <= 1024. */
+int sc_layer_norm_forward(int B, int L, int D, const int32_t* rows, const float* in,
+                          const float* gamma, const float* beta, float eps, uint16_t* out,
+                          void* stream);
+
 /* Static, human-readable name of a status code. */
 const char* sc_status_string(int status);
 

@@ -54,6 +54,29 @@ class StackArgs(ctypes.Structure):
                 ("keep_rule", ctypes.c_int)]
 
 
+class EncoderArgs(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("L", ctypes.c_int), ("H", ctypes.c_int), ("w", ctypes.c_int),
+                ("X", ctypes.c_void_p), ("len", ctypes.c_void_p), ("pos", ctypes.c_void_p),
+                ("global_pos", ctypes.POINTER(ctypes.c_int32)), ("n_global", ctypes.c_int),
+                ("keep_rule", ctypes.c_int), ("alpha", ctypes.c_float), ("theta", ctypes.c_void_p),
+                ("W_qkv", ctypes.c_void_p), ("b_qkv", ctypes.c_void_p),
+                ("W_o", ctypes.c_void_p), ("b_o", ctypes.c_void_p),
+                ("ln1_gamma", ctypes.c_void_p), ("ln1_beta", ctypes.c_void_p),
+                ("W_1", ctypes.c_void_p), ("b_1", ctypes.c_void_p),
+                ("W_2", ctypes.c_void_p), ("b_2", ctypes.c_void_p),
+                ("ln2_gamma", ctypes.c_void_p), ("ln2_beta", ctypes.c_void_p),
+                ("Y", ctypes.c_void_p), ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
+                ("pos_out", ctypes.c_void_p), ("len_out", ctypes.c_void_p)]
+
+
+class LinearArgs(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("L", ctypes.c_int), ("N", ctypes.c_int), ("K", ctypes.c_int),
+                ("A", ctypes.c_void_p), ("rows", ctypes.c_void_p), ("gidx", ctypes.c_void_p),
+                ("W", ctypes.c_void_p), ("bias", ctypes.c_void_p), ("gelu", ctypes.c_int),
+                ("res", ctypes.c_void_p), ("res_gathered", ctypes.c_int),
+                ("out", ctypes.c_void_p), ("out_f32", ctypes.c_int)]
+
+
 SC_STACK_NO_TAIL = 1
 # keep rules (sc_keep_rule): what a layer's value alpha means
 SC_KEEP_RELATIVE = 0   # theta = alpha / n
@@ -65,7 +88,9 @@ TAIL_MAX_LEN = 384
 
 EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
             "sc_stack_forward_profiled", "sc_stack_launch_count",
-            "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error"]
+            "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error",
+            "sc_encoder_layer_forward", "sc_encoder_workspace_size", "sc_linear_forward",
+            "sc_layer_norm_forward"]
 
 
 def library_path() -> str:
@@ -109,6 +134,17 @@ def load(build_if_missing: bool = False):
         lib.sc_status_string.argtypes = [ctypes.c_int]
         lib.sc_last_error.restype = ctypes.c_char_p
         lib.sc_last_error.argtypes = []
+        lib.sc_encoder_workspace_size.restype = ctypes.c_size_t
+        lib.sc_encoder_workspace_size.argtypes = [ctypes.c_int] * 3
+        lib.sc_encoder_layer_forward.restype = ctypes.c_int
+        lib.sc_encoder_layer_forward.argtypes = [ctypes.POINTER(EncoderArgs), ctypes.c_void_p,
+                                                 ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_linear_forward.restype = ctypes.c_int
+        lib.sc_linear_forward.argtypes = [ctypes.POINTER(LinearArgs), ctypes.c_void_p,
+                                          ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_layer_norm_forward.restype = ctypes.c_int
+        lib.sc_layer_norm_forward.argtypes = [ctypes.c_int] * 3 + [ctypes.c_void_p] * 4 + [
+            ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p]
         _lib = lib
         return lib
 
@@ -246,3 +282,75 @@ def workspace_status(workspace, stream=None) -> int:
     """Synchronise and return (then clear) the workspace status code."""
     return int(load().sc_workspace_status(_ptr(workspace), workspace.numel(),
                                           _stream_handle(stream)))
+
+
+# ---------------------------------------------------------------------------
+# the encoder layer around the path
+# ---------------------------------------------------------------------------
+ENCODER_WEIGHTS = ("W_qkv", "b_qkv", "W_o", "b_o", "ln1_gamma", "ln1_beta", "W_1", "b_1",
+                   "W_2", "b_2", "ln2_gamma", "ln2_beta")
+
+
+def encoder_workspace_size(B, L, H) -> int:
+    return int(load().sc_encoder_workspace_size(int(B), int(L), int(H)))
+
+
+def new_encoder_workspace(B, L, H, device=None):
+    n = encoder_workspace_size(B, L, H)
+    if n == 0:
+        raise SparseCoderError(SC_ERR_INVALID_ARG, "invalid encoder sizes")
+    ws = torch.zeros(n + 256, dtype=torch.uint8, device=device or "cuda")
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + n]
+
+
+def encoder_layer_forward(X, length, pos, w, global_pos, weights, alpha=0.0, theta=None, *,
+                          keep_rule=SC_KEEP_RELATIVE, out=None, workspace=None, stream=None):
+    """One encoder layer (``sc_encoder_layer_forward``): X bf16 [B, L, D] current order,
+    length int32 [B], pos int32 [B, L]; ``weights`` maps ENCODER_WEIGHTS to cuda tensors
+    (bf16 matrices [out, in], fp32 vectors).  Returns dict(Y, O, scores, pos_out, len_out)."""
+    B, L, D = X.shape
+    H = D // 64
+    dev = X.device
+    if out is None:
+        out = {"Y": torch.empty((B, L, D), dtype=torch.bfloat16, device=dev),
+               "O": torch.empty((B, L, D), dtype=torch.bfloat16, device=dev),
+               "scores": torch.empty((B, L), dtype=torch.float32, device=dev),
+               "pos_out": torch.empty((B, L), dtype=torch.int32, device=dev),
+               "len_out": torch.empty((B,), dtype=torch.int32, device=dev)}
+    ws = workspace if workspace is not None else new_encoder_workspace(B, L, H, dev)
+    garr, ng = _int32_host(global_pos)
+    a = EncoderArgs(B, L, H, int(w), _ptr(X), _ptr(length), _ptr(pos),
+                    ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, int(keep_rule),
+                    float(alpha), _ptr(theta), *[_ptr(weights[k]) for k in ENCODER_WEIGHTS],
+                    _ptr(out["Y"]), _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos_out"]),
+                    _ptr(out["len_out"]))
+    _check(load().sc_encoder_layer_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
+                                           _stream_handle(stream)))
+    return out
+
+
+def linear_forward(A, W, *, B, L, rows=None, gidx=None, bias=None, gelu=False, res=None,
+                   res_gathered=False, out=None, out_f32=False, workspace=None, stream=None):
+    """``sc_linear_forward``: A bf16 [B*L, K] (any leading shape), W bf16 [N, K]."""
+    N, K = W.shape
+    if out is None:
+        out = torch.empty((B * L, N), dtype=torch.float32 if out_f32 else torch.bfloat16,
+                          device=A.device)
+    ws = workspace if workspace is not None else new_workspace(1, 1, 1, A.device)
+    a = LinearArgs(int(B), int(L), int(N), int(K), _ptr(A), _ptr(rows), _ptr(gidx), _ptr(W),
+                   _ptr(bias), int(bool(gelu)), _ptr(res), int(bool(res_gathered)), _ptr(out),
+                   int(bool(out_f32)))
+    _check(load().sc_linear_forward(ctypes.byref(a), _ptr(ws), ws.numel(), _stream_handle(stream)))
+    return out
+
+
+def layer_norm_forward(x, gamma, beta, *, B, L, rows=None, eps=1e-5, out=None, stream=None):
+    """``sc_layer_norm_forward``: x fp32 [B*L, D] -> bf16."""
+    D = x.shape[-1]
+    if out is None:
+        out = torch.empty((B * L, D), dtype=torch.bfloat16, device=x.device)
+    _check(load().sc_layer_norm_forward(int(B), int(L), int(D), _ptr(rows), _ptr(x), _ptr(gamma),
+                                        _ptr(beta), ctypes.c_float(eps), _ptr(out),
+                                        _stream_handle(stream)))
+    return out

@@ -25,6 +25,9 @@ cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st);
 cudaError_t configure_tail();
 cudaError_t tail_max_clusters(int H, int* out);
 cudaError_t launch_tail(const TailParams& p, cudaStream_t st);
+cudaError_t configure_encoder();
+cudaError_t launch_gemm(const GemmParams& p, cudaStream_t st);
+cudaError_t launch_layernorm(const LayerNormParams& p, cudaStream_t st);
 }  // namespace sc
 
 namespace {
@@ -142,6 +145,26 @@ bool encode_rows(CUtensorMap* m, const void* base, long long rows) {
   return r == CUDA_SUCCESS;
 }
 
+// Plain 2-D view [rows][cols] of a bf16 matrix (row stride cols), 128-byte
+// swizzle; one TMA box is 64 columns x box_rows rows.
+bool encode_2d(CUtensorMap* m, const void* base, long long rows, int cols, int box_rows) {
+  auto enc = get_encoder();
+  if (!enc) return fail(SC_ERR_CUDA, "tensor-map encoder", "cuTensorMapEncodeTiled unavailable"), false;
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t gstride[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estride[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), gdim, gstride,
+                   box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char d[64];
+    snprintf(d, sizeof d, "CUresult %d", static_cast<int>(r));
+    fail(SC_ERR_CUDA, "encode 2-D matrix map", d);
+  }
+  return r == CUDA_SUCCESS;
+}
+
 // Descriptors for the caller's Q, K, V (source 0, `tokens` tokens) and the
 // compacted copies in the workspace (source 1, B * L tokens).
 bool encode_maps(TensorMaps* m, const uint16_t* const src[3], long long tokens, uint16_t* const cmp[3],
@@ -169,6 +192,7 @@ int ensure_configured() {
   if (!done[dev]) {
     cudaError_t e = configure_kernels();
     if (e == cudaSuccess) e = configure_tail();
+    if (e == cudaSuccess) e = configure_encoder();
     if (e != cudaSuccess) return fail_cuda("kernel attributes", e);
     done[dev] = true;
   }
@@ -315,7 +339,20 @@ const char* sc_status_string(int status) {
   }
 }
 
+namespace {
+int layer_forward_impl(const sc_layer_args* a, void* workspace, size_t ws_bytes, void* stream,
+                       int32_t* kept_cur);
+}  // namespace
+
 int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, void* stream) {
+  return layer_forward_impl(a, workspace, ws_bytes, stream, nullptr);
+}
+
+namespace {
+// One layer; kept_cur (device [B][L] or nullptr) receives the current index of
+// each kept token, in order.
+int layer_forward_impl(const sc_layer_args* a, void* workspace, size_t ws_bytes, void* stream,
+                       int32_t* kept_cur) {
   if (!a) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
@@ -356,6 +393,7 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   p.theta = a->theta;
   p.keep_rule = a->keep_rule;
   fill_workspace(&p, ws, lay, 0);
+  p.kept_cur = kept_cur;
 
   PrepParams pp{};
   pp.B = a->B; pp.L = a->L;
@@ -372,6 +410,7 @@ int sc_layer_forward(const sc_layer_args* a, void* workspace, size_t ws_bytes, v
   if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
   return SC_OK;
 }
+}  // namespace
 
 // Which kernels a stack call launches: sequences with at most kTailMax tokens
 // left finish in the cluster kernel (when it can run with clusters of H CTAs);
@@ -776,5 +815,173 @@ extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
   if ((e = launch_prep(pp, st)) != cudaSuccess) return fail_cuda("launch prep kernel", e);
   if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
   if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
+  return SC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// the encoder layer around the path: GEMMs, layer norms, the layer driver
+// ---------------------------------------------------------------------------
+namespace {
+
+bool aligned_ptr16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Fills the GEMM parameters and descriptors for out = act(A[gather] W^T + b) (+ res).
+int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, const int32_t* rows,
+              const int32_t* gidx, const uint16_t* W, const float* bias, int gelu,
+              const uint16_t* res, int res_gathered, void* out, int out_f32, int* status) {
+  *g = GemmParams{};
+  if (!encode_2d(&g->map_a, A, static_cast<long long>(B) * L, K, 1) ||
+      !encode_2d(&g->map_w, W, N, K, kTile))
+    return SC_ERR_CUDA;
+  g->B = B; g->L = L; g->N = N; g->K = K;
+  g->rows = rows; g->gidx = gidx; g->bias = bias; g->gelu = gelu;
+  g->res = res; g->res_gathered = res_gathered;
+  g->out = out; g->out_f32 = out_f32; g->out_split = 0;
+  g->status = status;
+  return SC_OK;
+}
+
+struct EncLayout {
+  size_t attn, qkv, kept, s, h1, f, total;
+};
+
+bool enc_layout(int B, int L, int H, EncLayout* e) {
+  WsLayout lay;
+  if (!ws_layout(B, L, H, &lay)) return false;
+  const size_t rows = static_cast<size_t>(B) * L, D = static_cast<size_t>(H) * kHeadDim;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes);
+    return at;
+  };
+  e->attn = take(lay.total);
+  e->qkv = take(3 * rows * D * sizeof(uint16_t));
+  e->kept = take(rows * sizeof(int32_t));
+  e->s = take(rows * D * sizeof(float));
+  e->h1 = take(rows * D * sizeof(uint16_t));
+  e->f = take(rows * 4 * D * sizeof(uint16_t));
+  e->total = off;
+  return true;
+}
+
+}  // namespace
+
+extern "C" size_t sc_encoder_workspace_size(int B, int L, int H) {
+  if (B < 1 || L < 1 || H < 2 || (H & 1) || H > kTailMaxHeads || L > kMaxLen) return 0;
+  EncLayout e;
+  return enc_layout(B, L, H, &e) ? e.total : 0;
+}
+
+extern "C" int sc_linear_forward(const sc_linear_args* a, void* workspace, size_t ws_bytes,
+                                 void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  if (a->B < 1 || a->L < 1 || a->N < kTile || a->N % kTile || a->K < 64 || a->K % 64 ||
+      a->K > 8192 || static_cast<long long>(a->B) * a->L > (1ll << 31) - 1)
+    return SC_ERR_INVALID_ARG;
+  if (!a->A || !a->W || !a->out || !aligned_ptr16(a->A) || !aligned_ptr16(a->W) ||
+      !aligned_ptr16(a->out) || (a->res && !aligned_ptr16(a->res)))
+    return SC_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < kAlign || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
+    return SC_ERR_WORKSPACE;
+  int rc = ensure_configured();
+  if (rc != SC_OK) return rc;
+  GemmParams g;
+  if ((rc = make_gemm(&g, a->B, a->L, a->N, a->K, a->A, a->rows, a->gidx, a->W, a->bias, a->gelu,
+                      a->res, a->res_gathered, a->out, a->out_f32,
+                      static_cast<int*>(workspace))) != SC_OK)
+    return rc;
+  const cudaError_t e = launch_gemm(g, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? SC_OK : fail_cuda("launch gemm kernel", e);
+}
+
+extern "C" int sc_layer_norm_forward(int B, int L, int D, const int32_t* rows, const float* in,
+                                     const float* gamma, const float* beta, float eps,
+                                     uint16_t* out, void* stream) {
+  if (B < 1 || L < 1 || D < 32 || D % 32 || D > 1024 || !in || !gamma || !beta || !out ||
+      !(eps > 0.f))
+    return SC_ERR_INVALID_ARG;
+  int rc = ensure_configured();
+  if (rc != SC_OK) return rc;
+  LayerNormParams q{B, L, D, rows, in, gamma, beta, eps, out};
+  const cudaError_t e = launch_layernorm(q, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? SC_OK : fail_cuda("launch layer-norm kernel", e);
+}
+
+extern "C" int sc_encoder_layer_forward(const sc_encoder_args* a, void* workspace, size_t ws_bytes,
+                                        void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  if (a->H < 2 || (a->H & 1) || a->H > kTailMaxHeads) return SC_ERR_UNSUPPORTED;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if ((rc = check_keep(a->keep_rule, &a->alpha, 1, a->theta)) != SC_OK) return rc;
+  const void* need[] = {a->X, a->len, a->pos, a->W_qkv, a->b_qkv, a->W_o, a->b_o, a->ln1_gamma,
+                        a->ln1_beta, a->W_1, a->b_1, a->W_2, a->b_2, a->ln2_gamma, a->ln2_beta,
+                        a->Y, a->O, a->scores, a->pos_out, a->len_out};
+  for (const void* q : need)
+    if (!q) return SC_ERR_INVALID_ARG;
+  const void* al[] = {a->X, a->W_qkv, a->W_o, a->W_1, a->W_2, a->Y, a->O};
+  for (const void* q : al)
+    if (!aligned_ptr16(q)) return SC_ERR_INVALID_ARG;
+  if (a->pos_out == a->pos || a->len_out == a->len) return SC_ERR_INVALID_ARG;
+  EncLayout el;
+  if (!enc_layout(a->B, a->L, a->H, &el)) return SC_ERR_UNSUPPORTED;
+  if (!workspace || ws_bytes < el.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
+    return SC_ERR_WORKSPACE;
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char* ws = static_cast<char*>(workspace);
+  const int B = a->B, L = a->L, D = a->H * kHeadDim;
+  const size_t rows = static_cast<size_t>(B) * L;
+  uint16_t* qkv = reinterpret_cast<uint16_t*>(ws + el.qkv);
+  uint16_t* Qb = qkv;
+  uint16_t* Kb = qkv + rows * D;
+  uint16_t* Vb = qkv + 2 * rows * D;
+  int32_t* kept = reinterpret_cast<int32_t*>(ws + el.kept);
+  float* S = reinterpret_cast<float*>(ws + el.s);
+  uint16_t* H1 = reinterpret_cast<uint16_t*>(ws + el.h1);
+  uint16_t* F = reinterpret_cast<uint16_t*>(ws + el.f);
+  int* status = reinterpret_cast<int*>(ws + el.attn);   // the attention workspace's status word
+  cudaError_t e;
+
+  // Q, K, V of the current tokens: one GEMM, its column blocks split by tensor
+  GemmParams g;
+  if ((rc = make_gemm(&g, B, L, 3 * D, D, a->X, a->len, nullptr, a->W_qkv, a->b_qkv, 0, nullptr, 0,
+                      nullptr, 0, status)) != SC_OK)
+    return rc;
+  g.out_split = D;
+  g.outs[0] = Qb; g.outs[1] = Kb; g.outs[2] = Vb;
+  if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch QKV gemm", e);
+
+  // sparse attention with token pruning; the kept tokens' current indices
+  sc_layer_args la{};
+  la.B = B; la.L = L; la.H = a->H; la.w = a->w;
+  la.Q = Qb; la.K = Kb; la.V = Vb;
+  la.len = a->len; la.pos = a->pos;
+  la.global_pos = a->global_pos; la.n_global = a->n_global;
+  la.alpha = a->alpha; la.theta = a->theta; la.keep_rule = a->keep_rule;
+  la.O = a->O; la.scores = a->scores; la.pos_out = a->pos_out; la.len_out = a->len_out;
+  WsLayout lay;
+  ws_layout(B, L, a->H, &lay);
+  if ((rc = layer_forward_impl(&la, ws + el.attn, lay.total, stream, kept)) != SC_OK) return rc;
+
+  // S1 = X[kept] + O[kept] W_o^T + b_o (the compaction is this GEMM's row gather)
+  if ((rc = make_gemm(&g, B, L, D, D, a->O, a->len_out, kept, a->W_o, a->b_o, 0, a->X, 1, S, 1,
+                      status)) != SC_OK)
+    return rc;
+  if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch output gemm", e);
+  LayerNormParams ln{B, L, D, a->len_out, S, a->ln1_gamma, a->ln1_beta, 1e-5f, H1};
+  if ((e = launch_layernorm(ln, st)) != cudaSuccess) return fail_cuda("launch layer norm 1", e);
+  // the feed-forward block on the kept tokens
+  if ((rc = make_gemm(&g, B, L, 4 * D, D, H1, a->len_out, nullptr, a->W_1, a->b_1, 1, nullptr, 0, F,
+                      0, status)) != SC_OK)
+    return rc;
+  if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch ffn gemm 1", e);
+  if ((rc = make_gemm(&g, B, L, D, 4 * D, F, a->len_out, nullptr, a->W_2, a->b_2, 0, H1, 0, S, 1,
+                      status)) != SC_OK)
+    return rc;
+  if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch ffn gemm 2", e);
+  ln.gamma = a->ln2_gamma; ln.beta = a->ln2_beta; ln.out = a->Y;
+  if ((e = launch_layernorm(ln, st)) != cudaSuccess) return fail_cuda("launch layer norm 2", e);
   return SC_OK;
 }

@@ -84,6 +84,7 @@ struct LayerParams {
   uint32_t* cnt_tile;    // [B][T]
   uint32_t* cnt_seq;     // [B]
   uint32_t* rows_done;   // [B][H]: rows CTAs of (sequence, head) whose results are visible
+  int32_t* kept_cur;     // [B][L] out, or nullptr: current index of each kept token, in order
   int* status;
   // hand-over to the cluster kernel: sequence b is skipped here once
   // tail_from[b] <= layer; the finalize of a layer sets tail_from[b] = layer + 1
@@ -185,6 +186,38 @@ struct TailParams {
   int global_pos[kMaxGlobal];
   float alpha[kTailMaxLayers];   // the keep rule's value per layer
   int keep_rule;
+};
+
+// One GEMM of the encoder layer: out[(b, r)][n] = epi(sum_k A[row_a][k] W[n][k])
+// for r < rows[b], row_a = b L + (gidx ? gidx[b L + r] : r); epi adds bias[n],
+// then GELU (gelu != 0), then the bf16 residual res[row][n] (row = row_a when
+// res_gathered, else b L + r).  N % 128 == 0, K % 64 == 0.
+struct GemmParams {
+  CUtensorMap map_a;               // 2-D [B L][K] bf16, box 64 x 1 (four-row gathers)
+  CUtensorMap map_w;               // 2-D [N][K] bf16, box 64 x 128
+  int B, L, N, K;
+  const int32_t* rows;             // [B] rows per sequence, or nullptr (L)
+  const int32_t* gidx;             // [B][L] A row of output row (b, r), or nullptr
+  const float* bias;               // [N] or nullptr
+  int gelu;
+  const uint16_t* res;             // bf16 [B L][N] or nullptr
+  int res_gathered;
+  void* out;                       // [B L][N], bf16 or fp32 (out_f32)
+  int out_f32;
+  int out_split;                   // > 0: column block j of width out_split goes to outs[j]
+  void* outs[3];
+  int* status;
+};
+
+// Layer norm over D features of the rows (b, r), r < rows[b]: fp32 in, bf16 out.
+struct LayerNormParams {
+  int B, L, D;
+  const int32_t* rows;
+  const float* in;
+  const float* gamma;
+  const float* beta;
+  float eps;
+  uint16_t* out;
 };
 
 }  // namespace sc

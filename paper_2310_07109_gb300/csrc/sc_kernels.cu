@@ -1245,6 +1245,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     if (!kf[r]) continue;
     const int out = sm.kpre[r][warp] + __popc(sm.kbits[r][warp] & below);
     pos_out[out] = ps[r];
+    if (p.kept_cur) p.kept_cur[static_cast<size_t>(b) * p.L + out] = r * kColsThreads + tid;
     if (out == sm.total - 1) sm.last_pos = ps[r];
   }
   // next-layer index of each surviving global token

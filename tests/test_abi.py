@@ -153,3 +153,28 @@ def test_launch_count_rejects_bad_arguments(lib):
     assert count(L=8192) == bd.SC_ERR_UNSUPPORTED
     assert count(B=0) == bd.SC_ERR_INVALID_ARG
     assert lib.sc_stack_launch_count(None, None) == bd.SC_ERR_INVALID_ARG
+
+
+def test_encoder_calls_reject_bad_arguments(lib):
+    assert lib.sc_encoder_layer_forward(None, None, 0, None) == bd.SC_ERR_INVALID_ARG
+    a = bd.EncoderArgs()
+    a.B, a.L, a.H, a.w = 1, 256, 11, 64          # odd head count: D not a multiple of 128
+    assert lib.sc_encoder_layer_forward(ctypes.byref(a), ctypes.c_void_p(FAKE), 1 << 30,
+                                        None) == bd.SC_ERR_UNSUPPORTED
+    a.H = 12                                     # null pointers
+    assert lib.sc_encoder_layer_forward(ctypes.byref(a), ctypes.c_void_p(FAKE), 1 << 30,
+                                        None) == bd.SC_ERR_INVALID_ARG
+    assert bd.encoder_workspace_size(2, 1024, 12) > bd.workspace_size(2, 1024, 12)
+    assert bd.encoder_workspace_size(2, 1024, 11) == 0
+    lin = bd.LinearArgs(1, 128, 100, 64, FAKE, None, None, FAKE, None, 0, None, 0, FAKE, 0)
+    assert lib.sc_linear_forward(ctypes.byref(lin), ctypes.c_void_p(FAKE), 256,
+                                 None) == bd.SC_ERR_INVALID_ARG   # N not a multiple of 128
+    lin.N, lin.K = 128, 96
+    assert lib.sc_linear_forward(ctypes.byref(lin), ctypes.c_void_p(FAKE), 256,
+                                 None) == bd.SC_ERR_INVALID_ARG   # K not a multiple of 64
+    lin.K = 64
+    assert lib.sc_linear_forward(ctypes.byref(lin), ctypes.c_void_p(FAKE), 16,
+                                 None) == bd.SC_ERR_WORKSPACE
+    assert lib.sc_layer_norm_forward(1, 1, 100, None, ctypes.c_void_p(FAKE), ctypes.c_void_p(FAKE),
+                                     ctypes.c_void_p(FAKE), ctypes.c_float(1e-5),
+                                     ctypes.c_void_p(FAKE), None) == bd.SC_ERR_INVALID_ARG

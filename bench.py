@@ -4,12 +4,16 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
                     [--workload cfg4|cfg2|cfg3|cfg5_L512|...|cfg5_L4096[_theta0]
-                                |abs_theta|top_ratio|window_w16|...|window_w256]
+                                |abs_theta|top_ratio|window_w16|...|window_w512
+                                |encoder_cfg2]
 
 Besides the default, the workloads cover the other keep rules (abs_theta: the
 absolute per-layer thresholds 0.01 l / 12 of RQ4; top_ratio: a kept ratio per
 layer, 0.95 -> 0.8) and the window-size ablation of RQ3 (window_wNN: sparse
-attention alone, nothing pruned, L = 1024, B = 8); each prints its own line.
+attention alone, nothing pruned, L = 1024, B = 8); encoder_cfg2 times 12 whole
+encoder layers around the path (projections, attention with pruning, layer
+norms, feed-forward on the kept tokens; random-init weights) on the config-2
+shape.  Each prints its own line.
 
 One step = one call of sc_stack_forward over the whole workload: padding removal,
 then per layer the rows kernel (band + global attention, O, row LSE) and the
@@ -66,6 +70,8 @@ def pick_workload(name: str) -> wk.Workload:
         rest = name[len("cfg5_L"):]
         control = rest.endswith("_theta0")
         return wk.cfg5(int(rest.replace("_theta0", "")), control=control)
+    if name == "encoder_cfg2":
+        return wk.ENCODER_CFG2
     if name == "abs_theta":
         return wk.ABS_THETA
     if name == "top_ratio":
@@ -584,6 +590,206 @@ def run_native(args, wl):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------
+# the encoder layer around the path (--workload encoder_cfg2)
+# ---------------------------------------------------------------------------
+def encoder_oracle_sample(wl, X0, weights, b, threads):
+    """The oracle on sequence b for layer 0 of the encoder: (seconds, tokens, cores)."""
+    import oracle
+    from oracle import encoder as enc
+    D = wl.H * wl.d
+    w = {k: (wk.bf16_bits_to_f64(v) if k.startswith("W") else v.astype(np.float64))
+         for k, v in weights[0].items()}
+    x = wk.bf16_bits_to_f64(X0[b])
+    t0 = time.perf_counter()
+    q, k, v = enc.qkv(x, w["W_qkv"], w["b_qkv"])
+    n = x.shape[0]
+    gset = set(int(g) for g in wk.global_positions(wl))
+    isg = np.array([c in gset for c in range(n)])
+    O, s, keep = oracle.layer(q.reshape(n, wl.H, wl.d), k.reshape(n, wl.H, wl.d),
+                              v.reshape(n, wl.H, wl.d), isg, wl.w, wl.alphas()[0] / n,
+                              nthreads=threads)
+    kc = np.nonzero(keep)[0]
+    enc.output_and_ffn(x[kc], O.reshape(n, D)[kc], w["W_o"], w["b_o"], w["ln1_gamma"],
+                       w["ln1_beta"], w["W_1"], w["b_1"], w["W_2"], w["b_2"], w["ln2_gamma"],
+                       w["ln2_beta"])
+    return time.perf_counter() - t0, n, min(threads, wl.H)
+
+
+def run_reference_encoder(args, wl):
+    import oracle
+    oracle.build()
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    D = wl.H * wl.d
+    X0 = wk.encoder_input(wl)
+    wts = [wk.encoder_weights(D, 0, wl.seed)]
+    threads = oracle.default_threads()
+    for s in range(args.warmup):
+        encoder_oracle_sample(wl, X0, wts, s % wl.B, threads)
+    tot_t, tot_tok, cores = 0.0, 0, 1
+    for s in range(args.steps):
+        dt, tok, cores = encoder_oracle_sample(wl, X0, wts, s % wl.B, threads)
+        tot_t += dt
+        tot_tok += tok
+    value = tot_tok / tot_t
+    sample = "one sequence of the workload, encoder layer 0, per step"
+    print(json.dumps({"impl": "reference", "metric": "kept-tokens/sec per %d-layer pruned encoder "
+                      "at L=%d" % (wl.n_layers, wl.L), "value": value, "unit": UNIT,
+                      "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                      "ms_per_step": 1e3 * tot_t / args.steps, "higher_is_better": True,
+                      "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                      "config": {"workload": wl.describe(), "sample": sample},
+                      "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores,
+                                       "kind": "oracle", "sample": sample},
+                      "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                              "d2h_bytes_per_step": 0}}), flush=True)
+
+
+def run_encoder(args, wl):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2310_07109_gb300 import binding as sc
+    from paper_2310_07109_gb300 import build as sc_build
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    sc_build.build_library()
+    sc.load()
+    D = wl.H * wl.d
+    nl = wl.n_layers
+    X0 = wk.encoder_input(wl)
+    wts = [wk.encoder_weights(D, l, wl.seed) for l in range(nl)]
+    W = [{k: (torch.from_numpy(v.view(np.int16)).to(dev).view(torch.bfloat16) if k.startswith("W")
+              else torch.from_numpy(v).to(dev)) for k, v in wl_w.items()} for wl_w in wts]
+    hostX = torch.from_numpy(X0.view(np.int16)).view(torch.bfloat16).pin_memory()
+    X = hostX.to(dev)
+    len0 = torch.full((wl.B,), wl.L, dtype=torch.int32, device=dev)
+    pos0 = torch.arange(wl.L, dtype=torch.int32, device=dev).repeat(wl.B, 1)
+    gpos = [int(g) for g in wk.global_positions(wl)]
+    alpha = [float(a) for a in wl.alphas()]
+    ws = sc.new_encoder_workspace(wl.B, wl.L, wl.H, dev)
+    outs = [{"Y": torch.empty((wl.B, wl.L, D), dtype=torch.bfloat16, device=dev),
+             "O": torch.empty((wl.B, wl.L, D), dtype=torch.bfloat16, device=dev),
+             "scores": torch.empty((wl.B, wl.L), dtype=torch.float32, device=dev),
+             "pos_out": torch.empty((wl.B, wl.L), dtype=torch.int32, device=dev),
+             "len_out": torch.empty((wl.B,), dtype=torch.int32, device=dev)} for _ in range(nl)]
+
+    def step():
+        x, ln, ps = X, len0, pos0
+        for l in range(nl):
+            o = outs[l]
+            sc.encoder_layer_forward(x, ln, ps, wl.w, gpos, W[l], alpha[l], keep_rule=wl.keep_rule,
+                                     out=o, workspace=ws)
+            x, ln, ps = o["Y"], o["len_out"], o["pos_out"]
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    rc = sc.workspace_status(ws)
+    if rc != 0:
+        raise SystemExit("device status after warm-up: %s" % sc.status_string(rc))
+    graph = None
+    if not args.no_graph:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            step()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=side):
+                step()
+        torch.cuda.current_stream().wait_stream(side)
+        for _ in range(max(3, args.warmup)):
+            graph.replay()
+        torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device()) as clocks:
+        time.sleep(0.01)
+        barrier()
+        clocks.mark_start()
+        t0.record(stream)
+        for _ in range(args.steps):
+            if graph is not None:
+                graph.replay()
+            else:
+                step()
+        t1.record(stream)
+        barrier()
+        clocks.mark_end()
+    rc = sc.workspace_status(ws)
+    if rc != 0:
+        raise SystemExit("device status after the timed steps: %s" % sc.status_string(rc))
+    ms_per_step = max_over_ranks(t0.elapsed_time(t1), dev) / args.steps
+    lens = np.stack([np.full(wl.B, wl.L)] + [o["len_out"].cpu().numpy() for o in outs]).astype(np.int64)
+    kept_per_step = int(lens[:nl].sum())
+    value = whole_job_rate(world, kept_per_step, ms_per_step)
+    # algorithmic work: the GEMMs (Q/K/V on the current tokens, the rest on the
+    # kept ones) and the attention's QK^T and PV over the allowed pairs
+    pos = np.stack([np.tile(np.arange(wl.L), (wl.B, 1))] +
+                   [o["pos_out"].cpu().numpy() for o in outs])
+    work = layer_work(wl, {"global_pos": np.asarray(gpos)}, pos, lens)
+    gemm_flops = sum(2 * D * D * (3 * int(lens[l].sum()) + 9 * int(lens[l + 1].sum()))
+                     for l in range(nl))
+    flops = gemm_flops + sum(F for _, F in work)
+    peaks, peak_src = load_peaks()
+    t = ms_per_step * 1e-3
+    roofline = {"bound": "tensor", "achieved": flops / t / 1e12, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": flops / t / 1e12 / peaks["bf16_tflops"], "traffic": None,
+                "peak_source": peak_src,
+                "kernel": "the whole encoder step (GEMMs, attention, layer norms)",
+                "algorithmic": {"flops": int(flops), "gemm_flops": int(gemm_flops),
+                                "per_unit": "2 D^2 (3 n + 9 n') per layer (projections on the n "
+                                            "current tokens, the rest on the n' kept ones) + "
+                                            "3072 flop per allowed pair"}}
+    # end to end: layer-0 hidden states in from pinned memory, the last layer's out
+    hostY = torch.empty(outs[-1]["Y"].shape, dtype=torch.bfloat16, pin_memory=True)
+    e2e_steps = max(1, min(args.steps, 5))
+    barrier()
+    t0.record(stream)
+    for _ in range(e2e_steps):
+        X.copy_(hostX, non_blocking=True)
+        step()
+        hostY.copy_(outs[-1]["Y"], non_blocking=True)
+    t1.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(t0.elapsed_time(t1) / e2e_steps, dev)
+    line = {"metric": "kept-tokens/sec per %d-layer pruned encoder at L=%d" % (nl, wl.L),
+            "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic inputs, random-init weights",
+            "config": {"workload": wl.describe() + "; encoder layers (D=%d, FFN %d)" % (D, 4 * D),
+                       "n_layers": nl, "batch": wl.B, "seq_len": wl.L, "cuda_graph": graph is not None,
+                       "kept_tokens_per_step": kept_per_step,
+                       "survival": [round(float(x), 4) for x in lens.sum(axis=1) / lens[0].sum()]},
+            "roofline": roofline,
+            "e2e": {"value": whole_job_rate(world, kept_per_step, e2e_ms), "unit": UNIT,
+                    "h2d_bytes_per_step": int(hostX.numel() * 2),
+                    "d2h_bytes_per_step": int(hostY.numel() * 2), "ms_per_step": e2e_ms},
+            "gpu_launches": args.steps * nl * 9, "clocks": clocks.summary()}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        dt, tok, cores = encoder_oracle_sample(wl, X0, wts, 0, oracle.default_threads())
+        line["cpu_baseline"] = {"value": tok / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": "sequence 0, layer 0 (%d tokens, %.1f s)" % (tok, dt)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -599,10 +805,11 @@ def main():
                          "a captured CUDA graph")
     args = ap.parse_args()
     wl = pick_workload(args.workload)
+    encoder = args.workload.startswith("encoder")
     if args.impl == "reference":
-        run_reference(args, wl)
+        (run_reference_encoder if encoder else run_reference)(args, wl)
     else:
-        run_native(args, wl)
+        (run_encoder if encoder else run_native)(args, wl)
 
 
 if __name__ == "__main__":

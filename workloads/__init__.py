@@ -31,6 +31,8 @@ _TAG_SALIENT = 12
 _TAG_GLOBAL = 13
 _TAG_LENGTH = 14
 _TAG_REDRAW = 15
+_TAG_WEIGHTS = 16
+_TAG_HIDDEN = 17
 
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -215,3 +217,30 @@ def random_layer(n: int, H: int, d: int, seed: int, scale_k: float = 1.0):
     k = g.standard_normal((n, H, d), dtype=np.float32) * np.float32(scale_k)
     v = g.standard_normal((n, H, d), dtype=np.float32)
     return f32_to_bf16_bits(q), f32_to_bf16_bits(k), f32_to_bf16_bits(v)
+
+
+# ---------------------------------------------------------------------------
+# the encoder layer around the path: random-init weights and input hidden states
+# ---------------------------------------------------------------------------
+ENCODER_CFG2 = Workload("encoder_cfg2_L1024_B8", n_layers=12, B=8, L=1024)
+
+
+def encoder_weights(D: int, layer: int, seed: int = 1):
+    """Random-init weights of one RoBERTa-size layer (no checkpoint is available):
+    matrices N(0, 1/fan_in) as bf16 bits [out][in], biases N(0, 0.02^2), layer-norm
+    gains 1 + N(0, 0.1^2) and shifts N(0, 0.1^2) as float32."""
+    g = _rng(seed, _TAG_WEIGHTS, layer)
+    def mat(o, i):
+        return f32_to_bf16_bits(g.standard_normal((o, i), dtype=np.float32) / np.float32(np.sqrt(i)))
+    def vec(n, scale, shift=0.0):
+        return (np.float32(shift) + np.float32(scale) * g.standard_normal(n, dtype=np.float32))
+    return {"W_qkv": mat(3 * D, D), "b_qkv": vec(3 * D, 0.02), "W_o": mat(D, D), "b_o": vec(D, 0.02),
+            "ln1_gamma": vec(D, 0.1, 1.0), "ln1_beta": vec(D, 0.1), "W_1": mat(4 * D, D),
+            "b_1": vec(4 * D, 0.02), "W_2": mat(D, 4 * D), "b_2": vec(D, 0.02),
+            "ln2_gamma": vec(D, 0.1, 1.0), "ln2_beta": vec(D, 0.1)}
+
+
+def encoder_input(wl: Workload):
+    """Layer-0 hidden states: bf16 bits [B, L, D], N(0, 1)."""
+    g = _rng(wl.seed, _TAG_HIDDEN)
+    return f32_to_bf16_bits(g.standard_normal((wl.B, wl.L, wl.H * wl.d), dtype=np.float32))

@@ -830,10 +830,23 @@ int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, cons
               const int32_t* gidx, const uint16_t* W, const float* bias, int gelu,
               const uint16_t* res, int res_gathered, void* out, int out_f32, int* status) {
   *g = GemmParams{};
+  // 256-column tiles unless that leaves fewer than two tiles per SM (the row
+  // count is a bound: rows are counted on the device) and A is not gathered
+  // (a gathered A is fetched again for every column tile)
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    cudaGetLastError();
+    sms = 152;
+  }
+  const long long row_tiles = static_cast<long long>(B) * ((L + kTile - 1) / kTile);
+  const int bn = (!gidx && row_tiles * ((N + 255) / 256) < 2ll * sms) ? 128 : 256;
+  const int wbox = N < bn ? N : bn;
   if (!encode_2d(&g->map_a, A, static_cast<long long>(B) * L, K, 1) ||
-      !encode_2d(&g->map_w, W, N, K, kTile))
+      !encode_2d(&g->map_at, A, static_cast<long long>(B) * L, K, kTile) ||
+      !encode_2d(&g->map_w, W, N, K, wbox))
     return SC_ERR_CUDA;
-  g->B = B; g->L = L; g->N = N; g->K = K;
+  g->B = B; g->L = L; g->N = N; g->K = K; g->bn = bn; g->wbox = wbox;
   g->rows = rows; g->gidx = gidx; g->bias = bias; g->gelu = gelu;
   g->res = res; g->res_gathered = res_gathered;
   g->out = out; g->out_f32 = out_f32; g->out_split = 0;

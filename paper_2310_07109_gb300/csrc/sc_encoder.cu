@@ -13,12 +13,13 @@
 // compaction of the kept rows is the A-operand gather of the output
 // projection (Y is the next layer's X, already compacted).
 //
-// GEMM: one CTA per 128 x 128 output tile of one sequence (rows are (sequence,
-// row) pairs, row < rows[b] read on the device), K in steps of 64 through a
-// three-stage TMA ring: A's 128 rows by four-row gathers (tile::gather4, any
-// row order), W's 128 rows by one tiled copy, both 128B-swizzled and K-major;
-// one thread issues the MMAs into a 128-column fp32 accumulator in tensor
-// memory; four warps read it back and apply bias, GELU and the residual.
+// GEMM: 128 x 256 output tiles of one sequence each (rows are (sequence, row)
+// pairs, row < rows[b] read on the device), one persistent CTA per SM walking
+// the tiles; K in steps of 64 through a four-stage TMA ring: A's 128 rows by
+// four-row gathers (tile::gather4, any row order), W's 256 rows by one tiled
+// copy, both 128B-swizzled and K-major; one thread issues the MMAs (N = 256)
+// into one of two 256-column fp32 accumulators in tensor memory while four
+// warps read the other back and apply bias, GELU and the residual.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
@@ -28,17 +29,21 @@
 
 namespace sc {
 
-constexpr int kGemmThreads = 192;   // warp 0 loads, warp 1 issues, warps 2-5 write back
-constexpr int kGemmStages = 3;
+constexpr int kGemmThreads = 320;   // warp 0 loads, warp 1 issues, warps 2-9 write back
+constexpr int kGemmEpiWarps = 8;    // two per tensor-memory lane quarter, one column half each
+constexpr int kGemmStages = 4;
 constexpr int kGemmBK = 64;         // K per stage: one 128-byte swizzle atom of bf16
-constexpr uint32_t kGemmStageBytes = 2 * kTileBytes;   // A and W tiles, 16 KB each
+constexpr int kGemmBN = 256;        // output columns per tile (one MMA, N = 256)
+constexpr uint32_t kGemmABytes = kTileBytes;              // 128 rows x 64
+constexpr uint32_t kGemmWBytes = kGemmBN * kGemmBK * 2;   // 256 rows x 64
+constexpr uint32_t kGemmStageBytes = kGemmABytes + kGemmWBytes;
 constexpr uint32_t kGemmDyn = kGemmStages * kGemmStageBytes + 1024;
 
 struct GemmSmem {
-  uint64_t full[kGemmStages], empty[kGemmStages], done;
+  uint64_t full[kGemmStages], empty[kGemmStages];
+  uint64_t tfull[2], tempty[2];   // accumulator buffers: written by the MMAs, read back
   uint32_t tmem_base;
   int abort;
-  float bias[kTile];
 };
 
 // Bounded wait that ignores the abort flag (teardown: no copy or MMA may still
@@ -60,34 +65,55 @@ __device__ __forceinline__ float gelu_erf(float x) {
   return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
 }
 
-__global__ void __launch_bounds__(kGemmThreads, 2)
+// Tile t of the launch: column block nt of width bn (fastest, so that the
+// CTAs of a wave share A rows), row tile rt of sequence b.
+struct GemmTile {
+  int b, r0, n0, nw, rows;
+  bool skip;
+};
+
+__device__ __forceinline__ GemmTile gemm_tile(const GemmParams& p, int t) {
+  const int tiles_n = (p.N + p.bn - 1) / p.bn;
+  const int tiles_r = (p.L + kTile - 1) / kTile;
+  GemmTile g;
+  const int nt = t % tiles_n, rest = t / tiles_n;
+  g.b = rest / tiles_r;
+  g.r0 = (rest % tiles_r) * kTile;
+  g.n0 = nt * p.bn;
+  g.nw = min(p.bn, p.N - g.n0);
+  g.rows = p.rows ? min(__ldcg(p.rows + g.b), p.L) : p.L;
+  g.skip = g.r0 >= g.rows;
+  return g;
+}
+
+// Persistent: each CTA walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...;
+// the accumulator alternates between two 256-column buffers, so that the
+// write-back of one tile overlaps the MMAs of the next.
+__global__ void __launch_bounds__(kGemmThreads, 1)
     sc_gemm_kernel(const __grid_constant__ GemmParams p) {
   pdl_wait();
   pdl_launch_dependents();
-  const int n0 = blockIdx.x * kTile;
-  const int tiles_per_seq = (p.L + kTile - 1) / kTile;
-  const int b = blockIdx.y / tiles_per_seq, r0 = (blockIdx.y % tiles_per_seq) * kTile;
-  const int rows = p.rows ? min(__ldcg(p.rows + b), p.L) : p.L;
-  if (r0 >= rows) return;
-
   extern __shared__ uint8_t dyn_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dyn_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   __shared__ GemmSmem sm;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int ksteps = p.K / kGemmBK;
+  const int tiles = p.B * ((p.L + kTile - 1) / kTile) * ((p.N + p.bn - 1) / p.bn);
 
   if (tid == 0) {
     for (int s = 0; s < kGemmStages; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], 1);
     }
-    mbar_init(&sm.done, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sm.tfull[a], 1);
+      mbar_init(&sm.tempty[a], kGemmEpiWarps);   // one arrival per write-back warp
+    }
     sm.abort = 0;
     fence_mbar_init();
   }
-  if (tid < kTile) sm.bias[tid] = p.bias ? __ldg(p.bias + n0 + tid) : 0.f;
-  if (warp == 1) tmem_alloc(&sm.tmem_base, 128);
+  if (warp == 1) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -96,116 +122,163 @@ __global__ void __launch_bounds__(kGemmThreads, 2)
 
   if (warp == 0) {
     // ------------------------------------------------------------- loads
-    // this lane's four A rows (rows past the sequence read row 0: discarded)
-    int ar[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int r = r0 + 4 * lane + k;
-      const int src = r < rows ? (p.gidx ? __ldcg(p.gidx + static_cast<size_t>(b) * p.L + r) : r) : 0;
-      ar[k] = b * p.L + src;
-    }
     bool ok = true;
-    for (int kt = 0, s = 0, use = 0; ok && kt < ksteps; ++kt) {
-      if (kt >= kGemmStages) ok = warp_wait_gemm(&sm.empty[s], (use - 1) & 1, abort_flag);
-      if (!ok) break;
-      uint8_t* As = base + s * kGemmStageBytes;
-      uint8_t* Ws = As + kTileBytes;
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&sm.full[s], kGemmStageBytes);
-        tma_load_2d(Ws, &p.map_w, kt * kGemmBK, n0, &sm.full[s]);
-      }
-      __syncwarp();
-      tma_gather4(As + 512 * lane, &p.map_a, kt * kGemmBK, ar[0], ar[1], ar[2], ar[3], &sm.full[s]);
-      if (++s == kGemmStages) {
-        s = 0;
-        ++use;
-      }
-    }
-    // nothing may still be landing in shared memory when the CTA exits
-    if (lane == 0)
-      for (int s = 0; s < kGemmStages && s < ksteps; ++s) {
-        const int last = s + kGemmStages * ((ksteps - 1 - s) / kGemmStages);
-        drain_wait_gemm(&sm.full[s], (last / kGemmStages) & 1);
-      }
-    __syncwarp();
-  } else if (warp == 1) {
-    // ------------------------------------------------------------- MMA issue
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16(128, 128, false, false);
-      bool ok = true;
-      for (int kt = 0, s = 0, use = 0; ok && kt < ksteps; ++kt) {
-        if (!(ok = mbar_wait(&sm.full[s], use & 1, abort_flag))) break;
-        tc_fence_after();
-        const uint32_t a = smem_u32(base + s * kGemmStageBytes), w = a + kTileBytes;
+    int s = 0, use = 0;
+    for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x) {
+      const GemmTile g = gemm_tile(p, t);
+      if (g.skip) continue;
+      // gathered A: this lane's four rows (rows past the sequence read row 0:
+      // discarded); otherwise one tiled copy of 128 consecutive rows
+      int ar[4];
 #pragma unroll
-        for (int k = 0; k < kGemmBK / 16; ++k)
-          umma_bf16(tm, sdesc_sw128(a + 32 * k), sdesc_sw128(w + 32 * k), idesc, (kt | k) != 0);
-        umma_commit(&sm.empty[s]);   // the stage is free once these MMAs are done
+      for (int k = 0; k < 4; ++k) {
+        const int r = g.r0 + 4 * lane + k;
+        const int src =
+            r < g.rows ? (p.gidx ? __ldcg(p.gidx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
+        ar[k] = g.b * p.L + src;
+      }
+      const bool gather = p.gidx != nullptr;
+      for (int kt = 0; ok && kt < ksteps; ++kt) {
+        if (use > 0 && !(ok = warp_wait_gemm(&sm.empty[s], (use - 1) & 1, abort_flag))) break;
+        uint8_t* As = base + s * kGemmStageBytes;
+        uint8_t* Ws = As + kGemmABytes;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&sm.full[s], kGemmABytes + p.wbox * kGemmBK * 2);
+          tma_load_2d(Ws, &p.map_w, kt * kGemmBK, g.n0, &sm.full[s]);
+          if (!gather) tma_load_2d(As, &p.map_at, kt * kGemmBK, g.b * p.L + g.r0, &sm.full[s]);
+        }
+        __syncwarp();
+        if (gather)
+          tma_gather4(As + 512 * lane, &p.map_a, kt * kGemmBK, ar[0], ar[1], ar[2], ar[3],
+                      &sm.full[s]);
         if (++s == kGemmStages) {
           s = 0;
           ++use;
         }
       }
-      umma_commit(&sm.done);
-      drain_wait_gemm(&sm.done, 0);
+    }
+    // nothing may still be landing in shared memory when the CTA exits: the
+    // last fill of every slot
+    if (lane == 0)
+      for (int q = 0; q < kGemmStages; ++q) {
+        const int fills = use + (q < s ? 1 : 0);
+        if (fills > 0) drain_wait_gemm(&sm.full[q], (fills - 1) & 1);
+      }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------- MMA issue
+    if (lane == 0) {
+      bool ok = true;
+      int s = 0, use = 0, j = 0;
+      for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x) {
+        const GemmTile g = gemm_tile(p, t);
+        if (g.skip) continue;
+        const int acc = j & 1;
+        // the buffer's previous tile has been read back
+        if (j >= 2 && !(ok = mbar_wait(&sm.tempty[acc], ((j >> 1) - 1) & 1, abort_flag))) break;
+        tc_fence_after();
+        const uint32_t idesc = idesc_bf16(128, g.nw, false, false);
+        const uint32_t d = tm + acc * kGemmBN;
+        for (int kt = 0; ok && kt < ksteps; ++kt) {
+          if (!(ok = mbar_wait(&sm.full[s], use & 1, abort_flag))) break;
+          tc_fence_after();
+          const uint32_t a = smem_u32(base + s * kGemmStageBytes), w = a + kGemmABytes;
+#pragma unroll
+          for (int k = 0; k < kGemmBK / 16; ++k)
+            umma_bf16(d, sdesc_sw128(a + 32 * k), sdesc_sw128(w + 32 * k), idesc, (kt | k) != 0);
+          umma_commit(&sm.empty[s]);   // the stage is free once these MMAs are done
+          if (++s == kGemmStages) {
+            s = 0;
+            ++use;
+          }
+        }
+        umma_commit(&sm.tfull[acc]);
+        ++j;
+      }
+      // every MMA has completed before the tensor memory is freed
+      uint64_t* last = &sm.empty[(s + kGemmStages - 1) % kGemmStages];
+      if (use > 0 || s > 0) {
+        const int q = (s + kGemmStages - 1) % kGemmStages;
+        const int fills = use + (q < s ? 1 : 0);
+        drain_wait_gemm(last, (fills - 1) & 1);
+      }
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------- write back
-    const int q = warp & 3;                   // tensor-memory lane quarter of this warp
-    const int r = r0 + 32 * q + lane;         // output row of this thread
-    const bool valid = r < rows;
-    const bool ok = warp_wait_gemm(&sm.done, 0, abort_flag);
-    const size_t orow = static_cast<size_t>(b) * p.L + r;
-    const int rsrc = valid ? (p.res_gathered && p.gidx ? __ldcg(p.gidx + static_cast<size_t>(b) * p.L + r) : r) : 0;
-    const uint16_t* res = p.res ? p.res + (static_cast<size_t>(b) * p.L + rsrc) * p.N + n0 : nullptr;
-    // output block of this tile (split outputs: column blocks of out_split)
-    int nb = n0, ldo = p.N;
-    void* outp = p.out;
-    if (p.out_split > 0) {
-      const int j = n0 / p.out_split;
-      outp = p.outs[j];
-      nb = n0 - j * p.out_split;
-      ldo = p.out_split;
-    }
-    if (ok) tc_fence_after();
-#pragma unroll 1
-    for (int c = 0; c < kTile; c += 32) {
-      float v[32];
-      tmem_ld32(tm + (static_cast<uint32_t>(32 * q) << 16) + c, v);
-      tmem_ld_wait();
-      if (!ok || !valid) continue;
-#pragma unroll
-      for (int k = 0; k < 32; ++k) {
-        float x = v[k] + sm.bias[c + k];
-        if (p.gelu) x = gelu_erf(x);
-        v[k] = x;
+    const int q = warp & 3;                  // tensor-memory lane quarter of this warp
+    const int ch = (warp - 2) / 4;           // column half of the tile
+    bool ok = true;
+    int j = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
+      const GemmTile g = gemm_tile(p, t);
+      if (g.skip) continue;
+      const int acc = j & 1;
+      ok = ok && warp_wait_gemm(&sm.tfull[acc], (j >> 1) & 1, abort_flag);
+      const int r = g.r0 + 32 * q + lane;
+      const bool valid = ok && r < g.rows;
+      const size_t orow = static_cast<size_t>(g.b) * p.L + r;
+      const int rsrc = valid ? (p.res_gathered && p.gidx
+                                    ? __ldcg(p.gidx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
+      const uint16_t* res =
+          p.res ? p.res + (static_cast<size_t>(g.b) * p.L + rsrc) * p.N + g.n0 : nullptr;
+      int nb = g.n0, ldo = p.N;
+      void* outp = p.out;
+      if (p.out_split > 0) {
+        const int sj = g.n0 / p.out_split;
+        outp = p.outs[sj];
+        nb = g.n0 - sj * p.out_split;
+        ldo = p.out_split;
       }
-      if (res) {
+      tc_fence_after();
+#pragma unroll 1
+      for (int c = ch * (p.bn / 2); c < min(g.nw, (ch + 1) * (p.bn / 2)); c += 32) {
+        float v[32];
+        tmem_ld32(tm + acc * kGemmBN + (static_cast<uint32_t>(32 * q) << 16) + c, v);
+        tmem_ld_wait();
+        if (!valid) continue;
+        const float4* bp = reinterpret_cast<const float4*>(p.bias + g.n0 + c);
 #pragma unroll
-        for (int k = 0; k < 32; k += 8) {
-          const uint4 u = __ldcg(reinterpret_cast<const uint4*>(res + c + k));
-          const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+        for (int k = 0; k < 32; k += 4) {
+          const float4 b4 = p.bias ? __ldg(bp + k / 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+          v[k] += b4.x;
+          v[k + 1] += b4.y;
+          v[k + 2] += b4.z;
+          v[k + 3] += b4.w;
+        }
+        if (p.gelu)
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            v[k + 2 * e] += __uint_as_float(w4[e] << 16);
-            v[k + 2 * e + 1] += __uint_as_float(w4[e] & 0xffff0000u);
+          for (int k = 0; k < 32; ++k) v[k] = gelu_erf(v[k]);
+        if (res) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 8) {
+            const uint4 u = __ldcg(reinterpret_cast<const uint4*>(res + c + k));
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              v[k + 2 * e] += __uint_as_float(w4[e] << 16);
+              v[k + 2 * e + 1] += __uint_as_float(w4[e] & 0xffff0000u);
+            }
           }
         }
-      }
-      if (p.out_f32) {
-        float* o = static_cast<float*>(outp) + orow * ldo + nb + c;
+        if (p.out_f32) {
+          float* o = static_cast<float*>(outp) + orow * ldo + nb + c;
 #pragma unroll
-        for (int k = 0; k < 32; k += 4)
-          *reinterpret_cast<float4*>(o + k) = make_float4(v[k], v[k + 1], v[k + 2], v[k + 3]);
-      } else {
-        uint16_t* o = static_cast<uint16_t*>(outp) + orow * ldo + nb + c;
+          for (int k = 0; k < 32; k += 4)
+            *reinterpret_cast<float4*>(o + k) = make_float4(v[k], v[k + 1], v[k + 2], v[k + 3]);
+        } else {
+          uint16_t* o = static_cast<uint16_t*>(outp) + orow * ldo + nb + c;
 #pragma unroll
-        for (int k = 0; k < 32; k += 8)
-          *reinterpret_cast<uint4*>(o + k) =
-              make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
-                         pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
+          for (int k = 0; k < 32; k += 8)
+            *reinterpret_cast<uint4*>(o + k) =
+                make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
+                           pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
+        }
       }
+      // the buffer may take the tile after next
+      tc_fence_before();
+      warp_arrive(&sm.tempty[acc]);
+      ++j;
     }
   }
 
@@ -213,7 +286,7 @@ __global__ void __launch_bounds__(kGemmThreads, 2)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tm, 128);
+    tmem_dealloc(tm, 512);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 }
@@ -288,9 +361,17 @@ static cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 }
 
 cudaError_t launch_gemm(const GemmParams& p, cudaStream_t st) {
-  const int tiles_per_seq = (p.L + kTile - 1) / kTile;
-  return launch_pdl(sc_gemm_kernel, dim3(p.N / kTile, p.B * tiles_per_seq), dim3(kGemmThreads),
-                    kGemmDyn, st, p);
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+  }
+  const long long tiles = static_cast<long long>(p.B) * ((p.L + kTile - 1) / kTile) *
+                          ((p.N + p.bn - 1) / p.bn);
+  const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
+  return launch_pdl(sc_gemm_kernel, dim3(grid), dim3(kGemmThreads), kGemmDyn, st, p);
 }
 
 cudaError_t launch_layernorm(const LayerNormParams& p, cudaStream_t st) {

@@ -191,11 +191,15 @@ struct TailParams {
 // One GEMM of the encoder layer: out[(b, r)][n] = epi(sum_k A[row_a][k] W[n][k])
 // for r < rows[b], row_a = b L + (gidx ? gidx[b L + r] : r); epi adds bias[n],
 // then GELU (gelu != 0), then the bf16 residual res[row][n] (row = row_a when
-// res_gathered, else b L + r).  N % 128 == 0, K % 64 == 0.
+// res_gathered, else b L + r).  N % 128 == 0, K % 64 == 0; 128 x 256 tiles.
 struct GemmParams {
   CUtensorMap map_a;               // 2-D [B L][K] bf16, box 64 x 1 (four-row gathers)
-  CUtensorMap map_w;               // 2-D [N][K] bf16, box 64 x 128
+  CUtensorMap map_at;              // the same matrix, box 64 x 128 (consecutive rows)
+  CUtensorMap map_w;               // 2-D [N][K] bf16, box 64 x wbox
   int B, L, N, K;
+  int bn;                          // output columns per tile: 256, or 128 when that gives
+                                   // too few tiles for the SMs
+  int wbox;                        // W rows per copy: min(bn, N)
   const int32_t* rows;             // [B] rows per sequence, or nullptr (L)
   const int32_t* gidx;             // [B][L] A row of output row (b, r), or nullptr
   const float* bias;               // [N] or nullptr

@@ -23,6 +23,11 @@ HBM.  The default workload is the 12-layer stack B=2, L=4096, H=12, d=64, window
 The inputs of one step (453 MB of Q/K/V) are larger than the 129 MB L2, so no
 flush is needed between steps.
 
+e2e: the same metric through sc_stack_forward_host, the call that takes the
+inputs and results in page-locked host memory: each step the kernels read the
+rows each layer uses over the host link and write the defined result slots back
+(replayed as a CUDA graph, like the device-resident steps).
+
 Metric: kept tokens/s = sum over layers and sequences of the tokens entering the
 layer (token-layers processed) / stack time.  Under torchrun each rank runs an
 independent replica (weak scaling, no collective on the data path); value is the
@@ -539,25 +544,58 @@ def run_native(args, wl):
         "cols_ms_per_layer": [round(float(x), 5) for x in cols_ms],
     }
 
-    # ---- end to end through the public API: pinned host inputs in, results out
-    hout = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in out.items()}
-    h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = sum(t.numel() * t.element_size() for t in hout.values())
-    e2e_steps = max(1, min(args.steps, 5))
+    # ---- end to end through the public host-buffer call (sc_stack_forward_host):
+    # page-locked Q/K/V in, page-locked results out.  The kernels read each
+    # layer's surviving rows over the host link and write back the current slots
+    # of every layer, all inside the timed steps.
+    hout = sc.new_host_outputs(wl.n_layers, wl.B, wl.L, wl.H)
+    hmask = None if inp["pad_mask"] is None else torch.from_numpy(inp["pad_mask"]).pin_memory()
+    hws = sc.new_stack_host_workspace(wl.n_layers, wl.B, wl.L, wl.H, dev)
+
+    def host_step():
+        sc.stack_forward_host(host["Q"], host["K"], host["V"], hmask, gpos, wl.w, alpha,
+                              out=hout, workspace=hws, keep_rule=wl.keep_rule)
+
+    for _ in range(max(3, args.warmup)):
+        host_step()
+    hgraph = None
+    if not args.no_graph:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            host_step()
+            hgraph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(hgraph, stream=side):
+                host_step()
+        torch.cuda.current_stream().wait_stream(side)
+        for _ in range(max(3, args.warmup)):
+            hgraph.replay()
+    torch.cuda.synchronize()
     barrier()
     t0.record(stream)
-    for _ in range(e2e_steps):
-        for k in host:
-            dQKV[k].copy_(host[k], non_blocking=True)
-        step()
-        for k in out:
-            hout[k].copy_(out[k], non_blocking=True)
+    for _ in range(args.steps):
+        if hgraph is not None:
+            hgraph.replay()
+        else:
+            host_step()
     t1.record(stream)
     barrier()
-    e2e_ms = max_over_ranks(t0.elapsed_time(t1) / e2e_steps, dev)
+    e2e_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, dev)
+    rc = sc.workspace_status(hws)
+    if rc != 0:
+        raise SystemExit("device status after the end-to-end steps: %s" % sc.status_string(rc))
+    if not torch.equal(hout["len"], out["len"].cpu()):
+        raise SystemExit("the host-buffer call disagrees with the device call on the lengths")
+    # bytes that crossed the host link per step: the rows each layer read, the
+    # padding mask, and the defined result slots written back
+    row_bytes = wl.H * wl.d * 2
+    in_rows = int(lens[:wl.n_layers].sum())
+    h2d = 3 * row_bytes * in_rows + (0 if hmask is None else hmask.numel())
+    d2h = (row_bytes + 4) * in_rows + 4 * int(lens.sum()) + 4 * lens.size
     e2e = {"value": whole_job_rate(world, kept_per_step, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-           "ms_per_step": e2e_ms}
+           "ms_per_step": e2e_ms, "call": "sc_stack_forward_host",
+           "cuda_graph": hgraph is not None}
 
     line = {"metric": metric_name(wl), "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,

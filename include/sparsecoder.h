@@ -227,6 +227,44 @@ int sc_stack_forward_profiled(const sc_stack_args* args, void* workspace, size_t
  * launched.  Errors: see sc_status (SC_ERR_CUDA without a usable device). */
 int sc_stack_launch_count(const sc_stack_args* args, int* count);
 
+/*
+ * The pruned stack with its inputs and results in HOST memory: the same
+ * computation and results as sc_stack_forward (Fig. "sparsecoder"; Sec.
+ * "Sparse Attention", "Token Pruning"), for callers whose tensors live on the
+ * host.  The kernels move only what the method uses: layer l reads, over the
+ * host link, the Q/K/V rows of the tokens that survived layers 0..l-1 (token
+ * pruning, Sec. "Token Pruning" Step 3, removes the others from every later
+ * layer), and the results are written back only where sc_stack_forward
+ * defines them.
+ *
+ * args       as for sc_stack_forward, except that Q, K, V, pad_mask (or NULL),
+ *            O, scores, pos and len are HOST pointers to page-locked memory
+ *            (cudaHostAlloc / cudaMallocHost, or cudaHostRegister'ed) that the
+ *            device can address; alpha and global_pos are host arrays as there.
+ *            Written on the host: len (all of it), and for every (l, b) the
+ *            first len[l][b] entries of pos[l][b] (l <= n_layers), scores[l][b]
+ *            and rows of O[l][b] (l < n_layers); every other entry is left as
+ *            it was.
+ * workspace  DEVICE memory of sc_stack_host_workspace_size(n_layers, B, L, H)
+ *            bytes (256-byte aligned): the scratch of sc_stack_forward followed
+ *            by device copies of the results.
+ *
+ * Asynchronous on `stream` like every call: the host buffers must stay
+ * allocated and unmodified (inputs) or unread (results) until the stream has
+ * passed the call.  Capturable in a CUDA graph (it issues kernels only).
+ * Errors: as sc_stack_forward, and SC_ERR_INVALID_ARG with nothing launched
+ * when a host range is not page-locked memory mapped for the device (checked
+ * at both ends of each range) or a mapped address is misaligned (Q, K, V, O:
+ * 16 bytes; scores, pos, len: 4 bytes).
+ */
+size_t sc_stack_host_workspace_size(int n_layers, int B, int L, int H);
+int sc_stack_forward_host(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
+                          void* stream);
+
+/* Number of kernels that sc_stack_forward_host launches for these arguments,
+ * as sc_stack_launch_count for sc_stack_forward. */
+int sc_stack_host_launch_count(const sc_stack_args* args, int* count);
+
 /* Synchronises `stream`, returns SC_ERR_TIMEOUT if any kernel since the last
  * query recorded an expired wait (else SC_OK, or SC_ERR_CUDA), and clears
  * the status word. */

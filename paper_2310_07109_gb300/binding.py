@@ -87,7 +87,8 @@ SC_KEEP_TOP_RATIO = 2  # keep ceil(alpha n) tokens: the first and the best other
 TAIL_MAX_LEN = 384
 
 EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
-            "sc_stack_forward_profiled", "sc_stack_launch_count",
+            "sc_stack_forward_profiled", "sc_stack_launch_count", "sc_stack_forward_host",
+            "sc_stack_host_workspace_size", "sc_stack_host_launch_count",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error",
             "sc_encoder_layer_forward", "sc_encoder_workspace_size", "sc_linear_forward",
             "sc_layer_norm_forward"]
@@ -128,6 +129,14 @@ def load(build_if_missing: bool = False):
         lib.sc_stack_launch_count.restype = ctypes.c_int
         lib.sc_stack_launch_count.argtypes = [ctypes.POINTER(StackArgs),
                                               ctypes.POINTER(ctypes.c_int)]
+        lib.sc_stack_host_workspace_size.restype = ctypes.c_size_t
+        lib.sc_stack_host_workspace_size.argtypes = [ctypes.c_int] * 4
+        lib.sc_stack_forward_host.restype = ctypes.c_int
+        lib.sc_stack_forward_host.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
+                                              ctypes.c_size_t, ctypes.c_void_p]
+        lib.sc_stack_host_launch_count.restype = ctypes.c_int
+        lib.sc_stack_host_launch_count.argtypes = [ctypes.POINTER(StackArgs),
+                                                   ctypes.POINTER(ctypes.c_int)]
         lib.sc_workspace_status.restype = ctypes.c_int
         lib.sc_workspace_status.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         lib.sc_status_string.restype = ctypes.c_char_p
@@ -265,8 +274,10 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
     return out
 
 
-def stack_launch_count(n_layers, B, L, H, w, global_pos, has_pad_mask, no_tail=False) -> int:
-    """Kernels one ``stack_forward`` call launches for these sizes on the current device."""
+def stack_launch_count(n_layers, B, L, H, w, global_pos, has_pad_mask, no_tail=False,
+                       host=False) -> int:
+    """Kernels one ``stack_forward`` (``host``: ``stack_forward_host``) call launches for
+    these sizes on the current device."""
     garr, ng = _int32_host(global_pos)
     # only whether pad_mask is NULL matters: a non-null marker is never dereferenced
     a = StackArgs(int(n_layers), int(B), int(L), int(H), int(w), None, None, None,
@@ -274,8 +285,61 @@ def stack_launch_count(n_layers, B, L, H, w, global_pos, has_pad_mask, no_tail=F
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng, None, None, None,
                   None, None, SC_STACK_NO_TAIL if no_tail else 0)
     cnt = ctypes.c_int(0)
-    _check(load().sc_stack_launch_count(ctypes.byref(a), ctypes.byref(cnt)))
+    fn = load().sc_stack_host_launch_count if host else load().sc_stack_launch_count
+    _check(fn(ctypes.byref(a), ctypes.byref(cnt)))
     return int(cnt.value)
+
+
+def stack_host_workspace_size(n_layers, B, L, H) -> int:
+    return int(load().sc_stack_host_workspace_size(int(n_layers), int(B), int(L), int(H)))
+
+
+def new_stack_host_workspace(n_layers, B, L, H, device=None) -> torch.Tensor:
+    n = stack_host_workspace_size(n_layers, B, L, H)
+    if n == 0:
+        raise SparseCoderError(SC_ERR_INVALID_ARG, "invalid workspace sizes")
+    ws = torch.zeros(n + 256, dtype=torch.uint8, device=device or "cuda")
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + n]
+
+
+def new_host_outputs(n_layers, B, L, H):
+    """Page-locked host result tensors for ``stack_forward_host``."""
+    return {"O": torch.empty((n_layers, B, L, H, 64), dtype=torch.bfloat16, pin_memory=True),
+            "scores": torch.empty((n_layers, B, L), dtype=torch.float32, pin_memory=True),
+            "pos": torch.empty((n_layers + 1, B, L), dtype=torch.int32, pin_memory=True),
+            "len": torch.empty((n_layers + 1, B), dtype=torch.int32, pin_memory=True)}
+
+
+def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
+                       stream=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE):
+    """The pruned stack on host tensors (``sc_stack_forward_host``).
+
+    Q, K, V: bf16 [n_layers, B, L, H, 64] page-locked CPU tensors (``pin_memory()``);
+    pad_mask: uint8 [B, L] page-locked CPU tensor or None; the other arguments as for
+    ``stack_forward``.  ``out``: page-locked result tensors (``new_host_outputs``);
+    only the current slots of each layer (and all of ``len``) are written.
+    The call is asynchronous on ``stream`` (default: torch's current stream of the
+    current device): synchronise before reading ``out``.
+    Returns the dict of host tensors O, scores, pos, len.
+    """
+    nl, B, L, H, D = Q.shape
+    for name, t in (("Q", Q), ("K", K), ("V", V), ("pad_mask", pad_mask)):
+        if t is not None and (t.device.type != "cpu" or not t.is_pinned()):
+            raise SparseCoderError(SC_ERR_INVALID_ARG, name + " must be a page-locked CPU tensor")
+    if out is None:
+        out = new_host_outputs(nl, B, L, H)
+    ws = workspace if workspace is not None else new_stack_host_workspace(nl, B, L, H)
+    garr, ng = _int32_host(global_pos)
+    al = (ctypes.c_float * nl)(*[float(x) for x in alpha])
+    a = StackArgs(nl, B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(pad_mask),
+                  ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
+                  ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
+                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
+                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule))
+    _check(load().sc_stack_forward_host(ctypes.byref(a), _ptr(ws), ws.numel(),
+                                        _stream_handle(stream)))
+    return out
 
 
 def workspace_status(workspace, stream=None) -> int:

@@ -21,6 +21,7 @@ cudaError_t configure_kernels();
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st);
+cudaError_t launch_export(const ExportParams& e, cudaStream_t st);
 cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st);
 cudaError_t configure_tail();
 cudaError_t tail_max_clusters(int H, int* out);
@@ -427,8 +428,12 @@ static int stack_plan(const sc_stack_args* a, bool* use_tail, bool* per_layer) {
   return SC_OK;
 }
 
+// host_io: Q, K, V (and pad_mask) are device-mapped addresses of host memory,
+// which only the gather and cluster kernels read (plain loads): the tensor
+// maps of the "source" slot are pointed at the compacted copies and never
+// selected, and every layer's rows are gathered.
 static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
-                              void* stream, void** events, int n_events) {
+                              void* stream, void** events, int n_events, bool host_io = false) {
   if (!a) return SC_ERR_INVALID_ARG;
   if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
@@ -453,7 +458,10 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   compacted_qkv(ws, lay, a->B, a->L, a->H, cmp);
   const uint16_t* src[3] = {a->Q, a->K, a->V};
   const long long BLt = static_cast<long long>(a->B) * a->L;
-  if (!encode_maps(&maps, src, a->n_layers * BLt, cmp, BLt, a->H)) return SC_ERR_CUDA;
+  const uint16_t* map_src[3] = {host_io ? cmp[0] : src[0], host_io ? cmp[1] : src[1],
+                                host_io ? cmp[2] : src[2]};
+  if (!encode_maps(&maps, map_src, host_io ? BLt : a->n_layers * BLt, cmp, BLt, a->H))
+    return SC_ERR_CUDA;
   if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
 
   const size_t BL = static_cast<size_t>(a->B) * a->L;
@@ -468,6 +476,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   p.keep_rule = a->keep_rule;
   p.tail_from = tail_from;
   p.tail_max = use_tail ? kTailMax : 0;
+  p.no_ident = host_io ? 1 : 0;
   fill_workspace(&p, ws, lay, 0);
 
   PrepParams pp{};
@@ -480,6 +489,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   pp.ident = const_cast<int32_t*>(p.ident);
   pp.tail_from = tail_from;
   pp.tail_max = p.tail_max;
+  pp.no_ident = p.no_ident;
   pp.n_global = a->n_global;
   for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
   auto mark = [&](int k) {
@@ -534,7 +544,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     gp.dst[t] = cmp[t];
   }
   if (dev_loop) {
-    if (a->pad_mask != nullptr) {
+    if (a->pad_mask != nullptr || host_io) {
       // padding removal may have moved rows: compact layer 0 as well
       gp.src_base = 0;
       gp.layer = 0;
@@ -622,7 +632,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     p.O = a->O + static_cast<size_t>(l) * BL * a->H * kHeadDim;
     p.scores = a->scores + static_cast<size_t>(l) * BL;
     p.alpha = a->alpha[l];
-    if (l == 0 && a->pad_mask != nullptr) {
+    if (l == 0 && (a->pad_mask != nullptr || host_io)) {
       // padding removal may have moved rows: compact layer 0 as well
       gp.src_base = 0;
       gp.layer = 0;
@@ -655,6 +665,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     tp.scores = a->scores;
     tp.status = p.status;
     for (int t = 0; t < 3; ++t) tp.src[t] = src[t];
+    tp.src_host = host_io ? 1 : 0;
     tp.n_global = a->n_global;
     for (int g = 0; g < a->n_global; ++g) tp.global_pos[g] = a->global_pos[g];
     for (int l = 0; l < a->n_layers; ++l) tp.alpha[l] = a->alpha[l];
@@ -675,6 +686,127 @@ int sc_stack_forward_profiled(const sc_stack_args* a, void* workspace, size_t ws
   for (int k = 0; k < 3 + 3 * a->n_layers; ++k)
     if (!events[k]) return SC_ERR_INVALID_ARG;
   return stack_forward_impl(a, workspace, ws_bytes, stream, events, n_events);
+}
+
+// ---------------------------------------------------------------------------
+// The stack with host inputs and results
+// ---------------------------------------------------------------------------
+
+// Device-side copies of a stack's results, after the sc_stack_forward
+// workspace: O, scores, pos, len.
+struct HostIoLayout {
+  size_t O, scores, pos, len, total;
+};
+
+static bool host_io_layout(int n_layers, int B, int L, int H, HostIoLayout* h) {
+  WsLayout lay;
+  if (n_layers < 1 || !ws_layout(B, L, H, &lay)) return false;
+  const size_t BL = static_cast<size_t>(B) * L;
+  size_t off = align_up(lay.total);
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes);
+    return at;
+  };
+  h->O = take(sizeof(uint16_t) * n_layers * BL * H * kHeadDim);
+  h->scores = take(sizeof(float) * n_layers * BL);
+  h->pos = take(sizeof(int32_t) * (n_layers + 1) * BL);
+  h->len = take(sizeof(int32_t) * (n_layers + 1) * B);
+  h->total = off;
+  return true;
+}
+
+// The device address of page-locked host memory [p, p + bytes), or nullptr
+// unless both ends of the range are page-locked host memory mapped for the
+// device at consecutive addresses (so a kernel may read or write all of it).
+static void* mapped_host_range(const void* p, size_t bytes) {
+  if (p == nullptr || bytes == 0) return nullptr;
+  const char* first = static_cast<const char*>(p);
+  const char* last = first + (bytes - 1);
+  cudaPointerAttributes a0{}, a1{};
+  if (cudaPointerGetAttributes(&a0, first) != cudaSuccess ||
+      cudaPointerGetAttributes(&a1, last) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a0.type != cudaMemoryTypeHost || a1.type != cudaMemoryTypeHost ||
+      a0.devicePointer == nullptr || a1.devicePointer == nullptr)
+    return nullptr;
+  char* d0 = static_cast<char*>(a0.devicePointer);
+  if (static_cast<char*>(a1.devicePointer) != d0 + (bytes - 1)) return nullptr;
+  return d0;
+}
+
+size_t sc_stack_host_workspace_size(int n_layers, int B, int L, int H) {
+  HostIoLayout h;
+  if (!host_io_layout(n_layers, B, L, H, &h)) return 0;
+  return h.total;
+}
+
+int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
+  if (!a) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
+    return SC_ERR_INVALID_ARG;
+  HostIoLayout hl;
+  if (!host_io_layout(a->n_layers, a->B, a->L, a->H, &hl)) return SC_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < hl.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
+    return SC_ERR_WORKSPACE;
+  const size_t BL = static_cast<size_t>(a->B) * a->L;
+  const size_t qkv_bytes = sizeof(uint16_t) * a->n_layers * BL * a->H * kHeadDim;
+  void* q = mapped_host_range(a->Q, qkv_bytes);
+  void* k = mapped_host_range(a->K, qkv_bytes);
+  void* v = mapped_host_range(a->V, qkv_bytes);
+  void* o = mapped_host_range(a->O, qkv_bytes);
+  void* sc = mapped_host_range(a->scores, sizeof(float) * a->n_layers * BL);
+  void* ps = mapped_host_range(a->pos, sizeof(int32_t) * (a->n_layers + 1) * BL);
+  void* ln = mapped_host_range(a->len, sizeof(int32_t) * (a->n_layers + 1) * a->B);
+  void* pm = a->pad_mask ? mapped_host_range(a->pad_mask, BL) : nullptr;
+  if (!q || !k || !v || !o || !sc || !ps || !ln || (a->pad_mask && !pm))
+    return fail(SC_ERR_INVALID_ARG, "sc_stack_forward_host",
+                "a host buffer is not page-locked memory mapped for the device");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) ||
+      (reinterpret_cast<uintptr_t>(sc) & 3u) || (reinterpret_cast<uintptr_t>(ps) & 3u) ||
+      (reinterpret_cast<uintptr_t>(ln) & 3u))
+    return SC_ERR_INVALID_ARG;
+  char* ws = static_cast<char*>(workspace);
+  sc_stack_args d = *a;
+  d.Q = static_cast<const uint16_t*>(q);
+  d.K = static_cast<const uint16_t*>(k);
+  d.V = static_cast<const uint16_t*>(v);
+  d.pad_mask = static_cast<const uint8_t*>(pm);
+  d.O = reinterpret_cast<uint16_t*>(ws + hl.O);
+  d.scores = reinterpret_cast<float*>(ws + hl.scores);
+  d.pos = reinterpret_cast<int32_t*>(ws + hl.pos);
+  d.len = reinterpret_cast<int32_t*>(ws + hl.len);
+  if ((rc = stack_forward_impl(&d, workspace, hl.O, stream, nullptr, 0, true)) != SC_OK) return rc;
+  ExportParams e{};
+  e.n_layers = a->n_layers; e.B = a->B; e.L = a->L; e.H = a->H;
+  e.O = d.O; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
+  e.hO = static_cast<uint16_t*>(o);
+  e.hscores = static_cast<float*>(sc);
+  e.hpos = static_cast<int32_t*>(ps);
+  e.hlen = static_cast<int32_t*>(ln);
+  const cudaError_t ce = launch_export(e, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return fail_cuda("launch export kernel", ce);
+  return SC_OK;
+}
+
+int sc_stack_host_launch_count(const sc_stack_args* a, int* count) {
+  if (!a || !count) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
+  if (rc != SC_OK) return rc;
+  if ((rc = ensure_configured()) != SC_OK) return rc;
+  bool use_tail = false, per_layer = true;
+  if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
+  int k = 2;   // padding removal / global lookup, and the export
+  if (per_layer) k += 1 + 2 * a->n_layers + (a->n_layers - 1);
+  if (use_tail) k += 1;
+  *count = k;
+  return SC_OK;
 }
 
 int sc_stack_launch_count(const sc_stack_args* a, int* count) {

@@ -92,6 +92,9 @@ struct LayerParams {
   int32_t* tail_from;    // [B]
   int layer;
   int tail_max;
+  // nonzero: the source tensors are host memory, which the tensor maps never
+  // read: every layer's rows are gathered (ident is never set)
+  int no_ident;
   // Device-driven layer loop (a CUDA graph WHILE node): when dev_layer is set,
   // the layer is *dev_layer and the per-layer fields above hold their layer-0
   // values, advanced by these strides (gcur/ng/ident swap slots on odd layers;
@@ -169,8 +172,24 @@ struct PrepParams {
   int* dev_layer;            // device-driven loop: set to 0 here, or nullptr
   unsigned long long cond;   // ... and its WHILE condition: some sequence has > tail_max tokens
   int has_cond;
+  int no_ident;              // see LayerParams::no_ident
   int n_global;
   int global_pos[kMaxGlobal];
+};
+
+// Copies the results of a stack from the device to page-locked host memory:
+// len[l][b] for every l <= n_layers, and for each (l, b) the first len[l][b]
+// entries of pos (l <= n_layers), scores and O rows (l < n_layers).
+struct ExportParams {
+  int n_layers, B, L, H;
+  const uint16_t* O;           // device [n_layers][B][L][H][64]
+  const float* scores;         // device [n_layers][B][L]
+  const int32_t* pos;          // device [n_layers + 1][B][L]
+  const int32_t* len;          // device [n_layers + 1][B]
+  uint16_t* hO;                // host (device-mapped addresses), same layouts
+  float* hscores;
+  int32_t* hpos;
+  int32_t* hlen;
 };
 
 struct TailParams {
@@ -182,6 +201,9 @@ struct TailParams {
   float* scores;               // [n_layers][B][L]
   int* status;
   const uint16_t* src[3];      // Q, K, V [n_layers][B][L][H][64]
+  // nonzero: src is host memory; the next layer's rows are not prefetched
+  // (that would pull the rows of the tokens a layer prunes over the host link)
+  int src_host;
   int n_global;
   int global_pos[kMaxGlobal];
   float alpha[kTailMaxLayers];   // the keep rule's value per layer

@@ -1287,7 +1287,7 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     v.len_out[b] = total;
     if (p.tail_from != nullptr && total <= p.tail_max) p.tail_from[b] = v.layer + 1;
     // the survivors are original positions 0..total-1 exactly when the last one is total-1
-    v.ident_out[b] = (total == 0 || sm.last_pos == total - 1) ? 1 : 0;
+    v.ident_out[b] = (!p.no_ident && (total == 0 || sm.last_pos == total - 1)) ? 1 : 0;
     p.cnt_seq[b] = 0u;
     for (int hh = 0; hh < p.H; ++hh) p.rows_done[b * p.H + hh] = 0u;
   }
@@ -1350,6 +1350,52 @@ __global__ void __launch_bounds__(kGatherThreads)
 #pragma unroll
       for (int u = 0; u < kPer; ++u)
         if (so[u] >= 0) reinterpret_cast<uint4*>(g.dst[t])[doff[u]] = v[t][u];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// export kernel: a stack's results to page-locked host memory
+// ---------------------------------------------------------------------------
+constexpr int kExportTokens = 32;
+constexpr int kExportThreads = 256;
+
+// One CTA per 32 current slots of one (layer, sequence): only the slots below
+// the layer's length are copied.  Loads from device memory are issued in
+// groups of four before the stores, which cross the host link.
+__global__ void __launch_bounds__(kExportThreads)
+    sc_export_kernel(const ExportParams e) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int b = blockIdx.y, l = blockIdx.z;
+  const size_t li = static_cast<size_t>(l) * e.B + b;
+  const int n = __ldcg(e.len + li);
+  if (blockIdx.x == 0 && threadIdx.x == 0) e.hlen[li] = n;
+  const int c0 = blockIdx.x * kExportTokens;
+  if (c0 >= n) return;
+  const int cnt = min(kExportTokens, n - c0);
+  const size_t row0 = (static_cast<size_t>(l) * e.B + b) * e.L + c0;
+  if (threadIdx.x < cnt) {
+    e.hpos[row0 + threadIdx.x] = __ldcg(e.pos + row0 + threadIdx.x);
+    if (l < e.n_layers) e.hscores[row0 + threadIdx.x] = __ldcg(e.scores + row0 + threadIdx.x);
+  }
+  if (l >= e.n_layers) return;
+  const int vec = e.H * kHeadDim / 8;   // 16-byte vectors per row
+  const int total = cnt * vec;
+  const uint4* src = reinterpret_cast<const uint4*>(e.O) + row0 * vec;
+  uint4* dst = reinterpret_cast<uint4*>(e.hO) + row0 * vec;
+  constexpr int kPer = 4;
+  for (int k0 = threadIdx.x; k0 < total; k0 += kExportThreads * kPer) {
+    uint4 v[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int k = k0 + u * kExportThreads;
+      if (k < total) v[u] = __ldcg(src + k);
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int k = k0 + u * kExportThreads;
+      if (k < total) dst[k] = v[u];
+    }
   }
 }
 
@@ -1450,7 +1496,8 @@ __global__ void __launch_bounds__(kPrepThreads)
       if (gfound[g] >= 0) pp.gcur[b * kMaxGlobal + m++] = gfound[g];
     pp.ng[b] = m;
     // single-layer calls read their (already current-order) inputs in place
-    pp.ident[b] = (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1) ? 1 : 0;
+    pp.ident[b] = (!pp.no_ident && (pp.pos_in != nullptr || n == 0 || spos[n - 1] == n - 1))
+                      ? 1 : 0;
     if (pp.tail_from != nullptr) pp.tail_from[b] = n <= pp.tail_max ? 0 : 0x7fffffff;
     if (pp.has_cond && n > pp.tail_max) cudaGraphSetConditional(pp.cond, 1u);
     if (pp.dev_layer != nullptr && b == 0) *pp.dev_layer = 0;
@@ -1541,6 +1588,11 @@ cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t 
 
 cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st) {
   return launch_chained(sc_advance_kernel, dim3(1), dim3(256), 0, st, a);
+}
+
+cudaError_t launch_export(const ExportParams& e, cudaStream_t st) {
+  dim3 grid((e.L + kExportTokens - 1) / kExportTokens, e.B, e.n_layers + 1);
+  return launch_chained(sc_export_kernel, grid, dim3(kExportThreads), 0, st, e);
 }
 
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {

@@ -216,7 +216,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         cp_async16(k_a + so, p.src[1] + off);
         cp_async16(v_a + so, p.src[2] + off);
       }
-      if (l + 1 < n_layers) {
+      if (l + 1 < n_layers && !p.src_host) {
         // the next layer's tokens are a subset of the current ones
         const size_t tok1 = (static_cast<size_t>(l + 1) * B + b) * L;
         for (int r = tid; r < n; r += kTailThreads) {

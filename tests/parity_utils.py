@@ -135,3 +135,23 @@ def layer_case(B, L, H, lens, w, gpos, alpha, seed, scale_k=2.0, gaps=False, max
     return {"Q": Q, "K": K, "V": V, "pos": pos, "len": np.asarray(lens, np.int32),
             "global_pos": np.asarray(sorted(gset), np.int32), "alpha": alpha,
             "expected": expected}
+
+
+def check_stack(wl, res, got):
+    """A stack's results (numpy dict O as float64, scores, pos, len) against the
+    oracle's: lengths and positions exactly, O and scores within tolerance."""
+    np.testing.assert_array_equal(got["len"], res["len"])
+    for l in range(wl.n_layers + 1):
+        for b in range(wl.B):
+            n = int(res["len"][l, b])
+            np.testing.assert_array_equal(got["pos"][l, b, :n], res["pos"][l, b, :n],
+                                          err_msg=f"layer {l} seq {b}")
+    for l in range(wl.n_layers):
+        for b in range(wl.B):
+            n = int(res["len"][l, b])
+            if n == 0:
+                continue
+            np.testing.assert_allclose(got["O"][l, b, :n], res["O"][l, b, :n], rtol=O_RTOL,
+                                       atol=O_ATOL, err_msg=f"O layer {l} seq {b}")
+            np.testing.assert_allclose(got["scores"][l, b, :n], res["scores"][l, b, :n], rtol=0,
+                                       atol=SCORE_ATOL, err_msg=f"scores layer {l} seq {b}")

@@ -137,6 +137,47 @@ def test_stack_rejects_bad_arguments(lib):
                 alpha=ctypes.cast(bad, ctypes.POINTER(ctypes.c_float))) == bd.SC_ERR_INVALID_ARG
 
 
+def test_stack_host_rejects_bad_arguments(lib):
+    """The host-buffer stack checks its sizes, its workspace and that every host
+    range is page-locked memory mapped for the device before anything runs."""
+    g = (ctypes.c_int32 * 1)(0)
+    al = (ctypes.c_float * 2)(0.5, 0.5)
+    nl, B, L, H = 2, 2, 256, 2
+    n_qkv = nl * B * L * H * 64
+    plain = {k: (ctypes.c_uint16 * n_qkv)() for k in ("Q", "K", "V", "O")}
+    small = {"scores": (ctypes.c_float * (nl * B * L))(), "pos": (ctypes.c_int32 * ((nl + 1) * B * L))(),
+             "len": (ctypes.c_int32 * ((nl + 1) * B))()}
+    bufs = {k: ctypes.addressof(v) for k, v in {**plain, **small}.items()}
+    need = bd.stack_host_workspace_size(nl, B, L, H)
+
+    def call(ws_bytes=need, **kw):
+        a = dict(n_layers=nl, B=B, L=L, H=H, w=64, pad_mask=None,
+                 global_pos=ctypes.cast(g, ctypes.POINTER(ctypes.c_int32)), n_global=1,
+                 alpha=ctypes.cast(al, ctypes.POINTER(ctypes.c_float)), **bufs)
+        a.update(kw)
+        return lib.sc_stack_forward_host(ctypes.byref(bd.StackArgs(**a)), ctypes.c_void_p(FAKE),
+                                         ws_bytes, None)
+
+    assert lib.sc_stack_forward_host(None, None, 0, None) == bd.SC_ERR_INVALID_ARG
+    assert call(n_layers=0) == bd.SC_ERR_INVALID_ARG
+    assert call(Q=None) == bd.SC_ERR_INVALID_ARG
+    assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
+    assert call(flags=2) == bd.SC_ERR_INVALID_ARG
+    assert call(ws_bytes=need - 256) == bd.SC_ERR_WORKSPACE
+    # ordinary (pageable) host memory is refused: the kernels could not reach it
+    assert call() == bd.SC_ERR_INVALID_ARG
+
+
+def test_stack_host_workspace_size(lib):
+    nl, B, L, H = 12, 2, 4096, 12
+    base = bd.workspace_size(B, L, H)
+    results = nl * B * L * (H * 64 * 2 + 4) + (nl + 1) * B * (L + 1) * 4
+    n = bd.stack_host_workspace_size(nl, B, L, H)
+    assert base + results <= n <= base + results + 5 * 256 and n % 256 == 0
+    assert bd.stack_host_workspace_size(0, B, L, H) == 0
+    assert bd.stack_host_workspace_size(nl, B, 4097, H) == 0
+
+
 def test_launch_count_rejects_bad_arguments(lib):
     g = (ctypes.c_int32 * 1)(0)
 

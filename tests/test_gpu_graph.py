@@ -12,8 +12,7 @@ import torch
 
 import oracle
 import workloads as wk
-from parity_utils import bits_to_torch, resample_stack, torch_bf16_to_f64
-from test_gpu_parity import _check_stack
+from parity_utils import bits_to_torch, check_stack, resample_stack, torch_bf16_to_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -62,7 +61,7 @@ def _replay_and_check(sc, wl, graph, t, out, ws, inp, res):
     torch.cuda.synchronize()
     assert sc.workspace_status(ws) == 0
     got = _host(out)
-    _check_stack(wl, res, got)
+    check_stack(wl, res, got)
     return got
 
 

@@ -15,9 +15,9 @@ import torch
 
 import oracle
 import workloads as wk
-from parity_utils import (MARGIN, O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, resample_stack,
-                          torch_bf16_to_f64)
-from test_gpu_parity import _check_stack, _run_stack
+from parity_utils import (MARGIN, O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, check_stack,
+                          resample_stack, torch_bf16_to_f64)
+from test_gpu_parity import _run_stack
 
 pytestmark = pytest.mark.gpu
 
@@ -64,7 +64,7 @@ def test_rule_stack_matches_oracle(sc, wl, no_tail):
     if no_tail and wl.L > 2 * sc.TAIL_MAX_LEN and wl.n_layers == 1:
         pytest.skip("a single long layer runs in the per-layer kernels either way")
     inp, res, _ = _resampled(wl)
-    _check_stack(wl, res, _run_stack(sc, wl, inp, no_tail))
+    check_stack(wl, res, _run_stack(sc, wl, inp, no_tail))
 
 
 def test_top_ratio_lengths_follow_the_ratio(sc):

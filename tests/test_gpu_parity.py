@@ -10,8 +10,8 @@ import pytest
 import torch
 
 import workloads as wk
-from parity_utils import (O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, layer_case, resample_stack,
-                          torch_bf16_to_f64)
+from parity_utils import (O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, check_stack, layer_case,
+                          resample_stack, torch_bf16_to_f64)
 
 pytestmark = pytest.mark.gpu
 
@@ -88,24 +88,6 @@ def _run_stack(sc, wl, inp, no_tail=False):
             "pos": out["pos"].cpu().numpy(), "len": out["len"].cpu().numpy()}
 
 
-def _check_stack(wl, res, got):
-    np.testing.assert_array_equal(got["len"], res["len"])
-    for l in range(wl.n_layers + 1):
-        for b in range(wl.B):
-            n = int(res["len"][l, b])
-            np.testing.assert_array_equal(got["pos"][l, b, :n], res["pos"][l, b, :n],
-                                          err_msg=f"layer {l} seq {b}")
-    for l in range(wl.n_layers):
-        for b in range(wl.B):
-            n = int(res["len"][l, b])
-            if n == 0:
-                continue
-            np.testing.assert_allclose(got["O"][l, b, :n], res["O"][l, b, :n], rtol=O_RTOL,
-                                       atol=O_ATOL, err_msg=f"O layer {l} seq {b}")
-            np.testing.assert_allclose(got["scores"][l, b, :n], res["scores"][l, b, :n], rtol=0,
-                                       atol=SCORE_ATOL, err_msg=f"scores layer {l} seq {b}")
-
-
 STACKS = [
     wk.Workload("small_12x700", n_layers=12, B=2, L=700, w=64, n_extra_global=3, seed=3),
     wk.Workload("ragged_6x600", n_layers=6, B=3, L=600, w=128, ragged=(200, 600), seed=4),
@@ -121,7 +103,7 @@ STACKS = [
 @pytest.mark.parametrize("wl", STACKS, ids=[w.name for w in STACKS])
 def test_stack_matches_oracle(sc, wl, no_tail):
     inp, res, _ = resample_stack(wl)
-    _check_stack(wl, res, _run_stack(sc, wl, inp, no_tail))
+    check_stack(wl, res, _run_stack(sc, wl, inp, no_tail))
 
 
 def test_stack_theta_zero_keeps_everything(sc):
@@ -153,4 +135,4 @@ def test_stack_scattered_padding_uses_compacted_rows(sc):
     mask[:, inp["global_pos"]] = 1
     inp["pad_mask"] = mask
     res = oracle.stack(inp["Q"], inp["K"], inp["V"], mask, inp["global_pos"], wl.w, inp["alpha"])
-    _check_stack(wl, res, _run_stack(sc, wl, inp))
+    check_stack(wl, res, _run_stack(sc, wl, inp))

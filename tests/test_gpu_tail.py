@@ -16,8 +16,8 @@ import torch
 
 import oracle
 import workloads as wk
-from parity_utils import resample_stack
-from test_gpu_parity import _check_stack, _run_stack
+from parity_utils import check_stack, resample_stack
+from test_gpu_parity import _run_stack
 
 pytestmark = pytest.mark.gpu
 
@@ -52,7 +52,7 @@ TAIL_STACKS = [
 @pytest.mark.parametrize("wl", TAIL_STACKS, ids=[w.name for w in TAIL_STACKS])
 def test_tail_stack_matches_oracle(sc, wl):
     inp, res, _ = resample_stack(wl)
-    _check_stack(wl, res, _run_stack(sc, wl, inp))
+    check_stack(wl, res, _run_stack(sc, wl, inp))
 
 
 def test_handover_happens_mid_stack(sc):
@@ -84,7 +84,7 @@ def test_tail_empty_and_single_token_sequences(sc):
     got = _run_stack(sc, wl, inp)
     assert (got["len"][:, 0] == 0).all()
     assert (got["len"][:, 1] == 1).all()
-    _check_stack(wl, res, got)
+    check_stack(wl, res, got)
 
 
 def test_tail_theta_zero_keeps_everything(sc):
@@ -94,7 +94,7 @@ def test_tail_theta_zero_keeps_everything(sc):
     res = oracle.stack(inp["Q"], inp["K"], inp["V"], None, inp["global_pos"], wl.w, inp["alpha"])
     got = _run_stack(sc, wl, inp)
     assert (got["len"] == 256).all()
-    _check_stack(wl, res, got)
+    check_stack(wl, res, got)
 
 
 def test_launch_plan(sc):

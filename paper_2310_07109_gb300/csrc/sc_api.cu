@@ -21,7 +21,7 @@ cudaError_t configure_kernels();
 cudaError_t launch_rows(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_cols(const TensorMaps& m, const LayerParams& p, cudaStream_t st);
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st);
-cudaError_t launch_export(const ExportParams& e, cudaStream_t st);
+cudaError_t launch_export(const ExportParams& e, int ctas, cudaStream_t st);
 cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st);
 cudaError_t configure_tail();
 cudaError_t tail_max_clusters(int H, int* out);
@@ -782,6 +782,14 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   d.pos = reinterpret_cast<int32_t*>(ws + hl.pos);
   d.len = reinterpret_cast<int32_t*>(ws + hl.len);
   if ((rc = stack_forward_impl(&d, workspace, hl.O, stream, nullptr, 0, true)) != SC_OK) return rc;
+  bool use_tail = false, per_layer = true;
+  if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
+  int dev = 0, sms = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce == cudaSuccess) ce = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (ce != cudaSuccess) return fail_cuda("device attributes", ce);
+  WsLayout lay;
+  ws_layout(a->B, a->L, a->H, &lay);
   ExportParams e{};
   e.n_layers = a->n_layers; e.B = a->B; e.L = a->L; e.H = a->H;
   e.O = d.O; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
@@ -789,8 +797,18 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   e.hscores = static_cast<float*>(sc);
   e.hpos = static_cast<int32_t*>(ps);
   e.hlen = static_cast<int32_t*>(ln);
-  const cudaError_t ce = launch_export(e, static_cast<cudaStream_t>(stream));
-  if (ce != cudaSuccess) return fail_cuda("launch export kernel", ce);
+  e.tail_from = reinterpret_cast<const int32_t*>(ws + lay.tail_from);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (use_tail) {
+    // the per-layer results go out beside the cluster kernel, on the SMs it
+    // leaves idle (one CTA per SM fits beside one of its CTAs), the rest after it
+    e.part = 1;
+    if ((ce = launch_export(e, sms, st)) != cudaSuccess) return fail_cuda("launch export kernel", ce);
+    e.part = 2;
+  } else {
+    e.part = 0;
+  }
+  if ((ce = launch_export(e, 4 * sms, st)) != cudaSuccess) return fail_cuda("launch export kernel", ce);
   return SC_OK;
 }
 
@@ -804,7 +822,7 @@ int sc_stack_host_launch_count(const sc_stack_args* a, int* count) {
   if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
   int k = 2;   // padding removal / global lookup, and the export
   if (per_layer) k += 1 + 2 * a->n_layers + (a->n_layers - 1);
-  if (use_tail) k += 1;
+  if (use_tail) k += 2;   // the cluster kernel, and the export in two parts
   *count = k;
   return SC_OK;
 }

@@ -190,6 +190,11 @@ struct ExportParams {
   float* hscores;
   int32_t* hpos;
   int32_t* hlen;
+  // part 0: every layer.  With the cluster kernel, part 1 copies the layers
+  // l < tail_from[b], complete before that kernel, while it runs, and part 2
+  // the layers l >= tail_from[b] after it.
+  int part;
+  const int32_t* tail_from;    // [B] (parts 1 and 2)
 };
 
 struct TailParams {

@@ -28,6 +28,7 @@
 // The method (allowed sets, row softmax, vertical accumulation, >= threshold,
 // order-preserving removal) is Sec. "Sparse Attention", Sec. "Extractor of
 // Attention Scores in Sparse Attention Matrix" and Sec. "Token Pruning".
+#include <algorithm>
 #include <cuda_runtime.h>
 #include <utility>
 #include <cuda_bf16.h>
@@ -1359,44 +1360,55 @@ __global__ void __launch_bounds__(kGatherThreads)
 constexpr int kExportTokens = 32;
 constexpr int kExportThreads = 256;
 
-// One CTA per 32 current slots of one (layer, sequence): only the slots below
-// the layer's length are copied.  Loads from device memory are issued in
-// groups of four before the stores, which cross the host link.
+// Work items of 32 current slots of one (layer, sequence), walked by a
+// grid-stride loop; only the slots below the layer's length are copied.  Loads
+// from device memory are issued in groups of four before the stores, which
+// cross the host link.
 __global__ void __launch_bounds__(kExportThreads)
     sc_export_kernel(const ExportParams e) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int b = blockIdx.y, l = blockIdx.z;
-  const size_t li = static_cast<size_t>(l) * e.B + b;
-  const int n = __ldcg(e.len + li);
-  if (blockIdx.x == 0 && threadIdx.x == 0) e.hlen[li] = n;
-  const int c0 = blockIdx.x * kExportTokens;
-  if (c0 >= n) return;
-  const int cnt = min(kExportTokens, n - c0);
-  const size_t row0 = (static_cast<size_t>(l) * e.B + b) * e.L + c0;
-  if (threadIdx.x < cnt) {
-    e.hpos[row0 + threadIdx.x] = __ldcg(e.pos + row0 + threadIdx.x);
-    if (l < e.n_layers) e.hscores[row0 + threadIdx.x] = __ldcg(e.scores + row0 + threadIdx.x);
-  }
-  if (l >= e.n_layers) return;
+  // part 1 runs beside the cluster kernel, which lets it start once every one
+  // of its CTAs has passed its own grid wait: what part 1 reads is complete
+  if (e.part != 1) pdl_wait();
+  const int nch = (e.L + kExportTokens - 1) / kExportTokens;
+  const int items = (e.n_layers + 1) * e.B * nch;
   const int vec = e.H * kHeadDim / 8;   // 16-byte vectors per row
-  const int total = cnt * vec;
-  const uint4* src = reinterpret_cast<const uint4*>(e.O) + row0 * vec;
-  uint4* dst = reinterpret_cast<uint4*>(e.hO) + row0 * vec;
-  constexpr int kPer = 4;
-  for (int k0 = threadIdx.x; k0 < total; k0 += kExportThreads * kPer) {
-    uint4 v[kPer];
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int k = k0 + u * kExportThreads;
-      if (k < total) v[u] = __ldcg(src + k);
+  for (int it = blockIdx.x; it < items; it += gridDim.x) {
+    const int ch = it % nch, lb = it / nch;
+    const int b = lb % e.B, l = lb / e.B;
+    if (e.part != 0 && (e.part == 1) != (l < __ldcg(e.tail_from + b))) continue;
+    const size_t li = static_cast<size_t>(l) * e.B + b;
+    const int n = __ldcg(e.len + li);
+    if (ch == 0 && threadIdx.x == 0) e.hlen[li] = n;
+    const int c0 = ch * kExportTokens;
+    if (c0 >= n) continue;
+    const int cnt = min(kExportTokens, n - c0);
+    const size_t row0 = li * e.L + c0;
+    if (threadIdx.x < cnt) {
+      e.hpos[row0 + threadIdx.x] = __ldcg(e.pos + row0 + threadIdx.x);
+      if (l < e.n_layers) e.hscores[row0 + threadIdx.x] = __ldcg(e.scores + row0 + threadIdx.x);
     }
+    if (l >= e.n_layers) continue;
+    const int total = cnt * vec;
+    const uint4* src = reinterpret_cast<const uint4*>(e.O) + row0 * vec;
+    uint4* dst = reinterpret_cast<uint4*>(e.hO) + row0 * vec;
+    constexpr int kPer = 4;
+    for (int k0 = threadIdx.x; k0 < total; k0 += kExportThreads * kPer) {
+      uint4 v[kPer];
 #pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int k = k0 + u * kExportThreads;
-      if (k < total) dst[k] = v[u];
+      for (int u = 0; u < kPer; ++u) {
+        const int k = k0 + u * kExportThreads;
+        if (k < total) v[u] = __ldcg(src + k);
+      }
+#pragma unroll
+      for (int u = 0; u < kPer; ++u) {
+        const int k = k0 + u * kExportThreads;
+        if (k < total) dst[k] = v[u];
+      }
     }
   }
+  // part 1 completes only after the cluster kernel, so that part 2, which
+  // waits for part 1's grid, finds that kernel's results complete
+  if (e.part == 1) pdl_wait();
 }
 
 // ---------------------------------------------------------------------------
@@ -1590,9 +1602,10 @@ cudaError_t launch_advance(const AdvanceParams& a, cudaStream_t st) {
   return launch_chained(sc_advance_kernel, dim3(1), dim3(256), 0, st, a);
 }
 
-cudaError_t launch_export(const ExportParams& e, cudaStream_t st) {
-  dim3 grid((e.L + kExportTokens - 1) / kExportTokens, e.B, e.n_layers + 1);
-  return launch_chained(sc_export_kernel, grid, dim3(kExportThreads), 0, st, e);
+cudaError_t launch_export(const ExportParams& e, int ctas, cudaStream_t st) {
+  const int items = (e.n_layers + 1) * e.B * ((e.L + kExportTokens - 1) / kExportTokens);
+  return launch_chained(sc_export_kernel, dim3(std::max(1, std::min(items, ctas))),
+                        dim3(kExportThreads), 0, st, e);
 }
 
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {

@@ -128,8 +128,11 @@ __device__ __forceinline__ int round16(int x) { return (x + 15) & ~15; }
 
 __global__ void __launch_bounds__(kTailThreads, 1)
     sc_tail_kernel(const __grid_constant__ TailParams p) {
-  pdl_launch_dependents();
+  // the successor may start once every CTA is past its own grid wait, so it
+  // finds the kernels before this one complete (the export of the per-layer
+  // results runs beside this kernel)
   pdl_wait();
+  pdl_launch_dependents();
   const int H = p.H, w = p.w, L = p.L, B = p.B, n_layers = p.n_layers;
   const int h = static_cast<int>(blockIdx.x) % H, b = static_cast<int>(blockIdx.x) / H;
   // every CTA of the cluster reads the same values: the exits below are uniform

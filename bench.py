@@ -815,7 +815,7 @@ def run_encoder(args, wl):
             "e2e": {"value": whole_job_rate(world, kept_per_step, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": int(hostX.numel() * 2),
                     "d2h_bytes_per_step": int(hostY.numel() * 2), "ms_per_step": e2e_ms},
-            "gpu_launches": args.steps * nl * 9, "clocks": clocks.summary()}
+            "gpu_launches": args.steps * nl * 10, "clocks": clocks.summary()}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()

@@ -271,8 +271,8 @@ int sc_stack_host_launch_count(const sc_stack_args* args, int* count);
 int sc_workspace_status(void* workspace, size_t workspace_bytes, void* stream);
 
 /*
- * The encoder layer around the path (SURVEY "next": the steps either side of
- * the attention, Fig. "sparsecoder"): a RoBERTa-style post-LN layer whose
+ * The encoder layer around the path (the steps either side of the attention,
+ * Fig. "sparsecoder"): a RoBERTa-style post-LN layer whose
  * self-attention is the sparse attention with token pruning above, and whose
  * output projection and feed-forward block run on the kept tokens only.  D = 64 H.
  *
@@ -283,6 +283,9 @@ int sc_workspace_status(void* workspace, size_t workspace_bytes, void* stream);
  * LN(x) = (x - mean) / sqrt(var + 1e-5) * gamma + beta over the D features
  * (population variance); GELU(x) = x/2 (1 + erf(x / sqrt 2)).  Stored as bf16:
  * Q, K, V, O, H1, GELU's output, Y; S1 and the second sum stay fp32.
+ * Kernels per call: the Q/K/V GEMM, the attention layer's kernels, a copy of
+ * O's kept rows into consecutive rows, the output-projection GEMM (X[kept]
+ * gathered in its epilogue), layer norm, the two feed-forward GEMMs, layer norm.
  *
  * X          bf16 [B][L][D] hidden states in current order (row c of sequence b
  *            is current token c; rows at or beyond len[b] are never read).

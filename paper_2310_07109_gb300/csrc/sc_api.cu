@@ -29,6 +29,7 @@ cudaError_t launch_tail(const TailParams& p, cudaStream_t st);
 cudaError_t configure_encoder();
 cudaError_t launch_gemm(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_layernorm(const LayerNormParams& p, cudaStream_t st);
+cudaError_t launch_row_gather(const RowGatherParams& p, cudaStream_t st);
 }  // namespace sc
 
 namespace {
@@ -975,10 +976,10 @@ namespace {
 
 bool aligned_ptr16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// Fills the GEMM parameters and descriptors for out = act(A[gather] W^T + b) (+ res).
+// Fills the GEMM parameters and descriptors for out = act(A[a_idx] W^T + b) (+ res[res_idx]).
 int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, const int32_t* rows,
-              const int32_t* gidx, const uint16_t* W, const float* bias, int gelu,
-              const uint16_t* res, int res_gathered, void* out, int out_f32, int* status) {
+              const int32_t* a_idx, const uint16_t* W, const float* bias, int gelu,
+              const uint16_t* res, const int32_t* res_idx, void* out, int out_f32, int* status) {
   *g = GemmParams{};
   // 256-column tiles unless that leaves fewer than two tiles per SM (the row
   // count is a bound: rows are counted on the device) and A is not gathered
@@ -990,15 +991,15 @@ int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, cons
     sms = 152;
   }
   const long long row_tiles = static_cast<long long>(B) * ((L + kTile - 1) / kTile);
-  const int bn = (!gidx && row_tiles * ((N + 255) / 256) < 2ll * sms) ? 128 : 256;
+  const int bn = (!a_idx && row_tiles * ((N + 255) / 256) < 2ll * sms) ? 128 : 256;
   const int wbox = N < bn ? N : bn;
   if (!encode_2d(&g->map_a, A, static_cast<long long>(B) * L, K, 1) ||
       !encode_2d(&g->map_at, A, static_cast<long long>(B) * L, K, kTile) ||
       !encode_2d(&g->map_w, W, N, K, wbox))
     return SC_ERR_CUDA;
   g->B = B; g->L = L; g->N = N; g->K = K; g->bn = bn; g->wbox = wbox;
-  g->rows = rows; g->gidx = gidx; g->bias = bias; g->gelu = gelu;
-  g->res = res; g->res_gathered = res_gathered;
+  g->rows = rows; g->a_idx = a_idx; g->bias = bias; g->gelu = gelu;
+  g->res = res; g->res_idx = res_idx;
   g->out = out; g->out_f32 = out_f32; g->out_split = 0;
   g->status = status;
   return SC_OK;
@@ -1051,7 +1052,7 @@ extern "C" int sc_linear_forward(const sc_linear_args* a, void* workspace, size_
   if (rc != SC_OK) return rc;
   GemmParams g;
   if ((rc = make_gemm(&g, a->B, a->L, a->N, a->K, a->A, a->rows, a->gidx, a->W, a->bias, a->gelu,
-                      a->res, a->res_gathered, a->out, a->out_f32,
+                      a->res, a->res_gathered ? a->gidx : nullptr, a->out, a->out_f32,
                       static_cast<int*>(workspace))) != SC_OK)
     return rc;
   const cudaError_t e = launch_gemm(g, static_cast<cudaStream_t>(stream));
@@ -1109,8 +1110,8 @@ extern "C" int sc_encoder_layer_forward(const sc_encoder_args* a, void* workspac
 
   // Q, K, V of the current tokens: one GEMM, its column blocks split by tensor
   GemmParams g;
-  if ((rc = make_gemm(&g, B, L, 3 * D, D, a->X, a->len, nullptr, a->W_qkv, a->b_qkv, 0, nullptr, 0,
-                      nullptr, 0, status)) != SC_OK)
+  if ((rc = make_gemm(&g, B, L, 3 * D, D, a->X, a->len, nullptr, a->W_qkv, a->b_qkv, 0, nullptr,
+                      nullptr, nullptr, 0, status)) != SC_OK)
     return rc;
   g.out_split = D;
   g.outs[0] = Qb; g.outs[1] = Kb; g.outs[2] = Vb;
@@ -1128,20 +1129,24 @@ extern "C" int sc_encoder_layer_forward(const sc_encoder_args* a, void* workspac
   ws_layout(B, L, a->H, &lay);
   if ((rc = layer_forward_impl(&la, ws + el.attn, lay.total, stream, kept)) != SC_OK) return rc;
 
-  // S1 = X[kept] + O[kept] W_o^T + b_o (the compaction is this GEMM's row gather)
-  if ((rc = make_gemm(&g, B, L, D, D, a->O, a->len_out, kept, a->W_o, a->b_o, 0, a->X, 1, S, 1,
+  // S1 = X[kept] + O[kept] W_o^T + b_o: the kept rows of O are compacted once
+  // (into F's space, unused until the feed-forward block) so that the GEMM reads
+  // A with tiled copies; X[kept] is gathered row by row in its epilogue
+  RowGatherParams rg{B, L, D, a->len_out, kept, a->O, F};
+  if ((e = launch_row_gather(rg, st)) != cudaSuccess) return fail_cuda("launch row gather", e);
+  if ((rc = make_gemm(&g, B, L, D, D, F, a->len_out, nullptr, a->W_o, a->b_o, 0, a->X, kept, S, 1,
                       status)) != SC_OK)
     return rc;
   if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch output gemm", e);
   LayerNormParams ln{B, L, D, a->len_out, S, a->ln1_gamma, a->ln1_beta, 1e-5f, H1};
   if ((e = launch_layernorm(ln, st)) != cudaSuccess) return fail_cuda("launch layer norm 1", e);
   // the feed-forward block on the kept tokens
-  if ((rc = make_gemm(&g, B, L, 4 * D, D, H1, a->len_out, nullptr, a->W_1, a->b_1, 1, nullptr, 0, F,
-                      0, status)) != SC_OK)
+  if ((rc = make_gemm(&g, B, L, 4 * D, D, H1, a->len_out, nullptr, a->W_1, a->b_1, 1, nullptr,
+                      nullptr, F, 0, status)) != SC_OK)
     return rc;
   if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch ffn gemm 1", e);
-  if ((rc = make_gemm(&g, B, L, D, 4 * D, F, a->len_out, nullptr, a->W_2, a->b_2, 0, H1, 0, S, 1,
-                      status)) != SC_OK)
+  if ((rc = make_gemm(&g, B, L, D, 4 * D, F, a->len_out, nullptr, a->W_2, a->b_2, 0, H1, nullptr,
+                      S, 1, status)) != SC_OK)
     return rc;
   if ((e = launch_gemm(g, st)) != cudaSuccess) return fail_cuda("launch ffn gemm 2", e);
   ln.gamma = a->ln2_gamma; ln.beta = a->ln2_beta; ln.out = a->Y;

@@ -134,10 +134,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int k = 0; k < 4; ++k) {
         const int r = g.r0 + 4 * lane + k;
         const int src =
-            r < g.rows ? (p.gidx ? __ldcg(p.gidx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
+            r < g.rows ? (p.a_idx ? __ldcg(p.a_idx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
         ar[k] = g.b * p.L + src;
       }
-      const bool gather = p.gidx != nullptr;
+      const bool gather = p.a_idx != nullptr;
       for (int kt = 0; ok && kt < ksteps; ++kt) {
         if (use > 0 && !(ok = warp_wait_gemm(&sm.empty[s], (use - 1) & 1, abort_flag))) break;
         uint8_t* As = base + s * kGemmStageBytes;
@@ -218,8 +218,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const int r = g.r0 + 32 * q + lane;
       const bool valid = ok && r < g.rows;
       const size_t orow = static_cast<size_t>(g.b) * p.L + r;
-      const int rsrc = valid ? (p.res_gathered && p.gidx
-                                    ? __ldcg(p.gidx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
+      const int rsrc =
+          valid ? (p.res_idx ? __ldcg(p.res_idx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
       const uint16_t* res =
           p.res ? p.res + (static_cast<size_t>(g.b) * p.L + rsrc) * p.N + g.n0 : nullptr;
       int nb = g.n0, ldo = p.N;
@@ -289,6 +289,44 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tmem_dealloc(tm, 512);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------------------
+// row gather: the kept rows of a bf16 matrix, consecutive (8 rows per CTA,
+// 16-byte vectors, every load of a thread issued before its stores)
+// ---------------------------------------------------------------------------
+constexpr int kRgRows = 8;
+constexpr int kRgThreads = 256;
+
+__global__ void __launch_bounds__(kRgThreads)
+    sc_row_gather_kernel(const __grid_constant__ RowGatherParams p) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int b = blockIdx.y, r0 = blockIdx.x * kRgRows;
+  const int n = __ldcg(p.rows + b);
+  if (r0 >= n) return;
+  const int cnt = min(kRgRows, n - r0);
+  const int vec = p.D / 8;
+  const int total = cnt * vec;
+  constexpr int kPer = 4;
+  const size_t base = static_cast<size_t>(b) * p.L;
+  for (int k0 = threadIdx.x; k0 < total; k0 += kRgThreads * kPer) {
+    uint4 v[kPer];
+    size_t dofs[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int k = k0 + u * kRgThreads;
+      if (k < total) {
+        const int rr = k / vec, e = k - rr * vec;
+        const int src = __ldcg(p.idx + base + r0 + rr);
+        v[u] = __ldcg(reinterpret_cast<const uint4*>(p.src + (base + src) * p.D) + e);
+        dofs[u] = (base + r0 + rr) * vec + e;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u)
+      if (k0 + u * kRgThreads < total) reinterpret_cast<uint4*>(p.dst)[dofs[u]] = v[u];
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -372,6 +410,11 @@ cudaError_t launch_gemm(const GemmParams& p, cudaStream_t st) {
                           ((p.N + p.bn - 1) / p.bn);
   const unsigned grid = static_cast<unsigned>(tiles < sms ? tiles : sms);
   return launch_pdl(sc_gemm_kernel, dim3(grid), dim3(kGemmThreads), kGemmDyn, st, p);
+}
+
+cudaError_t launch_row_gather(const RowGatherParams& p, cudaStream_t st) {
+  dim3 grid((p.L + kRgRows - 1) / kRgRows, p.B);
+  return launch_pdl(sc_row_gather_kernel, grid, dim3(kRgThreads), 0, st, p);
 }
 
 cudaError_t launch_layernorm(const LayerNormParams& p, cudaStream_t st) {

@@ -216,9 +216,9 @@ struct TailParams {
 };
 
 // One GEMM of the encoder layer: out[(b, r)][n] = epi(sum_k A[row_a][k] W[n][k])
-// for r < rows[b], row_a = b L + (gidx ? gidx[b L + r] : r); epi adds bias[n],
-// then GELU (gelu != 0), then the bf16 residual res[row][n] (row = row_a when
-// res_gathered, else b L + r).  N % 128 == 0, K % 64 == 0; 128 x 256 tiles.
+// for r < rows[b], row_a = b L + (a_idx ? a_idx[b L + r] : r); epi adds bias[n],
+// then GELU (gelu != 0), then the bf16 residual res[row][n] (row = b L +
+// (res_idx ? res_idx[b L + r] : r)).  N % 128 == 0, K % 64 == 0; 128 x 256 tiles.
 struct GemmParams {
   CUtensorMap map_a;               // 2-D [B L][K] bf16, box 64 x 1 (four-row gathers)
   CUtensorMap map_at;              // the same matrix, box 64 x 128 (consecutive rows)
@@ -228,11 +228,11 @@ struct GemmParams {
                                    // too few tiles for the SMs
   int wbox;                        // W rows per copy: min(bn, N)
   const int32_t* rows;             // [B] rows per sequence, or nullptr (L)
-  const int32_t* gidx;             // [B][L] A row of output row (b, r), or nullptr
+  const int32_t* a_idx;            // [B][L] A row of output row (b, r), or nullptr
   const float* bias;               // [N] or nullptr
   int gelu;
   const uint16_t* res;             // bf16 [B L][N] or nullptr
-  int res_gathered;
+  const int32_t* res_idx;          // [B][L] residual row of output row (b, r), or nullptr
   void* out;                       // [B L][N], bf16 or fp32 (out_f32)
   int out_f32;
   int out_split;                   // > 0: column block j of width out_split goes to outs[j]
@@ -241,6 +241,16 @@ struct GemmParams {
 };
 
 // Layer norm over D features of the rows (b, r), r < rows[b]: fp32 in, bf16 out.
+// Rows of a bf16 [B L][D] matrix gathered into consecutive rows:
+// dst[b L + r] = src[b L + idx[b L + r]] for r < rows[b].
+struct RowGatherParams {
+  int B, L, D;
+  const int32_t* rows;             // [B]
+  const int32_t* idx;              // [B][L]
+  const uint16_t* src;
+  uint16_t* dst;
+};
+
 struct LayerNormParams {
   int B, L, D;
   const int32_t* rows;

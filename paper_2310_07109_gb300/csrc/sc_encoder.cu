@@ -345,6 +345,44 @@ __global__ void __launch_bounds__(kLnThreads)
   const int b = static_cast<int>(row / p.L), r = static_cast<int>(row % p.L);
   if (r >= (p.rows ? min(__ldcg(p.rows + b), p.L) : p.L)) return;
   const float* x = p.in + row * p.D;
+  uint16_t* y = p.out + row * p.D;
+  if (p.vec) {
+    // lane covers features 4 lane + 128 k .. + 3: 16-byte loads, 8-byte stores
+    constexpr int kMaxChunks = kLnMaxPer / 4;
+    const int chunks = p.D / 128;
+    float4 v[kMaxChunks];
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxChunks; ++k) {
+      v[k] = k < chunks ? __ldcg(reinterpret_cast<const float4*>(x) + lane + 32 * k)
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+      s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
+    }
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    const float mean = s / static_cast<float>(p.D);
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < kMaxChunks; ++k)
+      if (k < chunks) {
+        const float a = v[k].x - mean, b2 = v[k].y - mean, c = v[k].z - mean, d = v[k].w - mean;
+        q += (a * a + b2 * b2) + (c * c + d * d);
+      }
+    for (int off = 16; off > 0; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
+    const float inv = 1.f / sqrtf(q / static_cast<float>(p.D) + p.eps);
+#pragma unroll
+    for (int k = 0; k < kMaxChunks; ++k)
+      if (k < chunks) {
+        const int f4 = lane + 32 * k;
+        const float4 g = __ldg(reinterpret_cast<const float4*>(p.gamma) + f4);
+        const float4 be = __ldg(reinterpret_cast<const float4*>(p.beta) + f4);
+        const uint2 o = make_uint2(pack_bf16x2((v[k].x - mean) * inv * g.x + be.x,
+                                               (v[k].y - mean) * inv * g.y + be.y),
+                                   pack_bf16x2((v[k].z - mean) * inv * g.z + be.z,
+                                               (v[k].w - mean) * inv * g.w + be.w));
+        reinterpret_cast<uint2*>(y)[f4] = o;
+      }
+    return;
+  }
   const int per = p.D / 32;   // features of this lane: lane, lane + 32, ...
   float v[kLnMaxPer];
   float s = 0.f;
@@ -364,7 +402,6 @@ __global__ void __launch_bounds__(kLnThreads)
     }
   for (int off = 16; off > 0; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
   const float inv = 1.f / sqrtf(q / static_cast<float>(p.D) + p.eps);
-  uint16_t* y = p.out + row * p.D;
 #pragma unroll
   for (int k = 0; k < kLnMaxPer; ++k)
     if (k < per) {
@@ -420,7 +457,11 @@ cudaError_t launch_row_gather(const RowGatherParams& p, cudaStream_t st) {
 cudaError_t launch_layernorm(const LayerNormParams& p, cudaStream_t st) {
   const long long rows = static_cast<long long>(p.B) * p.L;
   const unsigned blocks = static_cast<unsigned>((rows + kLnThreads / 32 - 1) / (kLnThreads / 32));
-  return launch_pdl(sc_layernorm_kernel, dim3(blocks), dim3(kLnThreads), 0, st, p);
+  auto al = [](const void* q, unsigned a) { return (reinterpret_cast<uintptr_t>(q) % a) == 0; };
+  LayerNormParams q = p;
+  q.vec = (p.D % 128 == 0 && al(p.in, 16) && al(p.gamma, 16) && al(p.beta, 16) && al(p.out, 8))
+              ? 1 : 0;
+  return launch_pdl(sc_layernorm_kernel, dim3(blocks), dim3(kLnThreads), 0, st, q);
 }
 
 }  // namespace sc

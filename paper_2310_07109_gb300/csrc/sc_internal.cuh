@@ -259,6 +259,7 @@ struct LayerNormParams {
   const float* beta;
   float eps;
   uint16_t* out;
+  int vec;   // set by the launcher: D % 128 == 0 and aligned rows (4 features per access)
 };
 
 }  // namespace sc

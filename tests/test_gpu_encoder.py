@@ -83,9 +83,12 @@ def test_linear_matches_oracle(sc, B, L, rows, N, K, gather, gelu, res, res_g, o
         assert np.isnan(got[b * L + n:(b + 1) * L]).all(), "rows past the sequence were written"
 
 
-def test_layer_norm_matches_oracle(sc):
-    rng = np.random.default_rng(7)
-    B, L, D = 2, 200, 768
+@pytest.mark.parametrize("D", [768, 128, 96, 1024], ids=lambda d: f"D{d}")
+def test_layer_norm_matches_oracle(sc, D):
+    """D a multiple of 128 takes the four-features-per-access path, D = 96 the
+    one-feature path."""
+    rng = np.random.default_rng(7 + D)
+    B, L = 2, 200
     x = (rng.standard_normal((B * L, D)) * 2.5 + 0.7).astype(np.float32)
     g = (1 + 0.1 * rng.standard_normal(D)).astype(np.float32)
     be = (0.1 * rng.standard_normal(D)).astype(np.float32)

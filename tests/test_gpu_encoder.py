@@ -83,6 +83,25 @@ def test_linear_matches_oracle(sc, B, L, rows, N, K, gather, gelu, res, res_g, o
         assert np.isnan(got[b * L + n:(b + 1) * L]).all(), "rows past the sequence were written"
 
 
+def test_gelu_epilogue_accuracy(sc):
+    """The GEMM's GELU (erf by Abramowitz & Stegun 7.1.26, |error| <= 1.5e-7)
+    against the fp64 definition: a 0/1 selector weight makes each fp32 output
+    GELU of one bf16 input exactly, so only the GELU's own error remains."""
+    K, N, M = 64, 128, 512
+    x = _bf16(np.linspace(-9.0, 9.0, M * K).reshape(M, K))
+    x[0, :8] = [0.0, -0.0, 1e-3, -1e-3, 2.0 ** -20, -(2.0 ** -20), 40.0, -40.0]
+    W = np.zeros((N, K))
+    W[np.arange(N), np.arange(N) % K] = 1.0
+    out = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    sc.linear_forward(_t_bf16(x), _t_bf16(W), B=1, L=M, bias=None, gelu=True, out=out,
+                      out_f32=True)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy().astype(np.float64)
+    want = enc.gelu(x[:, np.arange(N) % K])
+    err = np.abs(got - want)
+    assert (err <= 2e-6 * np.maximum(1.0, np.abs(want))).all(), err.max()
+
+
 @pytest.mark.parametrize("D", [768, 128, 96, 1024], ids=lambda d: f"D{d}")
 def test_layer_norm_matches_oracle(sc, D):
     """D a multiple of 128 takes the four-features-per-access path, D = 96 the

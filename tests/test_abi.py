@@ -181,19 +181,20 @@ def test_stack_host_workspace_size(lib):
 def test_launch_count_rejects_bad_arguments(lib):
     g = (ctypes.c_int32 * 1)(0)
 
-    def count(**kw):
+    def count(fn, **kw):
         a = dict(n_layers=12, B=2, L=1024, H=12, w=256, Q=None, K=None, V=None, pad_mask=None,
                  global_pos=ctypes.cast(g, ctypes.POINTER(ctypes.c_int32)), n_global=1,
                  alpha=None, O=None, scores=None, pos=None, len=None)
         a.update(kw)
         c = ctypes.c_int(-1)
-        return lib.sc_stack_launch_count(ctypes.byref(bd.StackArgs(**a)), ctypes.byref(c))
+        return fn(ctypes.byref(bd.StackArgs(**a)), ctypes.byref(c))
 
-    assert count(n_layers=0) == bd.SC_ERR_INVALID_ARG
-    assert count(flags=4) == bd.SC_ERR_INVALID_ARG
-    assert count(L=8192) == bd.SC_ERR_UNSUPPORTED
-    assert count(B=0) == bd.SC_ERR_INVALID_ARG
-    assert lib.sc_stack_launch_count(None, None) == bd.SC_ERR_INVALID_ARG
+    for fn in (lib.sc_stack_launch_count, lib.sc_stack_host_launch_count):
+        assert count(n_layers=0, fn=fn) == bd.SC_ERR_INVALID_ARG
+        assert count(flags=4, fn=fn) == bd.SC_ERR_INVALID_ARG
+        assert count(L=8192, fn=fn) == bd.SC_ERR_UNSUPPORTED
+        assert count(B=0, fn=fn) == bd.SC_ERR_INVALID_ARG
+        assert fn(None, None) == bd.SC_ERR_INVALID_ARG
 
 
 def test_encoder_calls_reject_bad_arguments(lib):

@@ -320,7 +320,9 @@ def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, wor
     ``stack_forward``.  ``out``: page-locked result tensors (``new_host_outputs``);
     only the current slots of each layer (and all of ``len``) are written.
     The call is asynchronous on ``stream`` (default: torch's current stream of the
-    current device): synchronise before reading ``out``.
+    current device): synchronise before reading ``out``.  The first call on newly
+    page-locked buffers is slower (milliseconds) while the device maps their pages;
+    reuse the buffers across calls.
     Returns the dict of host tensors O, scores, pos, len.
     """
     nl, B, L, H, D = Q.shape

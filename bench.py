@@ -145,6 +145,20 @@ def kernel_source_hash() -> str:
     return h.hexdigest()
 
 
+def host_link_bytes(lens, n_layers, H, d, mask_bytes):
+    """Bytes one sc_stack_forward_host call moves over the host link, from the
+    lengths it produced (lens [n_layers + 1][B]): host to device, the Q, K, V
+    rows of the tokens entering each layer and the padding mask; device to host,
+    those tokens' O rows and scores, pos[l][b][:len] for every l <= n_layers,
+    and len itself."""
+    lens = np.asarray(lens, dtype=np.int64)
+    row_bytes = H * d * 2
+    in_rows = int(lens[:n_layers].sum())
+    h2d = 3 * row_bytes * in_rows + int(mask_bytes)
+    d2h = (row_bytes + 4) * in_rows + 4 * int(lens.sum()) + 4 * lens.size
+    return h2d, d2h
+
+
 def measured_traffic(kernels):
     """DRAM bytes (read + write) of one launch of each kernel, summed, from the ncu
     capture recorded in profiles/traffic.json; None once any kernel source has
@@ -586,12 +600,8 @@ def run_native(args, wl):
         raise SystemExit("device status after the end-to-end steps: %s" % sc.status_string(rc))
     if not torch.equal(hout["len"], out["len"].cpu()):
         raise SystemExit("the host-buffer call disagrees with the device call on the lengths")
-    # bytes that crossed the host link per step: the rows each layer read, the
-    # padding mask, and the defined result slots written back
-    row_bytes = wl.H * wl.d * 2
-    in_rows = int(lens[:wl.n_layers].sum())
-    h2d = 3 * row_bytes * in_rows + (0 if hmask is None else hmask.numel())
-    d2h = (row_bytes + 4) * in_rows + 4 * int(lens.sum()) + 4 * lens.size
+    h2d, d2h = host_link_bytes(lens, wl.n_layers, wl.H, wl.d,
+                               0 if hmask is None else hmask.numel())
     e2e = {"value": whole_job_rate(world, kept_per_step, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
            "ms_per_step": e2e_ms, "call": "sc_stack_forward_host",

@@ -47,3 +47,16 @@ def test_two_gloo_ranks_take_the_slowest_time():
 def test_single_process_needs_no_group():
     assert bench.max_over_ranks(3.0) == 3.0
     assert bench.whole_job_rate(1, 10, 2.0) == pytest.approx(5000.0)
+
+
+def test_host_link_bytes_counts_the_defined_slots():
+    """Two layers, two sequences: the rows entering each layer go in (Q, K, V),
+    their O rows and scores come back, pos for every layer and len."""
+    import bench
+    lens = [[5, 3], [2, 3], [1, 0]]       # len[l][b], l = 0..2
+    H, d = 2, 64
+    row = H * d * 2                       # one bf16 row of one tensor
+    h2d, d2h = bench.host_link_bytes(lens, 2, H, d, mask_bytes=16)
+    entering = 5 + 3 + 2 + 3              # layers 0 and 1
+    assert h2d == 3 * row * entering + 16
+    assert d2h == entering * (row + 4) + 4 * (5 + 3 + 2 + 3 + 1 + 0) + 4 * 6

@@ -17,7 +17,14 @@ import torch
 import oracle
 import workloads as wk
 from oracle import encoder as enc
-from parity_utils import O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, torch_bf16_to_f64
+from parity_utils import (O_ATOL, SCORE_ATOL, bits_to_torch, check_o, check_scores,
+                          torch_bf16_to_f64)
+
+# The stages around the attention (GEMM outputs, the layer output Y) are not
+# attention outputs: their values reach several units, where the bf16 storage
+# rounding alone is half an ulp = 2^-9 |y|; their bar adds that rounding and one
+# more of the same size for a bf16 operand rounded inside the stage.
+STAGE_RTOL = 2.0 ** -8
 
 pytestmark = pytest.mark.gpu
 
@@ -78,7 +85,7 @@ def test_linear_matches_oracle(sc, B, L, rows, N, K, gather, gelu, res, res_g, o
         if res:
             y = y + R[src if res_g else b * L + np.arange(n)]
         g = got[b * L:b * L + n]
-        tol = (1e-4 * np.abs(y).max(), 0) if out_f32 else (O_ATOL / 4, O_RTOL)
+        tol = (1e-4 * np.abs(y).max(), 0) if out_f32 else (O_ATOL / 4, STAGE_RTOL)
         np.testing.assert_allclose(g, y, atol=tol[0], rtol=tol[1], err_msg=f"sequence {b}")
         assert np.isnan(got[b * L + n:(b + 1) * L]).all(), "rows past the sequence were written"
 
@@ -167,8 +174,8 @@ def _check_layer(sc, X, lens, pos, w64, wdev, L, H, wwin, gpos, alpha):
         isg = np.array([int(p) in gset for p in pos[b, :n]])
         Oe, se, keep_e = oracle.layer(q.reshape(n, H, 64), k.reshape(n, H, 64),
                                       v.reshape(n, H, 64), isg, wwin, theta)
-        np.testing.assert_allclose(O[b, :n], Oe.reshape(n, D), rtol=O_RTOL, atol=O_ATOL)
-        np.testing.assert_allclose(s[b, :n], se, rtol=0, atol=SCORE_ATOL)
+        check_o(O[b, :n], Oe.reshape(n, D), f"sequence {b}")
+        check_scores(s[b, :n], se, f"sequence {b}")
         # the kept list: the kernels' own decision on their own scores, and the
         # oracle's wherever its score is clear of the threshold
         keep_g = (np.arange(n) == 0) | (s[b, :n] >= np.float32(alpha) / np.float32(n))
@@ -182,7 +189,7 @@ def _check_layer(sc, X, lens, pos, w64, wdev, L, H, wwin, gpos, alpha):
         r = enc.output_and_ffn(X[b, kc], O[b, kc], w64["W_o"], w64["b_o"], w64["ln1_gamma"],
                                w64["ln1_beta"], w64["W_1"], w64["b_1"], w64["W_2"], w64["b_2"],
                                w64["ln2_gamma"], w64["ln2_beta"], round_h1=_bf16, round_f=_bf16)
-        np.testing.assert_allclose(Y[b, :len(kc)], r["Y"], rtol=O_RTOL, atol=O_ATOL,
+        np.testing.assert_allclose(Y[b, :len(kc)], r["Y"], rtol=STAGE_RTOL, atol=O_ATOL,
                                    err_msg=f"sequence {b}")
     return Y, po, lo
 

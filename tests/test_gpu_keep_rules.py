@@ -15,7 +15,7 @@ import torch
 
 import oracle
 import workloads as wk
-from parity_utils import (MARGIN, O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, check_stack,
+from parity_utils import (MARGIN, bits_to_torch, check_o, check_scores, check_stack,
                           resample_stack, torch_bf16_to_f64)
 from test_gpu_parity import _run_stack
 
@@ -140,5 +140,5 @@ def test_layer_call_top_ratio(sc):
         Oe, se, kept = exp[b]
         assert lo[b] == len(kept)
         assert list(po[b, :len(kept)]) == list(kept)
-        np.testing.assert_allclose(O[b, :n], Oe, rtol=O_RTOL, atol=O_ATOL)
-        np.testing.assert_allclose(s[b, :n], se, rtol=0, atol=SCORE_ATOL)
+        check_o(O[b, :n], Oe, f"sequence {b}")
+        check_scores(s[b, :n], se, f"sequence {b}")

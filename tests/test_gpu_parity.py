@@ -10,7 +10,7 @@ import pytest
 import torch
 
 import workloads as wk
-from parity_utils import (O_ATOL, O_RTOL, SCORE_ATOL, bits_to_torch, check_stack, layer_case,
+from parity_utils import (bits_to_torch, check_o, check_scores, check_stack, layer_case,
                           resample_stack, torch_bf16_to_f64)
 
 pytestmark = pytest.mark.gpu
@@ -46,8 +46,8 @@ def _check_layer(case, got):
         assert list(po[b, :len(kept)]) == kept, f"sequence {b}: kept positions"
         if n == 0:
             continue
-        np.testing.assert_allclose(O[b, :n], Oe, rtol=O_RTOL, atol=O_ATOL)
-        np.testing.assert_allclose(s[b, :n], se, rtol=0, atol=SCORE_ATOL)
+        check_o(O[b, :n], Oe, f"sequence {b}")
+        check_scores(s[b, :n], se, f"sequence {b}")
         assert abs(float(s[b, :n].astype(np.float64).sum()) - 1.0) < 1e-4
 
 

@@ -410,3 +410,39 @@ def test_resampling_clears_the_keep_decision(rule, values):
                     assert srt[kept - 1] - srt[kept] >= 2 * MARGIN / n
             else:
                 assert (np.abs(s - inp["alpha"][l]) >= MARGIN / n).all()
+
+
+@pytest.mark.parametrize("wl", [
+    wk.Workload("rs_rel", n_layers=4, B=3, L=200, H=2, w=20, n_extra_global=3, seed=31),
+    wk.Workload("rs_ragged", n_layers=3, B=3, L=180, H=3, w=16, ragged=(60, 180), seed=32),
+    wk.Workload("rs_abs", n_layers=3, B=2, L=150, H=2, w=12, alpha_first=0.004,
+                alpha_last=0.012, keep_rule=oracle.KEEP_ABSOLUTE, seed=33),
+    wk.Workload("rs_top", n_layers=3, B=2, L=150, H=2, w=12, alpha_first=0.9,
+                alpha_last=0.6, keep_rule=oracle.KEEP_TOP_RATIO, seed=34),
+], ids=lambda w: w.name)
+def test_resampled_results_equal_the_oracle_stack(wl):
+    """The resampler's layer-by-layer results are those of the oracle's own
+    stack driver on the final (redrawn) inputs, and the redraws are exactly
+    what make_inputs reproduces from the returned redraw counts."""
+    from parity_utils import resample_stack
+    inp, res, redraws = resample_stack(wl)
+    again = wk.make_inputs(wl, redraws)
+    for t in ("Q", "K", "V"):
+        np.testing.assert_array_equal(again[t], inp[t])
+    ref = oracle.stack(inp["Q"], inp["K"], inp["V"], inp["pad_mask"], inp["global_pos"], wl.w,
+                       inp["alpha"], keep_rule=wl.keep_rule)
+    np.testing.assert_array_equal(res["len"], ref["len"])
+    np.testing.assert_array_equal(res["pos"], ref["pos"])
+    np.testing.assert_array_equal(res["scores"], ref["scores"])
+    np.testing.assert_array_equal(res["O"], ref["O"])
+
+
+def test_stored_redraws_clear_the_benchmark_workload():
+    """The benchmark times config 4 with the redraws stored in
+    tests/golden/redraws.json: starting from them the resampler finds no token
+    of any layer within the margin of its threshold, so they are complete."""
+    from parity_utils import resample_stack
+    stored = wk.stored_redraws(wk.CFG4)
+    assert stored, "no stored redraws for the benchmark workload"
+    _, _, redraws = resample_stack(wk.CFG4, redraws=stored, o_dtype=np.float32)
+    assert redraws == stored

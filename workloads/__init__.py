@@ -22,6 +22,9 @@ from __future__ import annotations
 from dataclasses import dataclass, replace
 from typing import Dict, Optional, Tuple
 
+import json
+import os
+
 import numpy as np
 
 HEAD_DIM = 64
@@ -198,16 +201,24 @@ def make_inputs(wl: Workload, redraws: Optional[Dict[Tuple[int, int, int], int]]
             Q[l, b] = f32_to_bf16_bits(q)
             K[l, b] = f32_to_bf16_bits(k)
             V[l, b] = f32_to_bf16_bits(v)
+    inp = {"Q": Q, "K": K, "V": V, "pad_mask": pad_mask(wl),
+           "global_pos": global_positions(wl), "alpha": wl.alphas(), "salient": sal}
     for (l, b, p), cnt in (redraws or {}).items():
-        g = _rng(wl.seed, _TAG_REDRAW, l, b, p, cnt)
-        q = g.standard_normal((H, d), dtype=np.float32)
-        k = g.standard_normal((H, d), dtype=np.float32)
-        if sal[b, p]:
-            k *= np.float32(wl.salient_scale)
-        Q[l, b, p] = f32_to_bf16_bits(q)
-        K[l, b, p] = f32_to_bf16_bits(k)
-    return {"Q": Q, "K": K, "V": V, "pad_mask": pad_mask(wl),
-            "global_pos": global_positions(wl), "alpha": wl.alphas(), "salient": sal}
+        redraw_row(wl, inp, l, b, p, cnt)
+    return inp
+
+
+def redraw_row(wl: Workload, inp, l: int, b: int, p: int, cnt: int) -> None:
+    """Replace, in place, the Q and K rows of token ``p`` of sequence ``b`` at
+    layer ``l`` in ``inp`` (from ``make_inputs``) by draw number ``cnt`` of its
+    redraw stream (V is kept; a salient token's key row keeps its scale)."""
+    g = _rng(wl.seed, _TAG_REDRAW, l, b, p, cnt)
+    q = g.standard_normal((wl.H, wl.d), dtype=np.float32)
+    k = g.standard_normal((wl.H, wl.d), dtype=np.float32)
+    if inp["salient"][b, p]:
+        k *= np.float32(wl.salient_scale)
+    inp["Q"][l, b, p] = f32_to_bf16_bits(q)
+    inp["K"][l, b, p] = f32_to_bf16_bits(k)
 
 
 def random_layer(n: int, H: int, d: int, seed: int, scale_k: float = 1.0):
@@ -244,3 +255,26 @@ def encoder_input(wl: Workload):
     """Layer-0 hidden states: bf16 bits [B, L, D], N(0, 1)."""
     g = _rng(wl.seed, _TAG_HIDDEN)
     return f32_to_bf16_bits(g.standard_normal((wl.B, wl.L, wl.H * wl.d), dtype=np.float32))
+
+
+# ---------------------------------------------------------------------------
+# stored redraws: the near-threshold resampling of each named workload, found
+# by the oracle (tests/golden/make_redraws.py writes the file; nothing here
+# computes them)
+# ---------------------------------------------------------------------------
+_REDRAWS_FILE = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                             "tests", "golden", "redraws.json")
+
+
+def stored_redraws(wl: Workload) -> Dict[Tuple[int, int, int], int]:
+    """{(layer, sequence, original position): redraw count} stored for ``wl``
+    (matched by name and seed), or {} when the file has no entry for it."""
+    try:
+        with open(_REDRAWS_FILE) as f:
+            table = json.load(f)
+    except FileNotFoundError:
+        return {}
+    entry = table.get(wl.name)
+    if entry is None or entry.get("seed") != wl.seed:
+        return {}
+    return {tuple(int(x) for x in k.split(",")): int(c) for k, c in entry["redraws"].items()}

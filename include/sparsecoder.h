@@ -135,7 +135,8 @@ typedef struct {
  *            theta_{l,b} = alpha[l] / n_{l,b} (SC_KEEP_RELATIVE), theta_l =
  *            alpha[l] (SC_KEEP_ABSOLUTE) or the kept ratio rho_l
  *            (SC_KEEP_TOP_RATIO; finite).
- * O          bf16 [n_layers][B][L][H][64] out (current slots of each layer).
+ * O          bf16 [n_layers][B][L][H][64] out (current slots of each layer), or
+ *            NULL: then no layer's O is written but the last layer's, to O_last.
  * scores     float [n_layers][B][L] out.
  * pos        int32 [n_layers+1][B][L] out: pos[0] = real tokens after padding
  *            removal, pos[l+1] = survivors of layer l.
@@ -143,6 +144,11 @@ typedef struct {
  * flags      0, or SC_STACK_NO_TAIL: run every layer of every sequence through
  *            the per-layer kernels (see sc_stack_forward).
  * keep_rule  an sc_keep_rule (0 = SC_KEEP_RELATIVE), the same for every layer.
+ * O_last     used only when O is NULL: bf16 [B][L][H][64] out, the last layer's
+ *            O at its current slots; or NULL as well (no O is written at all,
+ *            which saves the 1536 bytes per token and layer of O stores).
+ *            Earlier layers' O is not needed to decide the kept tokens, whose
+ *            scores come from the probabilities alone (Sec. "Token Pruning").
  */
 #define SC_STACK_NO_TAIL 1
 
@@ -161,6 +167,7 @@ typedef struct {
   int32_t* len;
   int flags;
   int keep_rule;
+  uint16_t* O_last;
 } sc_stack_args;
 
 /*
@@ -175,16 +182,32 @@ typedef struct {
  * Same arguments, semantics and results as sc_layer_forward (the caller still
  * passes every input and output).  The scratch comes from a 6 MiB array
  * compiled into the library, which every GPU that loads it holds until the
- * process exits; sizes whose scratch does not fit (from roughly B*L*H = 130k
+ * process exits; sizes whose scratch does not fit (from roughly B*L*H = 100k
  * (sequence, token, head) rows on; B=2, L=4096, H=12 is 98k and fits) return
  * SC_ERR_UNSUPPORTED with the detail in sc_last_error().  The first call
  * on each device looks up the array's device address (cudaGetSymbolAddress);
  * make that first call before any stream capture.  All calls share the array:
  * calls that overlap on the GPU (different streams, without ordering) race.
- * A bounded-wait timeout cannot be queried for this entry point: its status
- * word is private and cleared at every call.
+ * A bounded wait that expires in any call is recorded in the array's status
+ * word, which keeps it until sc_layer_noalloc_status() reads it.
  */
 int sc_layer_forward_noalloc(const sc_layer_args* args, void* stream);
+
+/* Synchronises `stream`, returns SC_ERR_TIMEOUT if a bounded wait expired in a
+ * sc_layer_forward_noalloc call on the current device since the last query
+ * (else SC_OK, or SC_ERR_CUDA), and clears the word.  Allocates nothing. */
+int sc_layer_noalloc_status(void* stream);
+
+/* Test hook of the failure path; not for production use.  While ns > 0, the
+ * first MMA-issuing thread of every CTA of the per-layer attention kernel
+ * (sc_layer_forward, sc_layer_forward_noalloc and the per-layer part of the
+ * stacks) first waits at most ns nanoseconds on a barrier that nothing
+ * completes.  That bounded wait expires: the CTA abandons its work, drains
+ * its copies and matrix products, frees its tensor memory and records
+ * SC_ERR_TIMEOUT in the status word, so the call's results are undefined and
+ * the status query reports SC_ERR_TIMEOUT.  ns = 0 (the default) turns it off.
+ * Process-wide; read when a call enqueues its kernels. */
+void sc_debug_stall_waits(unsigned long long ns);
 
 /* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
 size_t sc_workspace_size(int B, int L, int H);

@@ -51,7 +51,7 @@ class StackArgs(ctypes.Structure):
                 ("alpha", ctypes.POINTER(ctypes.c_float)),
                 ("O", ctypes.c_void_p), ("scores", ctypes.c_void_p),
                 ("pos", ctypes.c_void_p), ("len", ctypes.c_void_p), ("flags", ctypes.c_int),
-                ("keep_rule", ctypes.c_int)]
+                ("keep_rule", ctypes.c_int), ("O_last", ctypes.c_void_p)]
 
 
 class EncoderArgs(ctypes.Structure):
@@ -91,7 +91,7 @@ EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
             "sc_stack_host_workspace_size", "sc_stack_host_launch_count",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error",
             "sc_encoder_layer_forward", "sc_encoder_workspace_size", "sc_linear_forward",
-            "sc_layer_norm_forward"]
+            "sc_layer_norm_forward", "sc_layer_noalloc_status", "sc_debug_stall_waits"]
 
 
 def library_path() -> str:
@@ -122,6 +122,10 @@ def load(build_if_missing: bool = False):
                                          ctypes.c_size_t, ctypes.c_void_p]
         lib.sc_layer_forward_noalloc.restype = ctypes.c_int
         lib.sc_layer_forward_noalloc.argtypes = [ctypes.POINTER(LayerArgs), ctypes.c_void_p]
+        lib.sc_layer_noalloc_status.restype = ctypes.c_int
+        lib.sc_layer_noalloc_status.argtypes = [ctypes.c_void_p]
+        lib.sc_debug_stall_waits.restype = None
+        lib.sc_debug_stall_waits.argtypes = [ctypes.c_ulonglong]
         lib.sc_stack_forward_profiled.restype = ctypes.c_int
         lib.sc_stack_forward_profiled.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                                   ctypes.c_size_t, ctypes.c_void_p,
@@ -237,8 +241,21 @@ def layer_forward_noalloc(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=
     return O, scores, pos_out, len_out
 
 
+def layer_noalloc_status(stream=None) -> int:
+    """Synchronise and return (then clear) the status of the no-allocation calls."""
+    return int(load().sc_layer_noalloc_status(_stream_handle(stream)))
+
+
+def debug_stall_waits(ns: int) -> None:
+    """Test hook (``sc_debug_stall_waits``): while ns > 0 every per-layer
+    attention CTA waits on a barrier nothing completes for at most ns ns and
+    aborts; 0 turns it off."""
+    load().sc_debug_stall_waits(int(ns))
+
+
 def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
-                  stream=None, events=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE):
+                  stream=None, events=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE,
+                  o_last_only=False):
     """The pruned layer stack (``sc_stack_forward``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
@@ -247,23 +264,28 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
     events: optional list of >= 3 + 3 * n_layers torch.cuda.Event(enable_timing=True),
     recorded around every kernel on the launching stream (sc_stack_forward_profiled).
     no_tail: run every layer through the per-layer kernels (SC_STACK_NO_TAIL).
-    Returns a dict with O, scores, pos, len (device tensors).
+    o_last_only: write no O but the last layer's, to out["O_last"] [B, L, H, 64]
+    (O = NULL in the arguments).
+    Returns a dict with O (or O_last), scores, pos, len (device tensors).
     """
     nl, B, L, H, D = Q.shape
     dev = Q.device
     if out is None:
-        out = {"O": torch.empty((nl, B, L, H, D), dtype=torch.bfloat16, device=dev),
-               "scores": torch.empty((nl, B, L), dtype=torch.float32, device=dev),
+        out = {"scores": torch.empty((nl, B, L), dtype=torch.float32, device=dev),
                "pos": torch.empty((nl + 1, B, L), dtype=torch.int32, device=dev),
                "len": torch.empty((nl + 1, B), dtype=torch.int32, device=dev)}
+        if o_last_only:
+            out["O_last"] = torch.empty((B, L, H, D), dtype=torch.bfloat16, device=dev)
+        else:
+            out["O"] = torch.empty((nl, B, L, H, D), dtype=torch.bfloat16, device=dev)
     ws = workspace if workspace is not None else new_workspace(B, L, H, dev)
     garr, ng = _int32_host(global_pos)
     al = (ctypes.c_float * nl)(*[float(x) for x in alpha])
     a = StackArgs(nl, B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(pad_mask),
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
-                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
-                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule))
+                  _ptr(out.get("O")), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
+                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule), _ptr(out.get("O_last")))
     if events is None:
         _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
                                        _stream_handle(stream)))
@@ -303,12 +325,17 @@ def new_stack_host_workspace(n_layers, B, L, H, device=None) -> torch.Tensor:
     return ws[off:off + n]
 
 
-def new_host_outputs(n_layers, B, L, H):
-    """Page-locked host result tensors for ``stack_forward_host``."""
-    return {"O": torch.empty((n_layers, B, L, H, 64), dtype=torch.bfloat16, pin_memory=True),
-            "scores": torch.empty((n_layers, B, L), dtype=torch.float32, pin_memory=True),
-            "pos": torch.empty((n_layers + 1, B, L), dtype=torch.int32, pin_memory=True),
-            "len": torch.empty((n_layers + 1, B), dtype=torch.int32, pin_memory=True)}
+def new_host_outputs(n_layers, B, L, H, o_last_only=False):
+    """Page-locked host result tensors for ``stack_forward_host`` (``o_last_only``:
+    the last layer's O alone, as "O_last")."""
+    out = {"scores": torch.empty((n_layers, B, L), dtype=torch.float32, pin_memory=True),
+           "pos": torch.empty((n_layers + 1, B, L), dtype=torch.int32, pin_memory=True),
+           "len": torch.empty((n_layers + 1, B), dtype=torch.int32, pin_memory=True)}
+    if o_last_only:
+        out["O_last"] = torch.empty((B, L, H, 64), dtype=torch.bfloat16, pin_memory=True)
+    else:
+        out["O"] = torch.empty((n_layers, B, L, H, 64), dtype=torch.bfloat16, pin_memory=True)
+    return out
 
 
 def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
@@ -318,7 +345,8 @@ def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, wor
     Q, K, V: bf16 [n_layers, B, L, H, 64] page-locked CPU tensors (``pin_memory()``);
     pad_mask: uint8 [B, L] page-locked CPU tensor or None; the other arguments as for
     ``stack_forward``.  ``out``: page-locked result tensors (``new_host_outputs``);
-    only the current slots of each layer (and all of ``len``) are written.
+    only the current slots of each layer (and all of ``len``) are written; with
+    "O_last" in place of "O", only the last layer's O.
     The call is asynchronous on ``stream`` (default: torch's current stream of the
     current device): synchronise before reading ``out``.  The first call on newly
     page-locked buffers is slower (milliseconds) while the device maps their pages;
@@ -337,8 +365,8 @@ def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, wor
     a = StackArgs(nl, B, L, H, int(w), _ptr(Q), _ptr(K), _ptr(V), _ptr(pad_mask),
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
-                  _ptr(out["O"]), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
-                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule))
+                  _ptr(out.get("O")), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
+                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule), _ptr(out.get("O_last")))
     _check(load().sc_stack_forward_host(ctypes.byref(a), _ptr(ws), ws.numel(),
                                         _stream_handle(stream)))
     return out

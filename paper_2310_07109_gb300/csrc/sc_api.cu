@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstdio>
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -41,6 +42,10 @@ constexpr size_t kAlign = 256;
 // Detail of the most recent failure on this thread (sc_last_error()).
 thread_local char g_last_error[256] = "";
 
+// Test hook of the failure path (sc_debug_stall_waits): nanoseconds that every
+// rows CTA waits on a barrier that nothing completes; 0 = off.
+std::atomic<unsigned long long> g_stall_ns{0};
+
 int fail(int code, const char* what, const char* detail) {
   snprintf(g_last_error, sizeof g_last_error, "%s: %s", what, detail ? detail : "");
   return code;
@@ -53,7 +58,8 @@ int fail_cuda(const char* what, cudaError_t e) {
 size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
-  size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, rows_done, gcur, ng,
+  size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, rows_done, cols_done,
+      gcur, ng,
       ident,
       tail_from,
       loop_layer, qkv, total;
@@ -73,11 +79,12 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->colpart = take(sizeof(float) * B * H * (size_t)L * kWideBandTiles);
   w->gpart = take(sizeof(float) * B * H * T * 4 * kMaxGlobal);
   w->gstat = take(sizeof(float) * B * H * T * 4 * kMaxGlobal * 2);
-  w->og = take(sizeof(float) * B * H * kMaxGlobal * kHeadDim);
+  w->og = take(sizeof(float) * B * H * ((T + 1) / 2) * kMaxGlobal * kHeadDim);
   w->keep = take(sizeof(uint8_t) * B * (size_t)L);
   w->cnt_tile = take(sizeof(uint32_t) * B * T);
   w->cnt_seq = take(sizeof(uint32_t) * B);
   w->rows_done = take(sizeof(uint32_t) * B * H);
+  w->cols_done = take(sizeof(uint32_t) * B * H);
   w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
   w->ng = take(sizeof(int32_t) * 2 * B);
   w->ident = take(sizeof(int32_t) * 2 * B);
@@ -288,6 +295,8 @@ void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   p->cnt_tile = reinterpret_cast<uint32_t*>(ws + lay.cnt_tile);
   p->cnt_seq = reinterpret_cast<uint32_t*>(ws + lay.cnt_seq);
   p->rows_done = reinterpret_cast<uint32_t*>(ws + lay.rows_done);
+  p->cols_done = reinterpret_cast<uint32_t*>(ws + lay.cols_done);
+  p->stall_ns = g_stall_ns.load(std::memory_order_relaxed);
   int32_t* gcur = reinterpret_cast<int32_t*>(ws + lay.gcur);
   int32_t* ng = reinterpret_cast<int32_t*>(ws + lay.ng);
   int32_t* ident = reinterpret_cast<int32_t*>(ws + lay.ident);
@@ -439,11 +448,14 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
-  if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
+  if (!a->Q || !a->K || !a->V || !a->alpha || !a->scores || !a->pos || !a->len)
     return SC_ERR_INVALID_ARG;
   if ((rc = check_keep(a->keep_rule, a->alpha, a->n_layers, nullptr)) != SC_OK) return rc;
-  if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O))
+  if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O) ||
+      !aligned16(a->O_last))
     return SC_ERR_INVALID_ARG;
+  // the O of every layer, or (O == NULL) only the last layer's, to O_last
+  uint16_t* const o_last = a->O != nullptr ? nullptr : a->O_last;
   const long long rows = static_cast<long long>(a->n_layers) * a->B * a->L * a->H;
   if (rows > (1ll << 31) - 1) return SC_ERR_UNSUPPORTED;
   WsLayout lay;
@@ -478,6 +490,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   p.tail_from = tail_from;
   p.tail_max = use_tail ? kTailMax : 0;
   p.no_ident = host_io ? 1 : 0;
+  p.n_layers = a->n_layers;
   fill_workspace(&p, ws, lay, 0);
 
   PrepParams pp{};
@@ -563,6 +576,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     pd.pos = a->pos;
     pd.pos_out = a->pos + BL;
     pd.O = a->O;
+    pd.O_last = o_last;
     pd.scores = a->scores;
     pd.alpha = a->alpha[0];
     pd.tok_stride = BLt;
@@ -630,7 +644,8 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     p.len_out = a->len + static_cast<size_t>(l + 1) * a->B;
     p.pos = a->pos + static_cast<size_t>(l) * BL;
     p.pos_out = a->pos + static_cast<size_t>(l + 1) * BL;
-    p.O = a->O + static_cast<size_t>(l) * BL * a->H * kHeadDim;
+    p.O = a->O != nullptr ? a->O + static_cast<size_t>(l) * BL * a->H * kHeadDim
+          : l == a->n_layers - 1 ? o_last : nullptr;
     p.scores = a->scores + static_cast<size_t>(l) * BL;
     p.alpha = a->alpha[l];
     if (l == 0 && (a->pad_mask != nullptr || host_io)) {
@@ -663,6 +678,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     tp.pos = a->pos;
     tp.len = a->len;
     tp.O = a->O;
+    tp.O_last = o_last;
     tp.scores = a->scores;
     tp.status = p.status;
     for (int t = 0; t < 3; ++t) tp.src[t] = src[t];
@@ -749,7 +765,7 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
-  if (!a->Q || !a->K || !a->V || !a->alpha || !a->O || !a->scores || !a->pos || !a->len)
+  if (!a->Q || !a->K || !a->V || !a->alpha || !a->scores || !a->pos || !a->len)
     return SC_ERR_INVALID_ARG;
   HostIoLayout hl;
   if (!host_io_layout(a->n_layers, a->B, a->L, a->H, &hl)) return SC_ERR_INVALID_ARG;
@@ -760,15 +776,19 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   void* q = mapped_host_range(a->Q, qkv_bytes);
   void* k = mapped_host_range(a->K, qkv_bytes);
   void* v = mapped_host_range(a->V, qkv_bytes);
-  void* o = mapped_host_range(a->O, qkv_bytes);
+  // O of every layer, or (O == NULL) only the last layer's to O_last, or none
+  const size_t layer_o_bytes = qkv_bytes / a->n_layers;
+  void* o = a->O ? mapped_host_range(a->O, qkv_bytes) : nullptr;
+  void* o_last = !a->O && a->O_last ? mapped_host_range(a->O_last, layer_o_bytes) : nullptr;
   void* sc = mapped_host_range(a->scores, sizeof(float) * a->n_layers * BL);
   void* ps = mapped_host_range(a->pos, sizeof(int32_t) * (a->n_layers + 1) * BL);
   void* ln = mapped_host_range(a->len, sizeof(int32_t) * (a->n_layers + 1) * a->B);
   void* pm = a->pad_mask ? mapped_host_range(a->pad_mask, BL) : nullptr;
-  if (!q || !k || !v || !o || !sc || !ps || !ln || (a->pad_mask && !pm))
+  if (!q || !k || !v || (a->O && !o) || (!a->O && a->O_last && !o_last) || !sc || !ps || !ln ||
+      (a->pad_mask && !pm))
     return fail(SC_ERR_INVALID_ARG, "sc_stack_forward_host",
                 "a host buffer is not page-locked memory mapped for the device");
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) ||
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(o_last) ||
       (reinterpret_cast<uintptr_t>(sc) & 3u) || (reinterpret_cast<uintptr_t>(ps) & 3u) ||
       (reinterpret_cast<uintptr_t>(ln) & 3u))
     return SC_ERR_INVALID_ARG;
@@ -778,7 +798,10 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   d.K = static_cast<const uint16_t*>(k);
   d.V = static_cast<const uint16_t*>(v);
   d.pad_mask = static_cast<const uint8_t*>(pm);
-  d.O = reinterpret_cast<uint16_t*>(ws + hl.O);
+  uint16_t* const dO = reinterpret_cast<uint16_t*>(ws + hl.O);
+  d.O = a->O ? dO : nullptr;
+  d.O_last = a->O ? nullptr
+             : a->O_last ? dO + (a->n_layers - 1) * (layer_o_bytes / sizeof(uint16_t)) : nullptr;
   d.scores = reinterpret_cast<float*>(ws + hl.scores);
   d.pos = reinterpret_cast<int32_t*>(ws + hl.pos);
   d.len = reinterpret_cast<int32_t*>(ws + hl.len);
@@ -793,8 +816,9 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   ws_layout(a->B, a->L, a->H, &lay);
   ExportParams e{};
   e.n_layers = a->n_layers; e.B = a->B; e.L = a->L; e.H = a->H;
-  e.O = d.O; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
+  e.O = dO; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
   e.hO = static_cast<uint16_t*>(o);
+  e.hO_last = static_cast<uint16_t*>(o_last);
   e.hscores = static_cast<float*>(sc);
   e.hpos = static_cast<int32_t*>(ps);
   e.hlen = static_cast<int32_t*>(ln);
@@ -842,6 +866,8 @@ int sc_stack_launch_count(const sc_stack_args* a, int* count) {
   *count = k;
   return SC_OK;
 }
+
+void sc_debug_stall_waits(unsigned long long ns) { g_stall_ns.store(ns); }
 
 int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {
   if (!workspace || ws_bytes < kAlign) return SC_ERR_WORKSPACE;
@@ -933,10 +959,10 @@ extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
                             const_cast<uint16_t*>(a->V)};
   const long long tokens = static_cast<long long>(a->B) * a->L;
   if (!encode_maps(&maps, src, tokens, cmp, tokens, a->H)) return SC_ERR_CUDA;
-  // the array keeps the previous call's contents: clear the status word and
-  // the counters, which must start at zero
-  cudaError_t e = cudaMemsetAsync(ws + lay.status, 0, sizeof(int), st);
-  if (e != cudaSuccess) return fail_cuda("static workspace status reset", e);
+  // the array keeps the previous call's contents: clear the counters, which
+  // must start at zero (the status word is kept until sc_layer_noalloc_status
+  // reads it, so that an expired wait of any call is reported)
+  cudaError_t e;
   if ((rc = reset_counters(ws, lay, st)) != SC_OK) return rc;
 
   LayerParams p{};
@@ -967,6 +993,20 @@ extern "C" int sc_layer_forward_noalloc(const sc_layer_args* a, void* stream) {
   if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
   if ((e = launch_cols(maps, p, st)) != cudaSuccess) return fail_cuda("launch cols kernel", e);
   return SC_OK;
+}
+
+extern "C" int sc_layer_noalloc_status(void* stream) {
+  char* ws = nullptr;
+  int rc = static_workspace(&ws);
+  if (rc != SC_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return SC_ERR_CUDA;
+  int word = 0;
+  if (cudaMemcpy(&word, ws, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return SC_ERR_CUDA;
+  if (word == 0) return SC_OK;
+  if (cudaMemset(ws, 0, sizeof(int)) != cudaSuccess) return SC_ERR_CUDA;
+  return (word & kStatusTimeout) ? SC_ERR_TIMEOUT : SC_ERR_CUDA;
 }
 
 // ---------------------------------------------------------------------------

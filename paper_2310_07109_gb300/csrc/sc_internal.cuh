@@ -79,13 +79,19 @@ struct LayerParams {
                          //   per (query tile, 32-row warp slice)
   float* gstat;          // [B][H][T][4][kMaxGlobal][2] (max, sum) of global rows per
                          //   (key tile, 32-key warp slice)
-  float* og;             // [B][H][kMaxGlobal][64] fp32 outputs of global rows
+  float* og;             // [B][H][T2][kMaxGlobal][64] fp32 parts of the global rows'
+                         //   outputs, one per key-tile pair (T2 = (T + 1) / 2)
   uint8_t* keep;         // [B][L]
   uint32_t* cnt_tile;    // [B][T]
   uint32_t* cnt_seq;     // [B]
   uint32_t* rows_done;   // [B][H]: rows CTAs of (sequence, head) whose results are visible
+  uint32_t* cols_done;   // [B][H]: cols CTAs of (sequence, head) whose global-row parts are stored
   int32_t* kept_cur;     // [B][L] out, or nullptr: current index of each kept token, in order
   int* status;
+  // test hook: when nonzero, the first MMA-issuing thread of every rows CTA
+  // first waits at most this many nanoseconds on a barrier that nothing
+  // completes, so that the bounded wait expires and the CTA aborts
+  unsigned long long stall_ns;
   // hand-over to the cluster kernel: sequence b is skipped here once
   // tail_from[b] <= layer; the finalize of a layer sets tail_from[b] = layer + 1
   // when at most tail_max tokens survive.  tail_from == nullptr: no hand-over.
@@ -103,6 +109,9 @@ struct LayerParams {
   long long tok_stride;   // tokens of one layer in the source tensors (B * L)
   long long row_stride;   // entries of one layer in pos, pos_out, scores (B * L)
   long long o_stride;     // elements of one layer in O (B * L * H * 64)
+  // O == nullptr: only the last layer's O is written, to O_last (when set)
+  uint16_t* O_last;
+  int n_layers;
   int len_stride;         // entries of one layer in len, len_out (B)
   float alphas[kTailMaxLayers];
 };
@@ -186,7 +195,8 @@ struct ExportParams {
   const float* scores;         // device [n_layers][B][L]
   const int32_t* pos;          // device [n_layers + 1][B][L]
   const int32_t* len;          // device [n_layers + 1][B]
-  uint16_t* hO;                // host (device-mapped addresses), same layouts
+  uint16_t* hO;                // host (device-mapped addresses), same layouts; or nullptr:
+  uint16_t* hO_last;           //   only the last layer's O rows, to hO_last [B][L][H][64]
   float* hscores;
   int32_t* hpos;
   int32_t* hlen;
@@ -202,7 +212,8 @@ struct TailParams {
   const int32_t* tail_from;    // [B] first layer run here (>= n_layers: none)
   int32_t* pos;                // [n_layers + 1][B][L]
   int32_t* len;                // [n_layers + 1][B]
-  uint16_t* O;                 // [n_layers][B][L][H][64]
+  uint16_t* O;                 // [n_layers][B][L][H][64], or nullptr: ...
+  uint16_t* O_last;            // ... only the last layer's [B][L][H][64] (when set)
   float* scores;               // [n_layers][B][L]
   int* status;
   const uint16_t* src[3];      // Q, K, V [n_layers][B][L][H][64]

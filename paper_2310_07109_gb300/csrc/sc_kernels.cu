@@ -103,7 +103,7 @@ __device__ __forceinline__ LayerView layer_view(const LayerParams& p) {
   v.ng_out = odd ? const_cast<int32_t*>(p.ng) : p.ng_out;
   v.ident = odd ? p.ident_out : p.ident;
   v.ident_out = odd ? const_cast<int32_t*>(p.ident) : p.ident_out;
-  v.O = p.O + l * p.o_stride;
+  v.O = p.O != nullptr ? p.O + l * p.o_stride : (l == p.n_layers - 1 ? p.O_last : nullptr);
   v.scores = p.scores + l * p.row_stride;
   v.alpha = p.alphas[l];
   return v;
@@ -228,6 +228,7 @@ struct RowsSmem {
   uint64_t bar_vfull[kVStages], bar_vempty[kVStages];
   uint64_t bar_sg[2], bar_sgend[2], bar_sfull[2], bar_sfree[2], bar_pready[2], bar_pvdone[2];
   uint64_t bar_fin[2];
+  uint64_t bar_stall;   // test hook: nothing ever completes it
   uint32_t tmem_base;
   int abort;
   int gc[kMaxGlobal];
@@ -349,6 +350,7 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       mbar_init(&sm.bar_pvdone[X], 1);
       mbar_init(&sm.bar_fin[X], 1);
     }
+    mbar_init(&sm.bar_stall, 1);
     sm.abort = 0;
     fence_mbar_init();
   }
@@ -396,18 +398,22 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     if (lane == 0) {
       const RowSource rs = row_source(p, v, b);
       bool ok = true;
+      int issued = 0;
       // slot s = k mod nvs and its use count, advanced without division
       for (int k = 0, s = 0, use = 0; ok && k < nk; ++k) {
         if (k >= nvs && !(ok = mbar_wait(&sm.bar_vempty[s], (use - 1) & 1, abort_flag))) break;
         mbar_arrive_expect_tx(&sm.bar_vfull[s], kTileBytes);
         load_tile(maps, 2, rs, h, (kt_lo + k) * kTile, Vs + s * kTileBytes, &sm.bar_vfull[s]);
+        issued = k + 1;
         if (++s == nvs) {
           s = 0;
           ++use;
         }
       }
-      for (int s = 0; s < nvs && s < nk; ++s) {
-        const int last = s + nvs * ((nk - 1 - s) / nvs);
+      // the last copy issued into each slot has landed (after an expired wait
+      // fewer than nk were issued)
+      for (int s = 0; s < nvs && s < issued; ++s) {
+        const int last = s + nvs * ((issued - 1 - s) / nvs);
         drain_wait(&sm.bar_vfull[s], (last / nvs) & 1);
       }
     }
@@ -418,7 +424,10 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
       const uint32_t q_a = smem_u32(Qs) + X * kTileBytes, k_a = smem_u32(Ks), v_a = smem_u32(Vs);
       const int kloX = klo[X], khiX = khi[X];
       const uint32_t tS = tm + col_s(X), tP = tm + col_p(X), tO = tm + col_o(X);
-      bool ok = mbar_wait(&sm.bar_q, 0, abort_flag);
+      bool ok = true;
+      if (X == 0 && p.stall_ns != 0)   // test hook: this bounded wait expires
+        ok = mbar_wait(&sm.bar_stall, 0, abort_flag, p.stall_ns);
+      ok = ok && mbar_wait(&sm.bar_q, 0, abort_flag);
       if (ok) {
         tc_fence_after();
         if (ngp) {
@@ -509,7 +518,11 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     const int lo = max(0, i - p.w);
     const int hi = min(n - 1, i + p.w);
 
-    float m_ref = -INFINITY, lsum = 0.f;
+    // lsum: the row sum of the exponentials (fp32), which gives the row's LSE
+    // for the column sums; osum: the sum of the same values rounded to the
+    // bf16 that P V multiplies, which normalises O (so that O is a weighted
+    // mean of V rows whatever the rounding of P)
+    float m_ref = -INFINITY, lsum = 0.f, osum = 0.f;
     bool ok = active;
     uint32_t pv_issued = 0;               // P V products issued for this warpgroup
 
@@ -534,8 +547,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         for (int g = 0; g < kMaxGlobal; g += 2) {
           const float a = ex2(fmaf(xg[g], kLogitScale2, nref));
           const float c = ex2(fmaf(xg[g + 1], kLogitScale2, nref));
-          lsum += a + c;
           pk[g / 2] = pack_bf16x2(a, c);
+          lsum += a + c;
+          osum = add_bf16_hi(add_bf16_lo(osum, pk[g / 2]), pk[g / 2]);
         }
         tmem_st8(tP + 16, pk);            // P_G
         tmem_st_wait();
@@ -597,10 +611,12 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         f = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - tmax);
         m_ref = tmax;
         lsum *= f;
+        osum *= f;
       }
       const float nref = (m_ref == -INFINITY) ? 0.f : -m_ref;
       const uint64_t n2 = f2_pack(nref, nref);
       uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+      float sq[4] = {0.f, 0.f, 0.f, 0.f};
       uint32_t pk[64];
 #pragma unroll
       for (int k = 0; k < kTile; k += 2) {
@@ -611,11 +627,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         if (k & 2) s2b = f2_add(s2b, f2_pack(u, w));
         else s2a = f2_add(s2a, f2_pack(u, w));
         pk[k >> 1] = pack_bf16x2(u, w);
+        const int c = (k >> 1) & 1;
+        sq[2 * c] = add_bf16_lo(sq[2 * c], pk[k >> 1]);
+        sq[2 * c + 1] = add_bf16_hi(sq[2 * c + 1], pk[k >> 1]);
       }
       float sa, sb, sc2, sd;
       f2_unpack(s2a, sa, sb);
       f2_unpack(s2b, sc2, sd);
       lsum += (sa + sb) + (sc2 + sd);
+      osum += (sq[0] + sq[1]) + (sq[2] + sq[3]);
       // every earlier P V has completed: O is final for a rescale and the P
       // columns of this warpgroup are free again
       if (pv_issued > 0 && !(ok = warp_wait(&sm.bar_pvdone[X], (pv_issued - 1) & 1, abort_flag)))
@@ -696,10 +716,6 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
         p.gstat[2 * (slot0 + gme)] = mme;
         p.gstat[2 * (slot0 + gme) + 1] = sme;
       }
-      if (qt == 0) {
-        float* og = p.og + (static_cast<size_t>(b) * p.H + h) * kMaxGlobal * kHeadDim;
-        for (int k = r; k < kMaxGlobal * kHeadDim; k += 128) og[k] = 0.f;
-      }
     }
 
     // Band pass (the column sums of Sec. "Extractor of Attention Scores"):
@@ -759,9 +775,9 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
 
     // ---- O: its rows leave through this warp's quarter of its Q tile; every
     // MMA that read the tile completed before the last S^T was awaited
-    if (ok && have_o) {
+    if (ok && have_o && v.O != nullptr) {
       tc_fence_after();
-      const float inv = 1.f / lsum;
+      const float inv = 1.f / osum;
       uint8_t* stage = Qs + X * kTileBytes + wq * 4096;
 #pragma unroll
       for (int c = 0; c < 64; c += 32) {
@@ -834,6 +850,9 @@ struct ColsSmem {
   int flag;
   float wpart[kColsThreads / 32];
   int gnew[kMaxGlobal];
+  // each key tile's part of the global rows' P V (warpgroup X), added in
+  // tile order into the pair's part
+  alignas(16) float ogx[2][kMaxGlobal][kHeadDim];   // read and written as float4
   // sequence compaction: per (round, warp) ballot of kept tokens and the
   // exclusive prefix of their counts
   uint32_t kbits[(kMaxLen + kColsThreads - 1) / kColsThreads][kColsThreads / 32];
@@ -1044,18 +1063,42 @@ __global__ void __launch_bounds__(kColsThreads, 2)
       tc_fence_before();
       warp_arrive(&sm.bar_pg[X]);
       bool ok3 = ok2 && warp_wait(&sm.bar_og[X], 0, abort_flag);
-      if (wq == 0 && ok3) {
-        tc_fence_after();
-        float* og = p.og + ((static_cast<size_t>(b) * p.H + h) * kMaxGlobal) * kHeadDim;
+      if (wq == 0) {
+        // this key tile's part of the global rows' outputs (TMEM lane g = global g)
+        if (ok3) tc_fence_after();
+        float* mine = &sm.ogx[X][lane & (kMaxGlobal - 1)][0];
+#pragma unroll 1
+        for (int c = 0; c < 64; c += 16) {
+          float o[16];
+          if (ok3) {
+            tmem_ld16(tOG + lane_off + c, o);
+            tmem_ld_wait();
+          } else {
 #pragma unroll
-        for (int c = 0; c < 64; c += 32) {
-          float o[32];
-          tmem_ld32(tOG + lane_off + c, o);
-          tmem_ld_wait();
-          if (lane < ng)
+            for (int k = 0; k < 16; ++k) o[k] = 0.f;
+          }
+          if (lane < kMaxGlobal)
 #pragma unroll
-            for (int k = 0; k < 32; k += 4)
-              red_add_v4(og + lane * kHeadDim + c + k, o[k], o[k + 1], o[k + 2], o[k + 3]);
+            for (int k = 0; k < 16; k += 4)
+              *reinterpret_cast<float4*>(mine + c + k) = make_float4(o[k], o[k + 1], o[k + 2], o[k + 3]);
+        }
+        // warps 0 and 4 (the first warp of each warpgroup) meet here when the
+        // pair has two key tiles; warp 0 adds the parts in tile order and
+        // stores the pair's part (plain stores: no order-dependent atomics)
+        if (hasB) asm volatile("bar.sync 5, 64;" ::: "memory");
+        else __syncwarp();
+        if (X == 0) {
+          float* part = p.og + (((static_cast<size_t>(b) * p.H + h) * T2 + pr) * kMaxGlobal) *
+                                   kHeadDim;
+          for (int k = lane; k < ng * (kHeadDim / 4); k += 32) {
+            const int g = k / (kHeadDim / 4), d = 4 * (k % (kHeadDim / 4));
+            float4 a4 = *reinterpret_cast<const float4*>(&sm.ogx[0][g][d]);
+            if (hasB) {
+              const float4 b4 = *reinterpret_cast<const float4*>(&sm.ogx[1][g][d]);
+              a4.x += b4.x; a4.y += b4.y; a4.z += b4.z; a4.w += b4.w;
+            }
+            *reinterpret_cast<float4*>(part + g * kHeadDim + d) = a4;
+          }
         }
       }
     }
@@ -1069,6 +1112,43 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     tmem_dealloc(tm, 256);
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
+
+  // ---- last pair of this (sequence, head): the global rows' outputs, the
+  // pairs' parts added in pair order
+  if (ngp) {
+    __threadfence();
+    __syncthreads();
+    if (tid == 0)
+      sm.flag = (atomicAdd(p.cols_done + b * p.H + h, 1u) == static_cast<uint32_t>(Tp - 1));
+    __syncthreads();
+    if (sm.flag) {
+      __threadfence();
+      const float* part0 =
+          p.og + (static_cast<size_t>(b) * p.H + h) * T2 * kMaxGlobal * kHeadDim;
+      for (int k = tid; k < ng * (kHeadDim / 4); k += kColsThreads) {
+        const int g = k / (kHeadDim / 4), d = 4 * (k % (kHeadDim / 4));
+        constexpr int kBatch = 8;   // loads in flight before they are added
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q0 = 0; q0 < Tp; q0 += kBatch) {
+          float4 x[kBatch];
+#pragma unroll
+          for (int u = 0; u < kBatch; ++u)
+            x[u] = q0 + u < Tp ? __ldcg(reinterpret_cast<const float4*>(
+                                     part0 + ((q0 + u) * kMaxGlobal + g) * kHeadDim + d))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int u = 0; u < kBatch; ++u) {
+            acc.x += x[u].x; acc.y += x[u].y; acc.z += x[u].z; acc.w += x[u].w;
+          }
+        }
+        if (v.O != nullptr)
+          *reinterpret_cast<uint2*>(v.O + ((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + h) *
+                                              kHeadDim + d) =
+              make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
+      }
+      if (tid == 0) p.cols_done[b * p.H + h] = 0u;
+    }
+  }
 
   // ---- last head of this pair of key tiles: scores and keep flags (fixed head order)
   __threadfence();
@@ -1256,28 +1336,6 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
     const uint32_t bits = sm.kbits[r][t >> 5];
     if ((bits >> (t & 31)) & 1u) sm.gnew[tid] = sm.kpre[r][t >> 5] + __popc(bits & ((1u << (t & 31)) - 1u));
   }
-  // bf16 outputs of the global rows, 4 values per load
-  const int nvec = ng * p.H * (kHeadDim / 4);
-  for (int k0 = 0; k0 < nvec; k0 += 8 * kColsThreads) {
-    float4 o4[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int k = k0 + tid + u * kColsThreads;
-      const int g = k / (p.H * 16), hh = (k / 16) % p.H, d4 = k % 16;
-      o4[u] = k < nvec ? __ldcg(reinterpret_cast<const float4*>(
-                             p.og + ((static_cast<size_t>(b) * p.H + hh) * kMaxGlobal + g) * kHeadDim) + d4)
-                       : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int k = k0 + tid + u * kColsThreads;
-      if (k >= nvec) continue;
-      const int g = k / (p.H * 16), hh = (k / 16) % p.H, d4 = k % 16;
-      uint2 w2 = make_uint2(pack_bf16x2(o4[u].x, o4[u].y), pack_bf16x2(o4[u].z, o4[u].w));
-      *reinterpret_cast<uint2*>(v.O + ((static_cast<size_t>(b) * p.L + sm.gc[g]) * p.H + hh) *
-                                          kHeadDim + 4 * d4) = w2;
-    }
-  }
   __syncthreads();
   if (tid == 0) {
     const int total = sm.total;
@@ -1388,9 +1446,13 @@ __global__ void __launch_bounds__(kExportThreads)
       if (l < e.n_layers) e.hscores[row0 + threadIdx.x] = __ldcg(e.scores + row0 + threadIdx.x);
     }
     if (l >= e.n_layers) continue;
+    uint4* dst;
+    if (e.hO != nullptr) dst = reinterpret_cast<uint4*>(e.hO) + row0 * vec;
+    else if (l == e.n_layers - 1 && e.hO_last != nullptr)
+      dst = reinterpret_cast<uint4*>(e.hO_last) + (static_cast<size_t>(b) * e.L + c0) * vec;
+    else continue;
     const int total = cnt * vec;
     const uint4* src = reinterpret_cast<const uint4*>(e.O) + row0 * vec;
-    uint4* dst = reinterpret_cast<uint4*>(e.hO) + row0 * vec;
     constexpr int kPer = 4;
     for (int k0 = threadIdx.x; k0 < total; k0 += kExportThreads * kPer) {
       uint4 v[kPer];

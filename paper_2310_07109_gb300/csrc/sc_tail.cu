@@ -350,10 +350,15 @@ __global__ void __launch_bounds__(kTailThreads, 1)
       // P = exp2(S - max) over half kh, written as bf16 pairs over the first
       // half of its columns (each step's pairs land on columns this or an
       // earlier step has read); returns the half's row sum
-      auto half_exp = [&](const Partners& me, int kh, float nmc) {
+      // Returns the half's sum of the exponentials (fp32: the row's LSE, which
+      // the column sums use) and adds to *osum the same values rounded to the
+      // bf16 that P V multiplies (the normaliser of O, so that O is a weighted
+      // mean of V rows whatever the rounding of P).
+      auto half_exp = [&](const Partners& me, int kh, float nmc, float* osum) {
         const int nh = min(256, n - 256 * kh);
         const uint64_t n2 = f2_pack(nmc, nmc);
         uint64_t s2a = f2_pack(0.f, 0.f), s2b = s2a;
+        float la = 0.f, lb = 0.f, lc = 0.f, ld = 0.f;
         for (int q2 = 0; q2 < (nh + 63) >> 6; ++q2) {
           float x[64];
           tmem_ld32(tR + 64 * q2, x);
@@ -373,15 +378,23 @@ __global__ void __launch_bounds__(kTailThreads, 1)
               if (k & 2) s2b = f2_add(s2b, f2_pack(u, v));
               else s2a = f2_add(s2a, f2_pack(u, v));
               pk[k >> 1] = pack_bf16x2(u, v);
+              if (k & 2) {
+                lc = add_bf16_lo(lc, pk[k >> 1]);
+                ld = add_bf16_hi(ld, pk[k >> 1]);
+              } else {
+                la = add_bf16_lo(la, pk[k >> 1]);
+                lb = add_bf16_hi(lb, pk[k >> 1]);
+              }
             }
             tmem_st16(tR + 32 * q2 + 16 * hq, pk);
           }
         }
         tmem_st_wait();
-        float la, lb, lc, ld;
-        f2_unpack(s2a, la, lb);
-        f2_unpack(s2b, lc, ld);
-        return (la + lb) + (lc + ld);
+        *osum += (la + lb) + (lc + ld);
+        float ea, eb, ec, ed;
+        f2_unpack(s2a, ea, eb);
+        f2_unpack(s2b, ec, ed);
+        return (ea + eb) + (ec + ed);
       };
       auto release = [&]() {   // the warpgroup's columns are read
         tc_fence_before();
@@ -400,7 +413,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         const float m0 = half_max(me, 0, -INFINITY);
         const float nmc0 = (me.valid && m0 != -INFINITY) ? -m0 * kLogitScale2 : 0.f;
         float nmc = nmc0;
-        float lsum = half_exp(me, 0, nmc0);
+        float osum = 0.f;
+        float lsum = half_exp(me, 0, nmc0, &osum);
         tc_fence_before();
         warp_arrive(&sm.bar_pready[X]);
         if (nkh == 2) {
@@ -420,6 +434,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
             f = m0 == -INFINITY ? 0.f : ex2((m0 - m1) * kLogitScale2);
             nmc = -m1 * kLogitScale2;
             lsum *= f;
+            osum *= f;
           }
           if (__any_sync(0xffffffffu, raise)) {
 #pragma unroll 1
@@ -433,13 +448,13 @@ __global__ void __launch_bounds__(kTailThreads, 1)
               tmem_st_wait();   // o is reused
             }
           }
-          lsum += half_exp(me, 1, nmc);
+          lsum += half_exp(me, 1, nmc, &osum);
           tc_fence_before();
           warp_arrive(&sm.bar_pready[X]);
         }
         if (!(ok = tail_wait(&sm.bar_odone[X], (n_odone++) & 1, abort_flag))) break;
         tc_fence_after();
-        const float inv = me.valid ? 1.f / lsum : 0.f;
+        const float inv = me.valid ? 1.f / osum : 0.f;
         float o[64];
         tmem_ld32(tO, o);
         tmem_ld32(tO + 32, o + 32);
@@ -447,13 +462,16 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         sm.nlse[i] = me.valid ? -(lg2(lsum) - nmc) : -INFINITY;
         // O is in registers: the columns may take S^T while O is stored
         release();
-        // the warp's 32 rows leave in two column halves of 64 bytes
+        // the warp's 32 rows leave in two column halves of 64 bytes (no O
+        // but the last layer's when O is not kept)
         uint8_t* stage = base + 3 * kTailOpBytes + warp * 2048;
+        uint16_t* const Ol = p.O != nullptr ? p.O + static_cast<size_t>(l) * B * L * H * kHeadDim
+                             : l == n_layers - 1 ? p.O_last : nullptr;
         uint16_t* row0 =
-            p.O + (((static_cast<size_t>(l) * B + b) * L + i - (r & 31)) * H + h) * kHeadDim;
+            Ol ? Ol + ((static_cast<size_t>(b) * L + i - (r & 31)) * H + h) * kHeadDim : nullptr;
         const uint32_t rows = __ballot_sync(0xffffffffu, me.valid);
 #pragma unroll
-        for (int c = 0; c < 64; c += 32) {
+        for (int c = 0; c < 64 && Ol != nullptr; c += 32) {
 #pragma unroll
           for (int k = 0; k < 32; k += 8)
             stage_row_piece<4>(stage, k >> 3,

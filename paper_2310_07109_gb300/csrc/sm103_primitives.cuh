@@ -485,6 +485,20 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+// s + (low bf16 of pk), s + (high bf16 of pk): one mixed-precision add each
+// (the bf16 operand widens exactly), so that a sum can be taken over the
+// rounded values themselves without unpacking them first
+__device__ __forceinline__ float add_bf16_lo(float s, uint32_t pk) {
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, lo, %0;\n\t}"
+      : "+f"(s) : "r"(pk));
+  return s;
+}
+__device__ __forceinline__ float add_bf16_hi(float s, uint32_t pk) {
+  asm("{\n\t.reg .b16 lo, hi;\n\tmov.b32 {lo, hi}, %1;\n\tadd.rn.f32.bf16 %0, hi, %0;\n\t}"
+      : "+f"(s) : "r"(pk));
+  return s;
+}
+
 // Coalesced store of a warp's 32 bf16 rows (one row per lane, kPieces 16-byte
 // pieces: 8 for 128-byte rows, 4 for 64-byte rows) through a 32 * kPieces * 16
 // byte shared-memory staging area.  Each lane first stages its pieces

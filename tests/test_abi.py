@@ -22,7 +22,8 @@ def lib():
 
 def declared_functions():
     text = open(HEADER).read()
-    return sorted(set(re.findall(r"^\s*(?:size_t|int|const char\*)\s+(sc_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*(?:size_t|int|void|const char\*)\s+(sc_\w+)\s*\(", text,
+                                 re.M)))
 
 
 def test_header_declares_the_documented_calls():
@@ -126,8 +127,11 @@ def test_stack_rejects_bad_arguments(lib):
 
     assert call(n_layers=0) == bd.SC_ERR_INVALID_ARG
     assert call(alpha=None) == bd.SC_ERR_INVALID_ARG
-    assert call(O=None) == bd.SC_ERR_INVALID_ARG
+    assert call(scores=None) == bd.SC_ERR_INVALID_ARG
     assert call(V=FAKE + 2) == bd.SC_ERR_INVALID_ARG
+    # O == NULL is a valid request (only the last layer's O, to O_last, or none);
+    # a misaligned O_last is refused before anything runs
+    assert call(O=None, O_last=FAKE + 2) == bd.SC_ERR_INVALID_ARG
     assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
     assert call(w=513) == bd.SC_ERR_UNSUPPORTED
     assert call(flags=2) == bd.SC_ERR_INVALID_ARG

@@ -288,6 +288,28 @@ int sc_stack_forward_host(const sc_stack_args* args, void* workspace, size_t wor
  * as sc_stack_launch_count for sc_stack_forward. */
 int sc_stack_host_launch_count(const sc_stack_args* args, int* count);
 
+/*
+ * The per-layer attention for windows of at most 256 tokens on each side can
+ * run in one of two designs (process-wide, read when a call enqueues its
+ * kernels; both give the method's results within the stated tolerances):
+ *   SC_ROWS_TWO_PASS (default): the row pass keeps only O and each row's LSE;
+ *     a second pass over the band recomputes S^T and its exponentials to form
+ *     the column sums of Sec. "Pruning" ("accumulated vertically", Fig. 1) in
+ *     fp32.
+ *   SC_ROWS_SINGLE_PASS: every band tile's S = q.k/8 is computed and
+ *     exponentiated once; each tile's bf16 probabilities stay on chip until
+ *     the row's normaliser is known, and the column sums are then one
+ *     tensor-core product per tile (P~^T times the per-row weights
+ *     2^(m_t - LSE_i)).  The bf16 rounding of P~ bounds the relative error of
+ *     each score by 2^-9; sequences of at least a few hundred tokens stay well
+ *     inside 1e-5 absolute, sequences of a few dozen tokens may not.
+ * Wider windows always use the two-pass design.  Returns SC_ERR_INVALID_ARG
+ * for any other value.
+ */
+#define SC_ROWS_SINGLE_PASS 0
+#define SC_ROWS_TWO_PASS 1
+int sc_select_rows_kernel(int which);
+
 /* Synchronises `stream`, returns SC_ERR_TIMEOUT if any kernel since the last
  * query recorded an expired wait (else SC_OK, or SC_ERR_CUDA), and clears
  * the status word. */

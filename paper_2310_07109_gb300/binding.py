@@ -91,7 +91,8 @@ EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
             "sc_stack_host_workspace_size", "sc_stack_host_launch_count",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error",
             "sc_encoder_layer_forward", "sc_encoder_workspace_size", "sc_linear_forward",
-            "sc_layer_norm_forward", "sc_layer_noalloc_status", "sc_debug_stall_waits"]
+            "sc_layer_norm_forward", "sc_layer_noalloc_status", "sc_debug_stall_waits",
+            "sc_select_rows_kernel"]
 
 
 def library_path() -> str:
@@ -126,6 +127,8 @@ def load(build_if_missing: bool = False):
         lib.sc_layer_noalloc_status.argtypes = [ctypes.c_void_p]
         lib.sc_debug_stall_waits.restype = None
         lib.sc_debug_stall_waits.argtypes = [ctypes.c_ulonglong]
+        lib.sc_select_rows_kernel.restype = ctypes.c_int
+        lib.sc_select_rows_kernel.argtypes = [ctypes.c_int]
         lib.sc_stack_forward_profiled.restype = ctypes.c_int
         lib.sc_stack_forward_profiled.argtypes = [ctypes.POINTER(StackArgs), ctypes.c_void_p,
                                                   ctypes.c_size_t, ctypes.c_void_p,
@@ -244,6 +247,15 @@ def layer_forward_noalloc(Q, K, V, length, pos, w, global_pos, alpha=0.0, theta=
 def layer_noalloc_status(stream=None) -> int:
     """Synchronise and return (then clear) the status of the no-allocation calls."""
     return int(load().sc_layer_noalloc_status(_stream_handle(stream)))
+
+
+SC_ROWS_SINGLE_PASS = 0
+SC_ROWS_TWO_PASS = 1
+
+
+def select_rows_kernel(which: int) -> None:
+    """``sc_select_rows_kernel``: SC_ROWS_TWO_PASS (default) or SC_ROWS_SINGLE_PASS."""
+    _check(load().sc_select_rows_kernel(int(which)))
 
 
 def debug_stall_waits(ns: int) -> None:

@@ -18,7 +18,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 LIB = os.path.join(HERE, "libsparsecoder.so")
-SOURCES = ["sc_kernels.cu", "sc_tail.cu", "sc_encoder.cu", "sc_api.cu"]
+SOURCES = ["sc_kernels.cu", "sc_band.cu", "sc_tail.cu", "sc_encoder.cu", "sc_api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

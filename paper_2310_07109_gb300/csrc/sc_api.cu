@@ -46,6 +46,29 @@ thread_local char g_last_error[256] = "";
 // rows CTA waits on a barrier that nothing completes; 0 = off.
 std::atomic<unsigned long long> g_stall_ns{0};
 
+// Which rows kernel computes the per-layer attention for windows up to 256
+// (sc_select_rows_kernel): SC_ROWS_SINGLE_PASS or SC_ROWS_TWO_PASS.
+std::atomic<int> g_rows_kernel{SC_ROWS_TWO_PASS};
+
+// Multiprocessors of the current device (cached per device; 0 if unknown).
+int device_sms() {
+  static std::atomic<int> cache[256];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) {
+    cudaGetLastError();
+    return 0;
+  }
+  int v = cache[dev].load(std::memory_order_relaxed);
+  if (v == 0) {
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      cudaGetLastError();
+      v = 0;
+    }
+    cache[dev].store(v, std::memory_order_relaxed);
+  }
+  return v;
+}
+
 int fail(int code, const char* what, const char* detail) {
   snprintf(g_last_error, sizeof g_last_error, "%s: %s", what, detail ? detail : "");
   return code;
@@ -310,6 +333,9 @@ void fill_workspace(LayerParams* p, char* ws, const WsLayout& lay, int slot) {
   // band reaches more than five key tiles
   p->wide = (p->w > kPairWindow && p->T > kMaxBandTiles) ? 1 : 0;
   p->band_slots = p->wide ? kWideBandTiles : kMaxBandTiles;
+  p->sms = device_sms();
+  p->band = (!p->wide && p->sms > 0 &&
+             g_rows_kernel.load(std::memory_order_relaxed) == SC_ROWS_SINGLE_PASS) ? 1 : 0;
 }
 
 void compacted_qkv(char* ws, const WsLayout& lay, int B, int L, int H, uint16_t* out[3]) {
@@ -868,6 +894,12 @@ int sc_stack_launch_count(const sc_stack_args* a, int* count) {
 }
 
 void sc_debug_stall_waits(unsigned long long ns) { g_stall_ns.store(ns); }
+
+int sc_select_rows_kernel(int which) {
+  if (which != SC_ROWS_SINGLE_PASS && which != SC_ROWS_TWO_PASS) return SC_ERR_INVALID_ARG;
+  g_rows_kernel.store(which);
+  return SC_OK;
+}
 
 int sc_workspace_status(void* workspace, size_t ws_bytes, void* stream) {
   if (!workspace || ws_bytes < kAlign) return SC_ERR_WORKSPACE;

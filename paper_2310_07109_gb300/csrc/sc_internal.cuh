@@ -75,6 +75,8 @@ struct LayerParams {
                          //   (slot = query tile mod band_slots)
   int band_slots;        // kMaxBandTiles, or kWideBandTiles with wide
   int wide;              // rows kernel: one query tile per CTA (256 < w on long sequences)
+  int band;              // the single-pass band kernel computes the rows (w <= 256)
+  int sms;               // multiprocessors of the device (the band kernel's grid)
   float* gpart;          // [B][H][T][4][kMaxGlobal] column sums of global keys over far rows,
                          //   per (query tile, 32-row warp slice)
   float* gstat;          // [B][H][T][4][kMaxGlobal][2] (max, sum) of global rows per

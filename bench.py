@@ -433,6 +433,8 @@ def run_native(args, wl):
         dist.init_process_group("nccl", device_id=dev)
     sc_build.build_library()
     sc.load()
+    sc.select_rows_kernel(sc.SC_ROWS_SINGLE_PASS if args.rows_kernel == "single-pass"
+                          else sc.SC_ROWS_TWO_PASS)
 
     redraws = wk.stored_redraws(wl)
     inp = wk.make_inputs(wl, redraws)
@@ -677,7 +679,7 @@ def run_native(args, wl):
             "config": {"workload": wl.describe(), "n_layers": wl.n_layers, "batch": wl.B,
                        "seq_len": wl.L, "heads": wl.H, "head_dim": wl.d, "window": wl.w,
                        "globals": len(gpos), "parallelism": "replicas" if world > 1 else "single",
-                       "cuda_graph": graph is not None,
+                       "cuda_graph": graph is not None, "rows_kernel": args.rows_kernel,
                        "l2": ("timed steps rotate over %d copies of the inputs and outputs "
                               "(%.0f MB touched by layer 0 per copy, L2 %.0f MB)" % (
                                   n_copies, lay0 / 1e6, l2_bytes / 1e6)) if n_copies > 1 else
@@ -925,6 +927,9 @@ def main():
     ap.add_argument("--no-graph", action="store_true",
                     help="call the library directly for each timed step instead of replaying "
                          "a captured CUDA graph")
+    ap.add_argument("--rows-kernel", choices=["two-pass", "single-pass"], default="two-pass",
+                    help="design of the per-layer attention for windows up to 256 "
+                         "(sc_select_rows_kernel)")
     args = ap.parse_args()
     wl = pick_workload(args.workload)
     encoder = args.workload.startswith("encoder")

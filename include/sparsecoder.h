@@ -240,7 +240,10 @@ int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspac
  * the gather of the next layer's rows, and events[2+3*n_layers] after the
  * cluster kernel of the short sequences.  Events of kernels that a call does
  * not launch are recorded anyway (back to back).  n_events >= 3 + 3 * n_layers.
- * The events are caller-owned. */
+ * A NULL entry records nothing at that point, so that kernels on both sides of
+ * it stay chained (programmatic dependent launch) as in an uninstrumented call,
+ * e.g. events[2] = NULL times layer 0's rows and cols kernels together as they
+ * overlap.  The events are caller-owned. */
 int sc_stack_forward_profiled(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
                               void* stream, void** events, int n_events);
 

@@ -273,8 +273,9 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
     pad_mask: uint8 [B, L] cuda tensor or None; alpha: host sequence [n_layers],
     the value of the keep rule ``keep_rule`` (an SC_KEEP_* value) per layer.
-    events: optional list of >= 3 + 3 * n_layers torch.cuda.Event(enable_timing=True),
-    recorded around every kernel on the launching stream (sc_stack_forward_profiled).
+    events: optional list of >= 3 + 3 * n_layers torch.cuda.Event(enable_timing=True)
+    or None (nothing recorded at that point), recorded around the kernels on the
+    launching stream (sc_stack_forward_profiled).
     no_tail: run every layer through the per-layer kernels (SC_STACK_NO_TAIL).
     o_last_only: write no O but the last layer's, to out["O_last"] [B, L, H, 64]
     (O = NULL in the arguments).
@@ -302,7 +303,8 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
         _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
                                        _stream_handle(stream)))
     else:
-        handles = (ctypes.c_void_p * len(events))(*[e.cuda_event for e in events])
+        handles = (ctypes.c_void_p * len(events))(
+            *[None if e is None else e.cuda_event for e in events])
         _check(load().sc_stack_forward_profiled(ctypes.byref(a), _ptr(ws), ws.numel(),
                                                 _stream_handle(stream), handles, len(events)))
     return out

@@ -533,7 +533,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   pp.n_global = a->n_global;
   for (int g = 0; g < a->n_global; ++g) pp.global_pos[g] = a->global_pos[g];
   auto mark = [&](int k) {
-    return events == nullptr ||
+    return events == nullptr || events[k] == nullptr ||
            cudaEventRecord(static_cast<cudaEvent_t>(events[k]), st) == cudaSuccess;
   };
   cudaError_t e;
@@ -726,8 +726,6 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
 int sc_stack_forward_profiled(const sc_stack_args* a, void* workspace, size_t ws_bytes,
                               void* stream, void** events, int n_events) {
   if (!a || !events || a->n_layers < 1 || n_events < 3 + 3 * a->n_layers) return SC_ERR_INVALID_ARG;
-  for (int k = 0; k < 3 + 3 * a->n_layers; ++k)
-    if (!events[k]) return SC_ERR_INVALID_ARG;
   return stack_forward_impl(a, workspace, ws_bytes, stream, events, n_events);
 }
 

@@ -674,9 +674,7 @@ struct ColsSmem {
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  float gsum[kMaxGlobal];
   int flag;
-  float wpart[kColsThreads / 32];
   int gnew[kMaxGlobal];
   // each key tile's part of the global rows' P V (warpgroup X), added in
   // tile order into the pair's part
@@ -831,6 +829,28 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     // slice) pieces; the warp combines them in a fixed order
     const size_t base_slot = (static_cast<size_t>(b) * p.H + h) * p.T * 4 * kMaxGlobal;
     float me[2][4], se[2][4];
+    // the far-row sums (rows whose band does not reach the key) of a global
+    // key among this warp's 32 keys, over the (query tile, warp slice) pieces
+    // of this head: lane k loads pieces k, k+32, k+64, k+96 (at most one
+    // global key per warp is usual; more are summed one after another below)
+    const int wk0 = j0 + 32 * wq;
+    float far[4] = {0.f, 0.f, 0.f, 0.f};
+    int far_g = -1;
+    if (active && ngp) {
+#pragma unroll 1
+      for (int g = 0; g < ng; ++g)
+        if (sm.gc[g] >= wk0 && sm.gc[g] < wk0 + 32) {
+          far_g = g;
+          break;
+        }
+      if (far_g >= 0) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int ent = lane + 32 * k;
+          far[k] = ent < 4 * Tn ? __ldcg(p.gpart + base_slot + ent * kMaxGlobal + far_g) : 0.f;
+        }
+      }
+    }
 #pragma unroll
     for (int gg = 0; gg < 2; ++gg) {
       const int g = warp + 8 * gg;
@@ -861,6 +881,24 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     float acc = 0.f;
 #pragma unroll
     for (int u = 0; u < kWideBandTiles; ++u) acc += part[u];
+    // far rows of the global keys among this warp's keys (gc increases with
+    // g, so they are consecutive entries of the list)
+    if (far_g >= 0) {
+#pragma unroll 1
+      for (int g = far_g; g < ng; ++g) {
+        const int cg = sm.gc[g];
+        if (cg >= wk0 + 32) break;
+        if (g != far_g) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int ent = lane + 32 * k;
+            far[k] = ent < 4 * Tn ? __ldcg(p.gpart + base_slot + ent * kMaxGlobal + g) : 0.f;
+          }
+        }
+        const float fs = warp_sum((far[0] + far[1]) + (far[2] + far[3]));
+        if (j == cg) acc += fs;
+      }
+    }
     const bool ok = active;
     float x[16];
 
@@ -1000,53 +1038,11 @@ __global__ void __launch_bounds__(kColsThreads, 2)
     hs[u] = my_key && u < p.H ? __ldcg(ap + static_cast<size_t>(u) * p.L) : 0.f;
   for (int h0 = kTailMaxHeads; my_key && h0 < p.H; ++h0)   // more than 16 heads
     a += __ldcg(ap + static_cast<size_t>(h0) * p.L);
-  // far-row partial sums of each global key that lies in this pair, over heads
-  // and (query tile, warp) slices: spread over the whole CTA, every load
-  // issued before the sums, reduced in a fixed order
-  for (int g = 0; g < ng; ++g) {
-    const int cg = sm.gc[g];
-    if (cg < j0 || cg >= jn) continue;   // CTA-uniform
-    const int per_head = Tn * 4, total = p.H * per_head;
-    const float* gp = p.gpart + static_cast<size_t>(b) * p.H * p.T * 4 * kMaxGlobal + g;
-    constexpr int kPer = 8;
-    float e[kPer];
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int k = tid + u * kColsThreads;
-      const int hh = k / per_head, q4 = k - hh * per_head;   // q4 = 4 * tile + warp
-      e[u] = k < total ? __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal) : 0.f;
-    }
-    float gv = 0.f;
-    for (int k0 = 0; k0 < total; k0 += kPer * kColsThreads) {
-      if (k0 > 0) {
-#pragma unroll
-        for (int u = 0; u < kPer; ++u) {
-          const int k = k0 + tid + u * kColsThreads;
-          const int hh = k / per_head, q4 = k - hh * per_head;
-          e[u] = k < total ? __ldcg(gp + (static_cast<size_t>(hh) * p.T * 4 + q4) * kMaxGlobal)
-                           : 0.f;
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kPer; ++u) gv += e[u];
-    }
-    gv = warp_sum(gv);
-    if (lane == 0) sm.wpart[warp] = gv;
-    __syncthreads();
-    if (tid == 0) {
-      float ga = 0.f;
-      for (int w = 0; w < kColsThreads / 32; ++w) ga += sm.wpart[w];
-      sm.gsum[g] = ga;
-    }
-    __syncthreads();
-  }
   if (my_key) {
     float hsum = 0.f;
 #pragma unroll
     for (int u = 0; u < kTailMaxHeads; ++u) hsum += hs[u];   // heads in order
     a = hsum + a;
-    for (int g = 0; g < ng; ++g)
-      if (sm.gc[g] == jj) a += sm.gsum[g];
     const float s = a / static_cast<float>(p.H * n);
     v.scores[static_cast<size_t>(b) * p.L + jj] = s;
     if (p.keep_rule != kKeepTopRatio) {   // the top-ratio cut needs every score first

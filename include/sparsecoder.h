@@ -273,7 +273,9 @@ int sc_stack_launch_count(const sc_stack_args* args, int* count);
  *            it was.
  * workspace  DEVICE memory of sc_stack_host_workspace_size(n_layers, B, L, H)
  *            bytes (256-byte aligned): the scratch of sc_stack_forward followed
- *            by device copies of the results.
+ *            by device copies of the results of the layers that run on the
+ *            per-layer kernels (the cluster kernel writes the results of the
+ *            layers it runs to the host buffers directly).
  *
  * Asynchronous on `stream` like every call: the host buffers must stay
  * allocated and unmodified (inputs) or unread (results) until the stream has

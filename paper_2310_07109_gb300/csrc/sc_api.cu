@@ -464,12 +464,24 @@ static int stack_plan(const sc_stack_args* a, bool* use_tail, bool* per_layer) {
   return SC_OK;
 }
 
+// The caller's page-locked result buffers of a host-buffer call (device-mapped
+// addresses): the cluster kernel writes its layers' results there directly.
+struct HostResults {
+  uint16_t* O;
+  uint16_t* O_last;
+  float* scores;
+  int32_t* pos;
+  int32_t* len;
+};
+
 // host_io: Q, K, V (and pad_mask) are device-mapped addresses of host memory,
 // which only the gather and cluster kernels read (plain loads): the tensor
 // maps of the "source" slot are pointed at the compacted copies and never
-// selected, and every layer's rows are gathered.
+// selected, and every layer's rows are gathered; hres (host_io only): where
+// the cluster kernel puts its results.
 static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
-                              void* stream, void** events, int n_events, bool host_io = false) {
+                              void* stream, void** events, int n_events, bool host_io = false,
+                              const HostResults* hres = nullptr) {
   if (!a) return SC_ERR_INVALID_ARG;
   if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
@@ -709,6 +721,13 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     tp.status = p.status;
     for (int t = 0; t < 3; ++t) tp.src[t] = src[t];
     tp.src_host = host_io ? 1 : 0;
+    if (hres != nullptr) {
+      tp.hO = hres->O;
+      tp.hO_last = hres->O_last;
+      tp.hscores = hres->scores;
+      tp.hpos = hres->pos;
+      tp.hlen = hres->len;
+    }
     tp.n_global = a->n_global;
     for (int g = 0; g < a->n_global; ++g) tp.global_pos[g] = a->global_pos[g];
     for (int l = 0; l < a->n_layers; ++l) tp.alpha[l] = a->alpha[l];
@@ -829,7 +848,11 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   d.scores = reinterpret_cast<float*>(ws + hl.scores);
   d.pos = reinterpret_cast<int32_t*>(ws + hl.pos);
   d.len = reinterpret_cast<int32_t*>(ws + hl.len);
-  if ((rc = stack_forward_impl(&d, workspace, hl.O, stream, nullptr, 0, true)) != SC_OK) return rc;
+  const HostResults hres{static_cast<uint16_t*>(o), static_cast<uint16_t*>(o_last),
+                         static_cast<float*>(sc), static_cast<int32_t*>(ps),
+                         static_cast<int32_t*>(ln)};
+  if ((rc = stack_forward_impl(&d, workspace, hl.O, stream, nullptr, 0, true, &hres)) != SC_OK)
+    return rc;
   bool use_tail = false, per_layer = true;
   if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
   int dev = 0, sms = 0;
@@ -850,14 +873,16 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (use_tail) {
     // the per-layer results go out beside the cluster kernel, on the SMs it
-    // leaves idle (one CTA per SM fits beside one of its CTAs), the rest after it
+    // leaves idle (one CTA per SM fits beside one of its CTAs); the cluster
+    // kernel writes its own layers' results to the host buffers itself.  The
+    // export ends with a grid wait, so the call ends after the cluster kernel.
     e.part = 1;
     if ((ce = launch_export(e, sms, st)) != cudaSuccess) return fail_cuda("launch export kernel", ce);
-    e.part = 2;
   } else {
     e.part = 0;
+    if ((ce = launch_export(e, 4 * sms, st)) != cudaSuccess)
+      return fail_cuda("launch export kernel", ce);
   }
-  if ((ce = launch_export(e, 4 * sms, st)) != cudaSuccess) return fail_cuda("launch export kernel", ce);
   return SC_OK;
 }
 
@@ -871,7 +896,7 @@ int sc_stack_host_launch_count(const sc_stack_args* a, int* count) {
   if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
   int k = 2;   // padding removal / global lookup, and the export
   if (per_layer) k += 1 + 2 * a->n_layers + (a->n_layers - 1);
-  if (use_tail) k += 2;   // the cluster kernel, and the export in two parts
+  if (use_tail) k += 1;   // the cluster kernel (it writes its own layers' results)
   *count = k;
   return SC_OK;
 }

@@ -203,8 +203,10 @@ struct ExportParams {
   int32_t* hpos;
   int32_t* hlen;
   // part 0: every layer.  With the cluster kernel, part 1 copies the layers
-  // l < tail_from[b], complete before that kernel, while it runs, and part 2
-  // the layers l >= tail_from[b] after it.
+  // l < tail_from[b], complete before that kernel, while it runs (the cluster
+  // kernel writes the layers l >= tail_from[b] to the host buffers itself);
+  // part 2, the layers l >= tail_from[b] from the device copies, is not used
+  // by the host-buffer call.
   int part;
   const int32_t* tail_from;    // [B] (parts 1 and 2)
 };
@@ -222,6 +224,16 @@ struct TailParams {
   // nonzero: src is host memory; the next layer's rows are not prefetched
   // (that would pull the rows of the tokens a layer prunes over the host link)
   int src_host;
+  // host-buffer call: the results of the layers run here go straight to the
+  // caller's page-locked buffers (device-mapped addresses, same layouts as
+  // O / O_last / scores / pos / len): the entering layer's len and pos, then
+  // each layer's O rows, scores, next pos and len; nullptr: device results
+  // as above
+  uint16_t* hO;
+  uint16_t* hO_last;
+  float* hscores;
+  int32_t* hpos;
+  int32_t* hlen;
   int n_global;
   int global_pos[kMaxGlobal];
   float alpha[kTailMaxLayers];   // the keep rule's value per layer

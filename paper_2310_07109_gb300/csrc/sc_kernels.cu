@@ -1293,8 +1293,9 @@ __global__ void __launch_bounds__(kExportThreads)
       }
     }
   }
-  // part 1 completes only after the cluster kernel, so that part 2, which
-  // waits for part 1's grid, finds that kernel's results complete
+  // part 1 completes only after the cluster kernel (which writes its own
+  // layers' results to the host buffers), so that the call's last kernel
+  // ends after every result is written
   if (e.part == 1) pdl_wait();
 }
 

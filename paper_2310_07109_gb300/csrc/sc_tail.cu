@@ -139,11 +139,19 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   const int l0 = __ldcg(p.tail_from + b);
   if (l0 >= n_layers) return;
   const int n0 = __ldcg(p.len + static_cast<size_t>(l0) * B + b);
+  // where this kernel's results go: the device arrays, or the caller's host buffers
+  const bool to_host = p.hlen != nullptr;
+  int32_t* const out_len = to_host ? p.hlen : p.len;
+  int32_t* const out_pos = to_host ? p.hpos : p.pos;
+  float* const out_scores = to_host ? p.hscores : p.scores;
+  uint16_t* const out_O = to_host ? p.hO : p.O;
+  uint16_t* const out_O_last = to_host ? p.hO_last : p.O_last;
   if (n0 <= 0 || n0 > kTailMax) {
     if (h == 0 && threadIdx.x == 0) {
       if (n0 > kTailMax) atomicOr(p.status, kStatusInternal);
       else
-        for (int l = l0; l < n_layers; ++l) p.len[static_cast<size_t>(l + 1) * B + b] = 0;
+        for (int l = l0; l < n_layers; ++l) out_len[static_cast<size_t>(l + 1) * B + b] = 0;
+      if (to_host && n0 <= kTailMax) p.hlen[static_cast<size_t>(l0) * B + b] = max(n0, 0);
     }
     return;
   }
@@ -172,6 +180,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
     fence_mbar_init();
   }
   if (tid < kMaxGlobal) sm.gpos[tid] = tid < p.n_global ? p.global_pos[tid] : -1;
+  if (to_host && h == 0 && tid == 0) p.hlen[static_cast<size_t>(l0) * B + b] = n0;
   if (warp == 8) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
@@ -179,6 +188,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
   for (int c = tid; c < kTailChunks * 32; c += kTailThreads) {
     int ps = -1;
     if (c < n0) ps = __ldcg(p.pos + (static_cast<size_t>(l0) * B + b) * L + c);
+    // the entering layer's tokens go to the host buffers with the rest
+    if (to_host && h == 0 && c < n0) p.hpos[(static_cast<size_t>(l0) * B + b) * L + c] = ps;
     if (c < kTailMax) sm.pos[0][c] = ps;
     const uint32_t bits = __ballot_sync(0xffffffffu, c < n0 && tail_is_global(sm, ps));
     if (lane == 0) sm.gbits[0][c >> 5] = bits;
@@ -465,8 +476,8 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         // the warp's 32 rows leave in two column halves of 64 bytes (no O
         // but the last layer's when O is not kept)
         uint8_t* stage = base + 3 * kTailOpBytes + warp * 2048;
-        uint16_t* const Ol = p.O != nullptr ? p.O + static_cast<size_t>(l) * B * L * H * kHeadDim
-                             : l == n_layers - 1 ? p.O_last : nullptr;
+        uint16_t* const Ol = out_O != nullptr ? out_O + static_cast<size_t>(l) * B * L * H * kHeadDim
+                             : l == n_layers - 1 ? out_O_last : nullptr;
         uint16_t* row0 =
             Ol ? Ol + ((static_cast<size_t>(b) * L + i - (r & 31)) * H + h) * kHeadDim : nullptr;
         const uint32_t rows = __ballot_sync(0xffffffffu, me.valid);
@@ -553,7 +564,7 @@ __global__ void __launch_bounds__(kTailThreads, 1)
           for (int hh = 0; hh < kTailMaxHeads; ++hh)
             if (hh < H) a += v[hh];
           sj[rd] = a / static_cast<float>(H * n);
-          if (h == 0) p.scores[(static_cast<size_t>(l) * B + b) * L + j] = sj[rd];
+          if (h == 0) out_scores[(static_cast<size_t>(l) * B + b) * L + j] = sj[rd];
         }
       }
       // keep flags: the threshold (relative or absolute), or the top-ratio cut
@@ -618,11 +629,11 @@ __global__ void __launch_bounds__(kTailThreads, 1)
         const int k = kpre[rd] + __popc(sm.kbits[rd][warp] & ((1u << lane) - 1u));
         const int ps = sm.pos[cur][j];
         sm.pos[nxt][k] = ps;
-        if (h == 0) p.pos[(static_cast<size_t>(l + 1) * B + b) * L + k] = ps;
+        if (h == 0) out_pos[(static_cast<size_t>(l + 1) * B + b) * L + k] = ps;
       }
       if (tid == 0) {
         sm.n[nxt] = total;
-        if (h == 0) p.len[static_cast<size_t>(l + 1) * B + b] = total;
+        if (h == 0) out_len[static_cast<size_t>(l + 1) * B + b] = total;
       }
       tail_named_sync();
 #pragma unroll

@@ -193,12 +193,13 @@ def test_host_stack_refuses_pageable_memory(sc):
                                            (700, False, True), (300, False, False)])
 def test_host_launch_count(sc, L, pad, no_tail):
     """The host-buffer call's plan: the device call's, plus the layer-0 gather
-    (when the per-layer kernels run and no padding already forces it) and the
-    export (in two parts beside and after the cluster kernel)."""
+    (when the per-layer kernels run and no padding already forces it) and one
+    export (beside the cluster kernel, which writes its own layers' results to
+    the host buffers, or after the per-layer kernels)."""
     dev = sc.stack_launch_count(12, 2, L, 12, 64, [0, 5], pad, no_tail=no_tail)
     host = sc.stack_launch_count(12, 2, L, 12, 64, [0, 5], pad, no_tail=no_tail, host=True)
     per_layer = L > sc.TAIL_MAX_LEN or no_tail
-    assert host == dev + (1 if per_layer and not pad else 0) + (1 if no_tail else 2)
+    assert host == dev + (1 if per_layer and not pad else 0) + 1
 
 
 def test_host_stack_last_layer_output_only(sc):

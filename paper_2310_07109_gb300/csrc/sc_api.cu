@@ -82,7 +82,7 @@ size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
 
 struct WsLayout {
   size_t status, acc, colpart, gpart, gstat, og, keep, cnt_tile, cnt_seq, rows_done, cols_done,
-      gcur, ng,
+      gathered, gcur, ng,
       ident,
       tail_from,
       loop_layer, qkv, total;
@@ -108,6 +108,7 @@ bool ws_layout(int B, int L, int H, WsLayout* w) {
   w->cnt_seq = take(sizeof(uint32_t) * B);
   w->rows_done = take(sizeof(uint32_t) * B * H);
   w->cols_done = take(sizeof(uint32_t) * B * H);
+  w->gathered = take(sizeof(uint32_t) * B);
   w->gcur = take(sizeof(int32_t) * 2 * B * kMaxGlobal);
   w->ng = take(sizeof(int32_t) * 2 * B);
   w->ident = take(sizeof(int32_t) * 2 * B);
@@ -595,6 +596,11 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     gp.src[t] = src[t];
     gp.dst[t] = cmp[t];
   }
+  // Host buffers: layer 0's rows cross the host link; the gather walks them
+  // sequence by sequence and counts what it has copied, and layer 0's rows and
+  // cols kernels start on a sequence as soon as its rows are in.
+  uint32_t* const gathered = host_io ? reinterpret_cast<uint32_t*>(ws + lay.gathered) : nullptr;
+  const uint32_t gather_target = static_cast<uint32_t>((a->L + 7) / 8);
   if (dev_loop) {
     if (a->pad_mask != nullptr || host_io) {
       // padding removal may have moved rows: compact layer 0 as well
@@ -603,7 +609,9 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
       gp.len = a->len;
       gp.pos = a->pos;
       gp.ident = p.ident;
+      gp.gathered = gathered;
       if ((e = launch_gather(gp, st)) != cudaSuccess) return fail_cuda("launch gather kernel", e);
+      gp.gathered = nullptr;
     }
     LayerParams pd = p;   // workspace slot 0: layer 0's ping-pong buffers
     pd.dev_layer = loop_layer;
@@ -639,6 +647,18 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
     ad.tail_from = tail_from;
     ad.cond = cond;
 
+    // layer 0 ahead of the loop (chained to the kernels before it), the loop
+    // from layer 1 on: the advance kernel sets the loop's condition
+    {
+      LayerParams p0 = pd;
+      p0.gathered = gathered;
+      p0.gather_target = gather_target;
+      cudaError_t le0 = launch_rows(maps, p0, st);
+      if (le0 == cudaSuccess) le0 = launch_cols(maps, p0, st);
+      if (le0 == cudaSuccess) le0 = launch_gather(gd, st);
+      if (le0 == cudaSuccess) le0 = launch_advance(ad, st);
+      if (le0 != cudaSuccess) return fail_cuda("launch layer 0", le0);
+    }
     cudaGraph_t g = nullptr;
     const cudaGraphNode_t* deps = nullptr;
     size_t ndeps = 0;
@@ -676,6 +696,7 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
       continue;
     }
     fill_workspace(&p, ws, lay, l & 1);
+    p.gathered = nullptr;   // only layer 0 of a host-buffer call counts its rows in
     p.layer = l;
     p.src_base = static_cast<long long>(l) * BLt;
     p.len = a->len + static_cast<size_t>(l) * a->B;
@@ -693,7 +714,11 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
       gp.len = p.len;
       gp.pos = p.pos;
       gp.ident = p.ident;
+      gp.gathered = gathered;
       if ((e = launch_gather(gp, st)) != cudaSuccess) return fail_cuda("launch gather kernel", e);
+      gp.gathered = nullptr;
+      p.gathered = gathered;
+      p.gather_target = gather_target;
     }
     if ((e = launch_rows(maps, p, st)) != cudaSuccess) return fail_cuda("launch rows kernel", e);
     if (!mark(2 + 3 * l)) return fail(SC_ERR_CUDA, "event record", "");

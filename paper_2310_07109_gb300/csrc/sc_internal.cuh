@@ -88,6 +88,12 @@ struct LayerParams {
   uint32_t* cnt_seq;     // [B]
   uint32_t* rows_done;   // [B][H]: rows CTAs of (sequence, head) whose results are visible
   uint32_t* cols_done;   // [B][H]: cols CTAs of (sequence, head) whose global-row parts are stored
+  // nonzero: the gather kernel before this launch is still copying later
+  // sequences' rows when it starts: sequence b's rows are complete once
+  // gathered[b] reaches gather_target (the rows and cols kernels wait for it
+  // instead of for the whole gather grid)
+  const uint32_t* gathered;
+  uint32_t gather_target;
   int32_t* kept_cur;     // [B][L] out, or nullptr: current index of each kept token, in order
   int* status;
   // test hook: when nonzero, the first MMA-issuing thread of every rows CTA
@@ -157,6 +163,13 @@ struct GatherParams {
   long long tok_stride, row_stride;
   int len_stride;
   const int32_t* ident_slot[2];
+  // nonzero: the CTAs walk the 8-token items sequence by sequence (grid
+  // stride) and raise gathered[b] (release) once an item of sequence b is
+  // copied, so that the next kernel can start on sequence b while later
+  // sequences are still being copied (layer 0 of the host-buffer call, whose
+  // rows cross the host link); their successors are launched only once the
+  // kernels before this one are complete
+  uint32_t* gathered;          // [B]
 };
 
 // One step of the device-driven layer loop: layer += 1, and the loop goes on

@@ -113,8 +113,11 @@ template <bool kWide>
 __global__ void __launch_bounds__(kRowsThreads, 1)
     sc_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ LayerParams p) {
   // the cols kernel is scheduled once every CTA here has passed this wait, so
-  // what the kernels before this one wrote is complete when it starts
-  pdl_wait();
+  // what the kernels before this one wrote is complete when it starts (with
+  // p.gathered, the gather kernel before this one lets it start only once the
+  // kernels before the gather are complete, and each CTA waits below for its
+  // own sequence's rows)
+  if (p.gathered == nullptr) pdl_wait();
   pdl_launch_dependents();
   // grid: pairs of query tiles (single tiles with a wide window),
   // (sequence, head)-major, so that the CTAs of a (sequence, head) finish
@@ -181,12 +184,15 @@ __global__ void __launch_bounds__(kRowsThreads, 1)
     mbar_init(&sm.bar_stall, 1);
     sm.abort = 0;
     fence_mbar_init();
+    // this sequence's rows may still be crossing the host link
+    if (p.gathered != nullptr) wait_count(p.gathered + b, p.gather_target, &sm.abort);
   }
   if (tid < kMaxGlobal) sm.gc[tid] = tid < ng ? gc_raw : -1;
   if (warp == 9) tmem_alloc(&sm.tmem_base, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (p.gathered != nullptr) fence_proxy_async_global();   // the copies, before any TMA load
   const uint32_t tm = sm.tmem_base;
   volatile int* abort_flag = &sm.abort;
 
@@ -765,6 +771,12 @@ __global__ void __launch_bounds__(kColsThreads, 2)
 
   if (warp == 8) {
     const RowSource rs = row_source(p, v, b);
+    // this sequence's rows may still be crossing the host link
+    if (p.gathered != nullptr) {
+      if (lane == 0) wait_count(p.gathered + b, p.gather_target, abort_flag);
+      __syncwarp();
+      fence_proxy_async_global();
+    }
     if (lane == 0) {
       mbar_arrive_expect_tx(&sm.bar_kv, (hasB ? 4 : 2) * kTileBytes + ngp * 128);
       for (int X = 0; X < (hasB ? 2 : 1); ++X) {
@@ -1183,29 +1195,14 @@ __device__ void finalize_sequence(const LayerParams& p, const LayerView& v, int 
 constexpr int kGatherTokens = 8;
 constexpr int kGatherThreads = 256;
 
-// 8 tokens x 3 tensors per CTA; with H = 12 each thread moves at most nine
-// 16-byte vectors, all loads issued before any store.
-__global__ void __launch_bounds__(kGatherThreads)
-    sc_gather_kernel(const GatherParams g) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int b = blockIdx.y;
-  int layer = g.layer;
-  long long src_base = g.src_base;
-  const int32_t* lenp = g.len;
-  const int32_t* posp = g.pos;
-  const int32_t* identp = g.ident;
-  if (g.dev_layer != nullptr) {
-    layer = __ldcg(g.dev_layer) + 1;
-    if (layer >= g.n_layers) return;
-    src_base = layer * g.tok_stride;
-    lenp += static_cast<size_t>(layer) * g.len_stride;
-    posp += layer * g.row_stride;
-    identp = g.ident_slot[layer & 1];
-  }
+// One item: tokens 8 ch .. 8 ch + 7 of sequence b, 3 tensors; with H = 12 each
+// thread moves at most nine 16-byte vectors, all loads issued before any store.
+__device__ __forceinline__ void gather_item(const GatherParams& g, int b, int ch, int layer,
+                                            long long src_base, const int32_t* lenp,
+                                            const int32_t* posp, const int32_t* identp) {
   if (g.tail_from != nullptr && __ldcg(g.tail_from + b) <= layer) return;
   const int n = __ldcg(lenp + b);
-  const int c0 = blockIdx.x * kGatherTokens;
+  const int c0 = ch * kGatherTokens;
   if (__ldcg(identp + b) != 0 || c0 >= n) return;
   const int cnt = min(kGatherTokens, n - c0);
   const int vec = g.H * kHeadDim / 8;  // 16-byte vectors per token row
@@ -1234,6 +1231,48 @@ __global__ void __launch_bounds__(kGatherThreads)
 #pragma unroll
       for (int u = 0; u < kPer; ++u)
         if (so[u] >= 0) reinterpret_cast<uint4*>(g.dst[t])[doff[u]] = v[t][u];
+  }
+}
+
+// One CTA per item (grid: chunks x sequences), or with g.gathered a grid-stride
+// walk over the items sequence by sequence that counts the items done.
+__global__ void __launch_bounds__(kGatherThreads)
+    sc_gather_kernel(const GatherParams g) {
+  if (g.gathered == nullptr) {
+    pdl_launch_dependents();
+    pdl_wait();
+  } else {
+    // the successor starts once every CTA is here: what the kernels before
+    // this one wrote is complete by then
+    pdl_wait();
+    pdl_launch_dependents();
+  }
+  int layer = g.layer;
+  long long src_base = g.src_base;
+  const int32_t* lenp = g.len;
+  const int32_t* posp = g.pos;
+  const int32_t* identp = g.ident;
+  if (g.dev_layer != nullptr) {
+    layer = __ldcg(g.dev_layer) + 1;
+    if (layer >= g.n_layers) return;
+    src_base = layer * g.tok_stride;
+    lenp += static_cast<size_t>(layer) * g.len_stride;
+    posp += layer * g.row_stride;
+    identp = g.ident_slot[layer & 1];
+  }
+  if (g.gathered == nullptr) {
+    gather_item(g, blockIdx.y, blockIdx.x, layer, src_base, lenp, posp, identp);
+    return;
+  }
+  const int nch = (g.L + kGatherTokens - 1) / kGatherTokens;
+  for (int it = blockIdx.x; it < g.B * nch; it += gridDim.x) {
+    const int b = it / nch;
+    gather_item(g, b, it - b * nch, layer, src_base, lenp, posp, identp);
+    __syncthreads();   // every copy of the item is stored ...
+    if (threadIdx.x == 0) {
+      __threadfence();
+      red_release_add_u32(g.gathered + b, 1u);   // ... before it is counted
+    }
   }
 }
 
@@ -1502,7 +1541,21 @@ cudaError_t launch_export(const ExportParams& e, int ctas, cudaStream_t st) {
 }
 
 cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {
-  dim3 grid((g.L + kGatherTokens - 1) / kGatherTokens, g.B);
+  const int nch = (g.L + kGatherTokens - 1) / kGatherTokens;
+  if (g.gathered != nullptr) {
+    // enough CTAs to keep the host link busy (about 2 MB in flight), few
+    // enough that the items complete nearly in order, so that the first
+    // sequences are in well before the last (measured on config 4 end to end:
+    // 608 CTAs 0.489 ms, 152 0.484, 96 0.468, 64 0.469, 32 0.472)
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int items = g.B * nch;
+    return launch_chained(sc_gather_kernel, dim3(std::max(1, std::min(items, std::max(32, sms / 2)))),
+                          dim3(kGatherThreads), 0, st, g);
+  }
+  dim3 grid(nch, g.B);
   return launch_chained(sc_gather_kernel, grid, dim3(kGatherThreads), 0, st, g);
 }
 

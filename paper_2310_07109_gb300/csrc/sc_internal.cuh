@@ -163,12 +163,13 @@ struct GatherParams {
   long long tok_stride, row_stride;
   int len_stride;
   const int32_t* ident_slot[2];
-  // nonzero: the CTAs walk the 8-token items sequence by sequence (grid
-  // stride) and raise gathered[b] (release) once an item of sequence b is
-  // copied, so that the next kernel can start on sequence b while later
-  // sequences are still being copied (layer 0 of the host-buffer call, whose
-  // rows cross the host link); their successors are launched only once the
-  // kernels before this one are complete
+  // nonzero (sc_gather_seq_kernel, the layer given explicitly): the CTAs walk
+  // the 8-token items sequence by sequence (grid stride) and raise
+  // gathered[b] (release) once an item of sequence b is copied, so that the
+  // next kernel can start on sequence b while later sequences are still being
+  // copied (layer 0 of the host-buffer call, whose rows cross the host link);
+  // their successors are launched only once the kernels before this one are
+  // complete
   uint32_t* gathered;          // [B]
 };
 

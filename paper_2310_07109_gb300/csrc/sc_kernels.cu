@@ -1234,19 +1234,11 @@ __device__ __forceinline__ void gather_item(const GatherParams& g, int b, int ch
   }
 }
 
-// One CTA per item (grid: chunks x sequences), or with g.gathered a grid-stride
-// walk over the items sequence by sequence that counts the items done.
+// The per-layer gather: one CTA per item (grid: chunks x sequences).
 __global__ void __launch_bounds__(kGatherThreads)
     sc_gather_kernel(const GatherParams g) {
-  if (g.gathered == nullptr) {
-    pdl_launch_dependents();
-    pdl_wait();
-  } else {
-    // the successor starts once every CTA is here: what the kernels before
-    // this one wrote is complete by then
-    pdl_wait();
-    pdl_launch_dependents();
-  }
+  pdl_launch_dependents();
+  pdl_wait();
   int layer = g.layer;
   long long src_base = g.src_base;
   const int32_t* lenp = g.len;
@@ -1260,14 +1252,22 @@ __global__ void __launch_bounds__(kGatherThreads)
     posp += layer * g.row_stride;
     identp = g.ident_slot[layer & 1];
   }
-  if (g.gathered == nullptr) {
-    gather_item(g, blockIdx.y, blockIdx.x, layer, src_base, lenp, posp, identp);
-    return;
-  }
+  gather_item(g, blockIdx.y, blockIdx.x, layer, src_base, lenp, posp, identp);
+}
+
+// The gather with per-sequence counts (g.gathered): a grid-stride walk over
+// the items sequence by sequence; gathered[b] is raised (release) once an item
+// of sequence b is copied.  Its successor is launched once every CTA has
+// passed the grid wait, so what the kernels before this one wrote is complete
+// by then.  Used for the layer (given explicitly) whose rows cross the host link.
+__global__ void __launch_bounds__(kGatherThreads)
+    sc_gather_seq_kernel(const GatherParams g) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int nch = (g.L + kGatherTokens - 1) / kGatherTokens;
   for (int it = blockIdx.x; it < g.B * nch; it += gridDim.x) {
     const int b = it / nch;
-    gather_item(g, b, it - b * nch, layer, src_base, lenp, posp, identp);
+    gather_item(g, b, it - b * nch, g.layer, g.src_base, g.len, g.pos, g.ident);
     __syncthreads();   // every copy of the item is stored ...
     if (threadIdx.x == 0) {
       __threadfence();
@@ -1552,7 +1552,8 @@ cudaError_t launch_gather(const GatherParams& g, cudaStream_t st) {
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
     const int items = g.B * nch;
-    return launch_chained(sc_gather_kernel, dim3(std::max(1, std::min(items, std::max(32, sms / 2)))),
+    return launch_chained(sc_gather_seq_kernel,
+                          dim3(std::max(1, std::min(items, std::max(32, sms / 2)))),
                           dim3(kGatherThreads), 0, st, g);
   }
   dim3 grid(nch, g.B);

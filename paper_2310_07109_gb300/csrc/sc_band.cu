@@ -850,8 +850,14 @@ __global__ void __launch_bounds__(kBandThreads, 1)
 }
 
 cudaError_t configure_band() {
-  cudaError_t e = cudaFuncSetAttribute(sc_band_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(kBandDyn));
+  // the warpgroups' register split (setmaxnreg) needs the whole launch
+  // allocation: with fewer registers a thread, an increase would never be granted
+  cudaFuncAttributes fa;
+  cudaError_t e = cudaFuncGetAttributes(&fa, sc_band_kernel);
+  if (e == cudaSuccess && fa.numRegs * kBandThreads < 65536) e = cudaErrorInvalidConfiguration;
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(sc_band_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kBandDyn));
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(sc_band_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);

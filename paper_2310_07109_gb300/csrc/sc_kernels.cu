@@ -70,9 +70,10 @@ namespace sc {
 // warpgroup 2 gives registers back so that the softmax warps, which hold a
 // whole 128-column row of S, get 200: 128 x 96 + 256 x 200 = 63488 <= 384 x 168.
 constexpr int kRowsThreads = 384;
+constexpr int kRowsLaunchRegs = 168;
 constexpr int kRowsCtlRegs = 96;
 constexpr int kRowsSoftmaxRegs = 200;
-static_assert(128 * kRowsCtlRegs + 256 * kRowsSoftmaxRegs <= kRowsThreads * 168,
+static_assert(128 * kRowsCtlRegs + 256 * kRowsSoftmaxRegs <= kRowsThreads * kRowsLaunchRegs,
               "register split exceeds the launch allocation");
 constexpr int kPairTiles = kMaxBandTiles + 1;
 // V slots: with six key tiles only the sixth reuses a slot, that of the first;
@@ -1498,6 +1499,11 @@ cudaError_t configure_kernels() {
   // the attention kernels use most of an SM's shared memory
   cudaError_t e = configure_band();
   for (auto k : {sc_rows_kernel<false>, sc_rows_kernel<true>}) {
+    // the warpgroups' register split (setmaxnreg) needs the whole launch
+    // allocation: with fewer registers a thread, an increase would never be granted
+    cudaFuncAttributes fa;
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k);
+    if (e == cudaSuccess && fa.numRegs < kRowsLaunchRegs) e = cudaErrorInvalidConfiguration;
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(kRowsDyn));

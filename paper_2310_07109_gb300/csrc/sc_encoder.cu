@@ -65,15 +65,26 @@ __device__ __forceinline__ uint16_t bf16_bits(float x) {
 // 7.1.26 (|error| <= 1.5e-7): erf(z) = 1 - (a1 t + ... + a5 t^5) exp(-z^2),
 // t = 1 / (1 + p z), z >= 0, extended as an odd function.  With
 // h = (1 - erf(|x| / sqrt 2)) / 2:  GELU(x) = x (1 - h) for x >= 0, x h below.
-__device__ __forceinline__ float gelu_erf(float x) {
-  const float z = fabsf(x) * 0.70710678118654752f;
-  const float t = __fdividef(1.f, fmaf(0.3275911f, z, 1.f));
-  float poly = fmaf(1.061405429f, t, -1.453152027f);
-  poly = fmaf(poly, t, 1.421413741f);
-  poly = fmaf(poly, t, -0.284496736f);
-  poly = fmaf(poly, t, 0.254829592f);
-  const float h = 0.5f * poly * t * __expf(-z * z);
-  return x * (x >= 0.f ? 1.f - h : h);
+// Two values at once: the polynomial, the products and the exponent in packed
+// fp32 pairs (the coefficients carry the factor 1/2), with
+// exp(-z^2) = 2^(-z^2 log2 e).
+__device__ __forceinline__ void gelu_erf2(float& x0, float& x1) {
+  const float z0 = fabsf(x0) * 0.70710678118654752f, z1 = fabsf(x1) * 0.70710678118654752f;
+  const uint64_t z = f2_pack(z0, z1);
+  float d0, d1;
+  f2_unpack(f2_fma(z, f2_pack(0.3275911f, 0.3275911f), f2_pack(1.f, 1.f)), d0, d1);
+  const uint64_t t = f2_pack(__fdividef(1.f, d0), __fdividef(1.f, d1));
+  uint64_t poly = f2_fma(f2_pack(0.5307027145f, 0.5307027145f), t,
+                         f2_pack(-0.7265760135f, -0.7265760135f));
+  poly = f2_fma(poly, t, f2_pack(0.7107068705f, 0.7107068705f));
+  poly = f2_fma(poly, t, f2_pack(-0.142248368f, -0.142248368f));
+  poly = f2_fma(poly, t, f2_pack(0.127414796f, 0.127414796f));
+  float e0, e1;
+  f2_unpack(f2_mul(f2_mul(z, z), f2_pack(-1.44269504088896341f, -1.44269504088896341f)), e0, e1);
+  float h0, h1;
+  f2_unpack(f2_mul(f2_mul(poly, t), f2_pack(ex2(e0), ex2(e1))), h0, h1);
+  x0 *= x0 >= 0.f ? 1.f - h0 : h0;
+  x1 *= x1 >= 0.f ? 1.f - h1 : h1;
 }
 
 // Tile t of the launch: column block nt of width bn (fastest, so that the
@@ -259,7 +270,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         if (p.gelu)
 #pragma unroll
-          for (int k = 0; k < 32; ++k) v[k] = gelu_erf(v[k]);
+          for (int k = 0; k < 32; k += 2) gelu_erf2(v[k], v[k + 1]);
         if (res) {
 #pragma unroll
           for (int k = 0; k < 32; k += 8) {

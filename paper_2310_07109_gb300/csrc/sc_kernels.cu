@@ -681,7 +681,7 @@ struct ColsSmem {
   int abort;
   int gc[kMaxGlobal];
   float lse_g[kMaxGlobal];
-  int flag;
+  int flag, flag2;
   int gnew[kMaxGlobal];
   // each key tile's part of the global rows' P V (warpgroup X), added in
   // tile order into the pair's part
@@ -993,14 +993,19 @@ __global__ void __launch_bounds__(kColsThreads, 2)
   }
   if (tid == 0 && sm.abort) atomicOr(p.status, kStatusTimeout);
 
+  // One hand-over for both roles below: this CTA's part of the global rows'
+  // outputs and its column sums are visible before either counter is raised.
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) {
+    sm.flag = ngp && atomicAdd(p.cols_done + b * p.H + h, 1u) == static_cast<uint32_t>(Tp - 1);
+    sm.flag2 = atomicAdd(p.cnt_tile + b * p.T + pr, 1u) == static_cast<uint32_t>(p.H - 1);
+  }
+  __syncthreads();
+
   // ---- last pair of this (sequence, head): the global rows' outputs, the
   // pairs' parts added in pair order
   if (ngp) {
-    __threadfence();
-    __syncthreads();
-    if (tid == 0)
-      sm.flag = (atomicAdd(p.cols_done + b * p.H + h, 1u) == static_cast<uint32_t>(Tp - 1));
-    __syncthreads();
     if (sm.flag) {
       __threadfence();
       const float* part0 =
@@ -1031,11 +1036,7 @@ __global__ void __launch_bounds__(kColsThreads, 2)
   }
 
   // ---- last head of this pair of key tiles: scores and keep flags (fixed head order)
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) sm.flag = (atomicAdd(p.cnt_tile + b * p.T + pr, 1u) == static_cast<uint32_t>(p.H - 1));
-  __syncthreads();
-  if (!sm.flag) return;
+  if (!sm.flag2) return;
   __threadfence();
   const int j0 = 2 * pr * kTile;
   const int jn = min(n, j0 + 2 * kTile);

@@ -392,7 +392,7 @@ def run_reference(args, wl):
         return
     inp = wk.make_inputs(wl, wk.stored_redraws(wl))
     threads = oracle.default_threads()
-    layers = max(1, min(wl.n_layers, args.ref_layers))
+    layers = wl.n_layers if args.ref_layers <= 0 else max(1, min(wl.n_layers, args.ref_layers))
     for s in range(args.warmup):
         oracle_sample(wl, inp, s % wl.B, layers, threads)
     tot_t, tot_tok, cores = 0.0, 0, 1
@@ -458,7 +458,7 @@ def run_native(args, wl):
     def step(events=None, c=0):
         outs[c] = sc.stack_forward(copies[c]["Q"], copies[c]["K"], copies[c]["V"], mask, gpos,
                                    wl.w, alpha, out=outs[c], workspace=ws, events=events,
-                                   keep_rule=wl.keep_rule)
+                                   keep_rule=wl.keep_rule, plain_launches=args.plain_launches)
 
     def barrier():
         if world > 1:
@@ -533,17 +533,19 @@ def run_native(args, wl):
     kept_per_step = int(lens[:wl.n_layers].sum())
     value = whole_job_rate(world, kept_per_step, ms_per_step)
 
-    # ---- kernels launched per timed step.  Eagerly: the library's plan.  A
-    # captured step runs the per-layer kernels in a device-driven loop: prep,
-    # [padding gather], rows + cols + gather + advance for each layer that some
-    # sequence still runs per layer (more than TAIL_MAX_LEN tokens), then the
-    # cluster kernel.
+    # ---- kernels launched per timed step.  A captured step, and an eager call
+    # (which the library records into a graph of its own), runs the per-layer
+    # kernels in a device-driven loop: prep, [padding gather], rows + cols +
+    # gather + advance for each layer that some sequence still runs per layer
+    # (more than TAIL_MAX_LEN tokens), then the cluster kernel.  With plain
+    # launches: the library's plan.
     eager_launches = sc.stack_launch_count(wl.n_layers, wl.B, wl.L, wl.H, wl.w, gpos,
                                            inp["pad_mask"] is not None)
     looped = sum(1 for l in range(wl.n_layers) if (lens[l] > sc.TAIL_MAX_LEN).any())
     graph_launches = (1 + (1 if inp["pad_mask"] is not None else 0) + 4 * looped + 1
                       if wl.L > sc.TAIL_MAX_LEN else 2)
-    launches_per_step = graph_launches if graph is not None else eager_launches
+    launches_per_step = (eager_launches if graph is None and args.plain_launches
+                         else graph_launches)
 
     # ---- per-kernel times on the launching stream (same steps, events between kernels)
     nev = 3 + 3 * wl.n_layers
@@ -651,7 +653,8 @@ def run_native(args, wl):
 
     def host_step():
         sc.stack_forward_host(host["Q"], host["K"], host["V"], hmask, gpos, wl.w, alpha,
-                              out=hout, workspace=hws, keep_rule=wl.keep_rule)
+                              out=hout, workspace=hws, keep_rule=wl.keep_rule,
+                              plain_launches=args.plain_launches)
 
     for _ in range(max(3, args.warmup)):
         host_step()
@@ -698,6 +701,7 @@ def run_native(args, wl):
                        "seq_len": wl.L, "heads": wl.H, "head_dim": wl.d, "window": wl.w,
                        "globals": len(gpos), "parallelism": "replicas" if world > 1 else "single",
                        "cuda_graph": graph is not None, "rows_kernel": args.rows_kernel,
+                       "plain_launches": bool(args.plain_launches),
                        "l2": ("timed steps rotate over %d copies of the inputs and outputs "
                               "(%.0f MB touched by layer 0 per copy, L2 %.0f MB)" % (
                                   n_copies, lay0 / 1e6, l2_bytes / 1e6)) if n_copies > 1 else
@@ -934,8 +938,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="cfg4")
-    ap.add_argument("--ref-layers", type=int, default=2,
-                    help="layers of one sequence per reference step")
+    ap.add_argument("--ref-layers", type=int, default=0,
+                    help="layers of one sequence per reference step (0: all, as the "
+                         "cpu_baseline sample)")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip the oracle legs (CPU baseline and the check of the results)")
     ap.add_argument("--warm-l2", action="store_true",
@@ -945,6 +950,9 @@ def main():
     ap.add_argument("--no-graph", action="store_true",
                     help="call the library directly for each timed step instead of replaying "
                          "a captured CUDA graph")
+    ap.add_argument("--plain-launches", action="store_true",
+                    help="with --no-graph: calls launch every layer's kernels directly "
+                         "(SC_STACK_PLAIN_LAUNCHES) instead of through the library's own graph")
     ap.add_argument("--rows-kernel", choices=["two-pass", "single-pass"], default="two-pass",
                     help="design of the per-layer attention for windows up to 256 "
                          "(sc_select_rows_kernel)")

@@ -141,8 +141,10 @@ typedef struct {
  * pos        int32 [n_layers+1][B][L] out: pos[0] = real tokens after padding
  *            removal, pos[l+1] = survivors of layer l.
  * len        int32 [n_layers+1][B] out.
- * flags      0, or SC_STACK_NO_TAIL: run every layer of every sequence through
- *            the per-layer kernels (see sc_stack_forward).
+ * flags      0, or a combination of SC_STACK_NO_TAIL: run every layer of every
+ *            sequence through the per-layer kernels, and SC_STACK_PLAIN_LAUNCHES:
+ *            launch the kernels directly on the stream even when the call is
+ *            not being captured (see sc_stack_forward).
  * keep_rule  an sc_keep_rule (0 = SC_KEEP_RELATIVE), the same for every layer.
  * O_last     used only when O is NULL: bf16 [B][L][H][64] out, the last layer's
  *            O at its current slots; or NULL as well (no O is written at all,
@@ -151,6 +153,7 @@ typedef struct {
  *            scores come from the probabilities alone (Sec. "Token Pruning").
  */
 #define SC_STACK_NO_TAIL 1
+#define SC_STACK_PLAIN_LAUNCHES 2
 
 typedef struct {
   int n_layers, B, L, H, w;
@@ -209,6 +212,12 @@ int sc_layer_noalloc_status(void* stream);
  * Process-wide; read when a call enqueues its kernels. */
 void sc_debug_stall_waits(unsigned long long ns);
 
+/* Test hook of the graph route of eager stack calls (sc_stack_forward,
+ * sc_stack_forward_host): since the library was loaded, how many calls were
+ * recorded into a new graph (*recorded) and how many launched a kept graph
+ * (*reused).  Process-wide; either pointer may be NULL. */
+void sc_debug_graph_counts(unsigned long long* recorded, unsigned long long* reused);
+
 /* Bytes of workspace a call with these sizes needs (0 on invalid sizes). */
 size_t sc_workspace_size(int B, int L, int H);
 
@@ -228,7 +237,23 @@ int sc_layer_forward(const sc_layer_args* args, void* workspace, size_t workspac
  * schedule clusters of H <= 16 CTAs and n_layers <= 64).  The hand-over is
  * decided on the device: the call never waits for the GPU and can be captured
  * in a CUDA graph.  Results are the same function of the inputs either way
- * (within the stated tolerances). */
+ * (within the stated tolerances).
+ *
+ * Launches: in a CUDA graph (a call made while `stream` is being captured)
+ * the per-layer kernels run in a loop whose condition the device sets, so
+ * the layers that every sequence runs in the cluster kernel launch nothing.
+ * An eager call (stream not capturing) that has both kinds of kernels in its
+ * plan runs the same way: the library records the call into a graph of its
+ * own, keeps the instantiated graph (up to 16 per process, least recently
+ * used replaced first) and launches it on `stream`; a later call with the
+ * same arguments (sizes, device addresses, the alpha and global values, the
+ * workspace, the device, and the process-wide settings read at enqueue)
+ * launches the kept graph without recording again.  Recording and
+ * instantiating make the first call with new arguments cost more host time
+ * (a fraction of a millisecond).  With SC_STACK_PLAIN_LAUNCHES, or when the
+ * plan has only one kind of kernel, an eager call launches its kernels
+ * directly: every layer's per-layer kernels, which skip the sequences that
+ * the cluster kernel runs. */
 int sc_stack_forward(const sc_stack_args* args, void* workspace, size_t workspace_bytes,
                      void* stream);
 
@@ -248,9 +273,14 @@ int sc_stack_forward_profiled(const sc_stack_args* args, void* workspace, size_t
                               void* stream, void** events, int n_events);
 
 /* Number of kernels that sc_stack_forward launches for these arguments (on the
- * current device), in *count.  Only the sizes, n_layers, pad_mask (NULL or
- * not) and the global list are read; no pointer is dereferenced and nothing is
- * launched.  Errors: see sc_status (SC_ERR_CUDA without a usable device). */
+ * current device) when it launches them directly (SC_STACK_PLAIN_LAUNCHES, or
+ * a plan with one kind of kernel), in *count.  A call that runs as a graph
+ * launches prep, [padding-removal gather], then rows, cols, gather and a
+ * loop-advance kernel for layer 0 and for each later layer that some sequence
+ * still runs per layer, then the cluster kernel.  Only the sizes, n_layers,
+ * flags, pad_mask (NULL or not) and the global list are read; no pointer is
+ * dereferenced and nothing is launched.  Errors: see sc_status (SC_ERR_CUDA
+ * without a usable device). */
 int sc_stack_launch_count(const sc_stack_args* args, int* count);
 
 /*

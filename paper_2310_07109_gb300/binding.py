@@ -78,6 +78,7 @@ class LinearArgs(ctypes.Structure):
 
 
 SC_STACK_NO_TAIL = 1
+SC_STACK_PLAIN_LAUNCHES = 2
 # keep rules (sc_keep_rule): what a layer's value alpha means
 SC_KEEP_RELATIVE = 0   # theta = alpha / n
 SC_KEEP_ABSOLUTE = 1   # theta = alpha
@@ -92,7 +93,7 @@ EXPORTED = ["sc_layer_forward", "sc_layer_forward_noalloc", "sc_stack_forward",
             "sc_workspace_size", "sc_workspace_status", "sc_status_string", "sc_last_error",
             "sc_encoder_layer_forward", "sc_encoder_workspace_size", "sc_linear_forward",
             "sc_layer_norm_forward", "sc_layer_noalloc_status", "sc_debug_stall_waits",
-            "sc_select_rows_kernel"]
+            "sc_select_rows_kernel", "sc_debug_graph_counts"]
 
 
 def library_path() -> str:
@@ -127,6 +128,9 @@ def load(build_if_missing: bool = False):
         lib.sc_layer_noalloc_status.argtypes = [ctypes.c_void_p]
         lib.sc_debug_stall_waits.restype = None
         lib.sc_debug_stall_waits.argtypes = [ctypes.c_ulonglong]
+        lib.sc_debug_graph_counts.restype = None
+        lib.sc_debug_graph_counts.argtypes = [ctypes.POINTER(ctypes.c_ulonglong),
+                                              ctypes.POINTER(ctypes.c_ulonglong)]
         lib.sc_select_rows_kernel.restype = ctypes.c_int
         lib.sc_select_rows_kernel.argtypes = [ctypes.c_int]
         lib.sc_stack_forward_profiled.restype = ctypes.c_int
@@ -265,9 +269,21 @@ def debug_stall_waits(ns: int) -> None:
     load().sc_debug_stall_waits(int(ns))
 
 
+def debug_graph_counts():
+    """Test hook (``sc_debug_graph_counts``): (stack calls recorded into a new
+    graph, stack calls that launched a kept graph) since the library was loaded."""
+    rec, reu = ctypes.c_ulonglong(0), ctypes.c_ulonglong(0)
+    load().sc_debug_graph_counts(ctypes.byref(rec), ctypes.byref(reu))
+    return int(rec.value), int(reu.value)
+
+
+def _stack_flags(no_tail, plain_launches):
+    return (SC_STACK_NO_TAIL if no_tail else 0) | (SC_STACK_PLAIN_LAUNCHES if plain_launches else 0)
+
+
 def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
                   stream=None, events=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE,
-                  o_last_only=False):
+                  o_last_only=False, plain_launches=False):
     """The pruned layer stack (``sc_stack_forward``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] cuda tensors in original-position order;
@@ -277,6 +293,8 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
     or None (nothing recorded at that point), recorded around the kernels on the
     launching stream (sc_stack_forward_profiled).
     no_tail: run every layer through the per-layer kernels (SC_STACK_NO_TAIL).
+    plain_launches: launch the kernels directly even when not capturing
+    (SC_STACK_PLAIN_LAUNCHES) instead of through the library's cached graph.
     o_last_only: write no O but the last layer's, to out["O_last"] [B, L, H, 64]
     (O = NULL in the arguments).
     Returns a dict with O (or O_last), scores, pos, len (device tensors).
@@ -298,7 +316,7 @@ def stack_forward(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspac
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
                   _ptr(out.get("O")), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
-                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule), _ptr(out.get("O_last")))
+                  _stack_flags(no_tail, plain_launches), int(keep_rule), _ptr(out.get("O_last")))
     if events is None:
         _check(load().sc_stack_forward(ctypes.byref(a), _ptr(ws), ws.numel(),
                                        _stream_handle(stream)))
@@ -353,7 +371,8 @@ def new_host_outputs(n_layers, B, L, H, o_last_only=False):
 
 
 def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, workspace=None,
-                       stream=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE):
+                       stream=None, no_tail=False, keep_rule=SC_KEEP_RELATIVE,
+                       plain_launches=False):
     """The pruned stack on host tensors (``sc_stack_forward_host``).
 
     Q, K, V: bf16 [n_layers, B, L, H, 64] page-locked CPU tensors (``pin_memory()``);
@@ -380,7 +399,7 @@ def stack_forward_host(Q, K, V, pad_mask, global_pos, w, alpha, *, out=None, wor
                   ctypes.cast(garr, ctypes.POINTER(ctypes.c_int32)), ng,
                   ctypes.cast(al, ctypes.POINTER(ctypes.c_float)),
                   _ptr(out.get("O")), _ptr(out["scores"]), _ptr(out["pos"]), _ptr(out["len"]),
-                  SC_STACK_NO_TAIL if no_tail else 0, int(keep_rule), _ptr(out.get("O_last")))
+                  _stack_flags(no_tail, plain_launches), int(keep_rule), _ptr(out.get("O_last")))
     _check(load().sc_stack_forward_host(ctypes.byref(a), _ptr(ws), ws.numel(),
                                         _stream_handle(stream)))
     return out

@@ -11,6 +11,7 @@
 #include <cstdio>
 #include <atomic>
 #include <cstring>
+#include <functional>
 #include <mutex>
 
 #include "../../include/sparsecoder.h"
@@ -480,11 +481,11 @@ struct HostResults {
 // maps of the "source" slot are pointed at the compacted copies and never
 // selected, and every layer's rows are gathered; hres (host_io only): where
 // the cluster kernel puts its results.
-static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
-                              void* stream, void** events, int n_events, bool host_io = false,
-                              const HostResults* hres = nullptr) {
+// The argument checks of a stack call (nothing is enqueued).
+static int stack_check(const sc_stack_args* a, void* workspace, size_t ws_bytes) {
   if (!a) return SC_ERR_INVALID_ARG;
-  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~(SC_STACK_NO_TAIL | SC_STACK_PLAIN_LAUNCHES)))
+    return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
   if (!a->Q || !a->K || !a->V || !a->alpha || !a->scores || !a->pos || !a->len)
@@ -493,15 +494,24 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   if (!aligned16(a->Q) || !aligned16(a->K) || !aligned16(a->V) || !aligned16(a->O) ||
       !aligned16(a->O_last))
     return SC_ERR_INVALID_ARG;
-  // the O of every layer, or (O == NULL) only the last layer's, to O_last
-  uint16_t* const o_last = a->O != nullptr ? nullptr : a->O_last;
   const long long rows = static_cast<long long>(a->n_layers) * a->B * a->L * a->H;
   if (rows > (1ll << 31) - 1) return SC_ERR_UNSUPPORTED;
   WsLayout lay;
   ws_layout(a->B, a->L, a->H, &lay);
   if (!workspace || ws_bytes < lay.total || (reinterpret_cast<uintptr_t>(workspace) % kAlign))
     return SC_ERR_WORKSPACE;
-  if ((rc = ensure_configured()) != SC_OK) return rc;
+  return ensure_configured();
+}
+
+static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws_bytes,
+                              void* stream, void** events, int n_events, bool host_io = false,
+                              const HostResults* hres = nullptr) {
+  int rc = stack_check(a, workspace, ws_bytes);
+  if (rc != SC_OK) return rc;
+  // the O of every layer, or (O == NULL) only the last layer's, to O_last
+  uint16_t* const o_last = a->O != nullptr ? nullptr : a->O_last;
+  WsLayout lay;
+  ws_layout(a->B, a->L, a->H, &lay);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   char* ws = static_cast<char*>(workspace);
 
@@ -763,8 +773,168 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   return SC_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Eager stack calls as CUDA graphs
+// ---------------------------------------------------------------------------
+// An eager call whose sequences can leave the per-layer kernels for the
+// cluster kernel is recorded into a CUDA graph, where the layer loop is a
+// device-driven WHILE node (layers that no sequence runs per layer launch
+// nothing), and the instantiated graph is launched on the caller's stream.
+// Later calls with the same arguments launch the cached graph without
+// recording again.  The key holds everything a recorded call reads on the
+// host: the sizes, the device addresses, the alpha and global arrays by value,
+// the workspace, the device and the process-wide settings read at enqueue
+// (rows-kernel design, stall hook).
+
+struct GraphKey {
+  int dev, host_io, flags, n_layers, B, L, H, w, n_global, keep_rule, rows_kernel;
+  unsigned long long stall_ns;
+  size_t ws_bytes;
+  const void* ptr[16];
+  float alpha[kTailMaxLayers];
+  int32_t gpos[SC_MAX_GLOBAL];
+};
+
+struct GraphEntry {
+  GraphKey key;
+  cudaGraphExec_t exec;
+  unsigned long long used;
+};
+
+constexpr int kGraphCacheSize = 16;
+
+// Calls recorded into a new graph, and calls that launched a kept one
+// (sc_debug_graph_counts).
+std::atomic<unsigned long long> g_graphs_recorded{0};
+std::atomic<unsigned long long> g_graphs_reused{0};
+
+// A stream of this library per device on which eager calls are recorded
+// (nullptr if it cannot be made).
+static cudaStream_t record_stream() {
+  static std::mutex mu;
+  static cudaStream_t rec[256] = {nullptr};
+  static bool tried[256] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!tried[dev]) {
+    tried[dev] = true;
+    if (cudaStreamCreateWithFlags(&rec[dev], cudaStreamNonBlocking) != cudaSuccess) {
+      cudaGetLastError();
+      rec[dev] = nullptr;
+    }
+  }
+  return rec[dev];
+}
+
+// The key of a stack call (a: the arguments as the kernels see them, with
+// device addresses; extra: further addresses the call uses).
+static GraphKey graph_key(const sc_stack_args* a, const void* ws, size_t ws_bytes, bool host_io,
+                          const void* const* extra, int n_extra) {
+  GraphKey k;
+  std::memset(&k, 0, sizeof(k));
+  cudaGetDevice(&k.dev);
+  k.host_io = host_io ? 1 : 0;
+  k.flags = a->flags;
+  k.n_layers = a->n_layers; k.B = a->B; k.L = a->L; k.H = a->H; k.w = a->w;
+  k.n_global = a->n_global;
+  k.keep_rule = a->keep_rule;
+  k.rows_kernel = g_rows_kernel.load(std::memory_order_relaxed);
+  k.stall_ns = g_stall_ns.load(std::memory_order_relaxed);
+  k.ws_bytes = ws_bytes;
+  const void* ptrs[] = {ws, a->Q, a->K, a->V, a->pad_mask, a->O, a->scores, a->pos, a->len,
+                        a->O_last};
+  int n = 0;
+  for (const void* q : ptrs) k.ptr[n++] = q;
+  for (int i = 0; i < n_extra && n < 16; ++i) k.ptr[n++] = extra[i];
+  for (int l = 0; l < a->n_layers && l < kTailMaxLayers; ++l) k.alpha[l] = a->alpha[l];
+  for (int g = 0; g < a->n_global && g < SC_MAX_GLOBAL; ++g) k.gpos[g] = a->global_pos[g];
+  return k;
+}
+
+// Launch the graph of `key` on `st`, recording it first (enqueue(stream)
+// issues the call's work on a capturing stream) when no cached graph has that
+// key.  The least recently used graph makes room for a new one; a graph that
+// is still running when it is destroyed is freed when it completes.
+static int launch_as_graph(const GraphKey& key, cudaStream_t st,
+                           const std::function<int(cudaStream_t)>& enqueue) {
+  static std::mutex mu;
+  static GraphEntry cache[kGraphCacheSize];
+  static int n_cached = 0;
+  static unsigned long long clock = 0;
+  std::lock_guard<std::mutex> lock(mu);
+  ++clock;
+  for (int i = 0; i < n_cached; ++i) {
+    if (std::memcmp(&cache[i].key, &key, sizeof(key)) == 0) {
+      cache[i].used = clock;
+      g_graphs_reused.fetch_add(1);
+      const cudaError_t e = cudaGraphLaunch(cache[i].exec, st);
+      return e == cudaSuccess ? SC_OK : fail_cuda("launch stack graph", e);
+    }
+  }
+  cudaStream_t rec = record_stream();
+  if (rec == nullptr) return enqueue(st);   // cannot record: launch the kernels directly
+  cudaError_t e = cudaStreamBeginCapture(rec, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return fail_cuda("record stack call", e);
+  const int rc = enqueue(rec);
+  cudaGraph_t g = nullptr;
+  e = cudaStreamEndCapture(rec, &g);
+  if (rc != SC_OK || e != cudaSuccess) {
+    if (g != nullptr) cudaGraphDestroy(g);
+    cudaGetLastError();
+    return rc != SC_OK ? rc : fail_cuda("end stack call record", e);
+  }
+  cudaGraphExec_t x = nullptr;
+  e = cudaGraphInstantiate(&x, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return fail_cuda("instantiate stack graph", e);
+  int slot = n_cached;
+  if (n_cached == kGraphCacheSize) {
+    slot = 0;
+    for (int i = 1; i < n_cached; ++i)
+      if (cache[i].used < cache[slot].used) slot = i;
+    cudaGraphExecDestroy(cache[slot].exec);
+  } else {
+    ++n_cached;
+  }
+  cache[slot].key = key;
+  cache[slot].exec = x;
+  cache[slot].used = clock;
+  g_graphs_recorded.fetch_add(1);
+  e = cudaGraphLaunch(x, st);
+  return e == cudaSuccess ? SC_OK : fail_cuda("launch stack graph", e);
+}
+
+// Whether a stack call on `st` runs as a graph of this library: eager (the
+// stream is not capturing), not asked for plain launches, and with both the
+// per-layer kernels and the cluster kernel in its plan.
+static bool graph_route(const sc_stack_args* a, cudaStream_t st) {
+  if (a->flags & SC_STACK_PLAIN_LAUNCHES) return false;
+  bool use_tail = false, per_layer = true;
+  if (stack_plan(a, &use_tail, &per_layer) != SC_OK || !(use_tail && per_layer)) return false;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return cap == cudaStreamCaptureStatusNone;
+}
+
 int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
-  return stack_forward_impl(a, workspace, ws_bytes, stream, nullptr, 0);
+  if (!a) return SC_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // the checks of stack_forward_impl come first (nothing is recorded for a
+  // rejected call): they run again, unchanged, while the call is recorded
+  int rc = stack_check(a, workspace, ws_bytes);
+  if (rc != SC_OK || !graph_route(a, st))
+    return rc != SC_OK ? rc : stack_forward_impl(a, workspace, ws_bytes, stream, nullptr, 0);
+  const GraphKey key = graph_key(a, workspace, ws_bytes, false, nullptr, 0);
+  return launch_as_graph(key, st, [&](cudaStream_t s) {
+    return stack_forward_impl(a, workspace, ws_bytes, s, nullptr, 0);
+  });
 }
 
 int sc_stack_forward_profiled(const sc_stack_args* a, void* workspace, size_t ws_bytes,
@@ -830,7 +1000,8 @@ size_t sc_stack_host_workspace_size(int n_layers, int B, int L, int H) {
 
 int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_bytes, void* stream) {
   if (!a) return SC_ERR_INVALID_ARG;
-  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~(SC_STACK_NO_TAIL | SC_STACK_PLAIN_LAUNCHES)))
+    return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
   if (!a->Q || !a->K || !a->V || !a->alpha || !a->scores || !a->pos || !a->len)
@@ -876,44 +1047,54 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   const HostResults hres{static_cast<uint16_t*>(o), static_cast<uint16_t*>(o_last),
                          static_cast<float*>(sc), static_cast<int32_t*>(ps),
                          static_cast<int32_t*>(ln)};
-  if ((rc = stack_forward_impl(&d, workspace, hl.O, stream, nullptr, 0, true, &hres)) != SC_OK)
-    return rc;
-  bool use_tail = false, per_layer = true;
-  if ((rc = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc;
-  int dev = 0, sms = 0;
-  cudaError_t ce = cudaGetDevice(&dev);
-  if (ce == cudaSuccess) ce = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (ce != cudaSuccess) return fail_cuda("device attributes", ce);
-  WsLayout lay;
-  ws_layout(a->B, a->L, a->H, &lay);
-  ExportParams e{};
-  e.n_layers = a->n_layers; e.B = a->B; e.L = a->L; e.H = a->H;
-  e.O = dO; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
-  e.hO = static_cast<uint16_t*>(o);
-  e.hO_last = static_cast<uint16_t*>(o_last);
-  e.hscores = static_cast<float*>(sc);
-  e.hpos = static_cast<int32_t*>(ps);
-  e.hlen = static_cast<int32_t*>(ln);
-  e.tail_from = reinterpret_cast<const int32_t*>(ws + lay.tail_from);
+  // the stack, then the export of the per-layer results, on stream s
+  auto enqueue = [&](cudaStream_t s) -> int {
+    int rc2 = stack_forward_impl(&d, workspace, hl.O, s, nullptr, 0, true, &hres);
+    if (rc2 != SC_OK) return rc2;
+    bool use_tail = false, per_layer = true;
+    if ((rc2 = stack_plan(a, &use_tail, &per_layer)) != SC_OK) return rc2;
+    int dev = 0, sms = 0;
+    cudaError_t ce = cudaGetDevice(&dev);
+    if (ce == cudaSuccess) ce = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (ce != cudaSuccess) return fail_cuda("device attributes", ce);
+    WsLayout lay;
+    ws_layout(a->B, a->L, a->H, &lay);
+    ExportParams e{};
+    e.n_layers = a->n_layers; e.B = a->B; e.L = a->L; e.H = a->H;
+    e.O = dO; e.scores = d.scores; e.pos = d.pos; e.len = d.len;
+    e.hO = static_cast<uint16_t*>(o);
+    e.hO_last = static_cast<uint16_t*>(o_last);
+    e.hscores = static_cast<float*>(sc);
+    e.hpos = static_cast<int32_t*>(ps);
+    e.hlen = static_cast<int32_t*>(ln);
+    e.tail_from = reinterpret_cast<const int32_t*>(ws + lay.tail_from);
+    if (use_tail) {
+      // the per-layer results go out beside the cluster kernel, on the SMs it
+      // leaves idle (one CTA per SM fits beside one of its CTAs); the cluster
+      // kernel writes its own layers' results to the host buffers itself.  The
+      // export ends with a grid wait, so the call ends after the cluster kernel.
+      e.part = 1;
+      if ((ce = launch_export(e, sms, s)) != cudaSuccess)
+        return fail_cuda("launch export kernel", ce);
+    } else {
+      e.part = 0;
+      if ((ce = launch_export(e, 4 * sms, s)) != cudaSuccess)
+        return fail_cuda("launch export kernel", ce);
+    }
+    return SC_OK;
+  };
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (use_tail) {
-    // the per-layer results go out beside the cluster kernel, on the SMs it
-    // leaves idle (one CTA per SM fits beside one of its CTAs); the cluster
-    // kernel writes its own layers' results to the host buffers itself.  The
-    // export ends with a grid wait, so the call ends after the cluster kernel.
-    e.part = 1;
-    if ((ce = launch_export(e, sms, st)) != cudaSuccess) return fail_cuda("launch export kernel", ce);
-  } else {
-    e.part = 0;
-    if ((ce = launch_export(e, 4 * sms, st)) != cudaSuccess)
-      return fail_cuda("launch export kernel", ce);
-  }
-  return SC_OK;
+  if ((rc = stack_check(&d, workspace, hl.O)) != SC_OK) return rc;
+  if (!graph_route(a, st)) return enqueue(st);
+  const void* results[] = {o, o_last, sc, ps, ln};
+  const GraphKey key = graph_key(&d, workspace, ws_bytes, true, results, 5);
+  return launch_as_graph(key, st, enqueue);
 }
 
 int sc_stack_host_launch_count(const sc_stack_args* a, int* count) {
   if (!a || !count) return SC_ERR_INVALID_ARG;
-  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~(SC_STACK_NO_TAIL | SC_STACK_PLAIN_LAUNCHES)))
+    return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
   if ((rc = ensure_configured()) != SC_OK) return rc;
@@ -928,7 +1109,8 @@ int sc_stack_host_launch_count(const sc_stack_args* a, int* count) {
 
 int sc_stack_launch_count(const sc_stack_args* a, int* count) {
   if (!a || !count) return SC_ERR_INVALID_ARG;
-  if (a->n_layers < 1 || (a->flags & ~SC_STACK_NO_TAIL)) return SC_ERR_INVALID_ARG;
+  if (a->n_layers < 1 || (a->flags & ~(SC_STACK_NO_TAIL | SC_STACK_PLAIN_LAUNCHES)))
+    return SC_ERR_INVALID_ARG;
   int rc = check_common(a->B, a->L, a->H, a->w, a->global_pos, a->n_global);
   if (rc != SC_OK) return rc;
   if ((rc = ensure_configured()) != SC_OK) return rc;
@@ -942,6 +1124,11 @@ int sc_stack_launch_count(const sc_stack_args* a, int* count) {
 }
 
 void sc_debug_stall_waits(unsigned long long ns) { g_stall_ns.store(ns); }
+
+void sc_debug_graph_counts(unsigned long long* recorded, unsigned long long* reused) {
+  if (recorded) *recorded = g_graphs_recorded.load();
+  if (reused) *reused = g_graphs_reused.load();
+}
 
 int sc_select_rows_kernel(int which) {
   if (which != SC_ROWS_SINGLE_PASS && which != SC_ROWS_TWO_PASS) return SC_ERR_INVALID_ARG;

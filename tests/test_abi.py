@@ -134,7 +134,7 @@ def test_stack_rejects_bad_arguments(lib):
     assert call(O=None, O_last=FAKE + 2) == bd.SC_ERR_INVALID_ARG
     assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
     assert call(w=513) == bd.SC_ERR_UNSUPPORTED
-    assert call(flags=2) == bd.SC_ERR_INVALID_ARG
+    assert call(flags=4) == bd.SC_ERR_INVALID_ARG   # bits 0 and 1 are the two flags
     assert call(keep_rule=7) == bd.SC_ERR_INVALID_ARG
     bad = (ctypes.c_float * 12)(*([0.5] * 11 + [float("nan")]))
     assert call(keep_rule=bd.SC_KEEP_TOP_RATIO,
@@ -166,7 +166,7 @@ def test_stack_host_rejects_bad_arguments(lib):
     assert call(n_layers=0) == bd.SC_ERR_INVALID_ARG
     assert call(Q=None) == bd.SC_ERR_INVALID_ARG
     assert call(L=8192) == bd.SC_ERR_UNSUPPORTED
-    assert call(flags=2) == bd.SC_ERR_INVALID_ARG
+    assert call(flags=4) == bd.SC_ERR_INVALID_ARG   # bits 0 and 1 are the two flags
     assert call(ws_bytes=need - 256) == bd.SC_ERR_WORKSPACE
     # ordinary (pageable) host memory is refused: the kernels could not reach it
     assert call() == bd.SC_ERR_INVALID_ARG

@@ -309,7 +309,10 @@ int sc_stack_launch_count(const sc_stack_args* args, int* count);
  *
  * Asynchronous on `stream` like every call: the host buffers must stay
  * allocated and unmodified (inputs) or unread (results) until the stream has
- * passed the call.  Capturable in a CUDA graph (it issues kernels only).
+ * passed the call.  Capturable in a CUDA graph (it issues kernels only); an
+ * eager call runs through a kept graph of the library (the export included)
+ * under the same rules as sc_stack_forward, the mapped host addresses being
+ * part of its key.
  * Errors: as sc_stack_forward, and SC_ERR_INVALID_ARG with nothing launched
  * when a host range is not page-locked memory mapped for the device (checked
  * at both ends of each range) or a mapped address is misaligned (Q, K, V, O:

@@ -564,8 +564,10 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
   // While the call is captured into a CUDA graph, the per-layer kernels run
   // in a WHILE node whose condition the device sets ("some sequence still has
   // more than kTailMax tokens"), with the layer index in device memory: layers
-  // that every sequence has left cost no launch.  Eager calls launch every
-  // layer's kernels, which then skip the sequences of the cluster kernel.
+  // that every sequence has left cost no launch.  Uncaptured calls here (plain
+  // launches, the profiled call) launch every layer's kernels, which then skip
+  // the sequences of the cluster kernel; other eager calls reach this point
+  // while the library records them into a graph of its own.
   bool dev_loop = false;
   cudaGraphConditionalHandle cond = 0;
   cudaStream_t side = nullptr;

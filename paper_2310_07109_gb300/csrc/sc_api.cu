@@ -788,14 +788,18 @@ static int stack_forward_impl(const sc_stack_args* a, void* workspace, size_t ws
 // the workspace, the device and the process-wide settings read at enqueue
 // (rows-kernel design, stall hook).
 
+// Compared and copied as bytes: laid out without padding, zeroed before use.
 struct GraphKey {
-  int dev, host_io, flags, n_layers, B, L, H, w, n_global, keep_rule, rows_kernel;
   unsigned long long stall_ns;
-  size_t ws_bytes;
+  unsigned long long ws_bytes;
   const void* ptr[16];
+  int dev, host_io, flags, n_layers, B, L, H, w, n_global, keep_rule, rows_kernel, unused;
   float alpha[kTailMaxLayers];
   int32_t gpos[SC_MAX_GLOBAL];
 };
+static_assert(sizeof(GraphKey) == 2 * 8 + 16 * sizeof(void*) + 12 * 4 + kTailMaxLayers * 4 +
+                                      SC_MAX_GLOBAL * 4,
+              "GraphKey has padding");
 
 struct GraphEntry {
   GraphKey key;
@@ -834,9 +838,9 @@ static cudaStream_t record_stream() {
 
 // The key of a stack call (a: the arguments as the kernels see them, with
 // device addresses; extra: further addresses the call uses).
-static GraphKey graph_key(const sc_stack_args* a, const void* ws, size_t ws_bytes, bool host_io,
-                          const void* const* extra, int n_extra) {
-  GraphKey k;
+static void graph_key(GraphKey* out, const sc_stack_args* a, const void* ws, size_t ws_bytes,
+                      bool host_io, const void* const* extra, int n_extra) {
+  GraphKey& k = *out;
   std::memset(&k, 0, sizeof(k));
   cudaGetDevice(&k.dev);
   k.host_io = host_io ? 1 : 0;
@@ -854,7 +858,6 @@ static GraphKey graph_key(const sc_stack_args* a, const void* ws, size_t ws_byte
   for (int i = 0; i < n_extra && n < 16; ++i) k.ptr[n++] = extra[i];
   for (int l = 0; l < a->n_layers && l < kTailMaxLayers; ++l) k.alpha[l] = a->alpha[l];
   for (int g = 0; g < a->n_global && g < SC_MAX_GLOBAL; ++g) k.gpos[g] = a->global_pos[g];
-  return k;
 }
 
 // Launch the graph of `key` on `st`, recording it first (enqueue(stream)
@@ -902,7 +905,7 @@ static int launch_as_graph(const GraphKey& key, cudaStream_t st,
   } else {
     ++n_cached;
   }
-  cache[slot].key = key;
+  std::memcpy(&cache[slot].key, &key, sizeof(key));
   cache[slot].exec = x;
   cache[slot].used = clock;
   g_graphs_recorded.fetch_add(1);
@@ -933,7 +936,8 @@ int sc_stack_forward(const sc_stack_args* a, void* workspace, size_t ws_bytes, v
   int rc = stack_check(a, workspace, ws_bytes);
   if (rc != SC_OK || !graph_route(a, st))
     return rc != SC_OK ? rc : stack_forward_impl(a, workspace, ws_bytes, stream, nullptr, 0);
-  const GraphKey key = graph_key(a, workspace, ws_bytes, false, nullptr, 0);
+  GraphKey key;
+  graph_key(&key, a, workspace, ws_bytes, false, nullptr, 0);
   return launch_as_graph(key, st, [&](cudaStream_t s) {
     return stack_forward_impl(a, workspace, ws_bytes, s, nullptr, 0);
   });
@@ -1089,7 +1093,8 @@ int sc_stack_forward_host(const sc_stack_args* a, void* workspace, size_t ws_byt
   if ((rc = stack_check(&d, workspace, hl.O)) != SC_OK) return rc;
   if (!graph_route(a, st)) return enqueue(st);
   const void* results[] = {o, o_last, sc, ps, ln};
-  const GraphKey key = graph_key(&d, workspace, ws_bytes, true, results, 5);
+  GraphKey key;
+  graph_key(&key, &d, workspace, ws_bytes, true, results, 5);
   return launch_as_graph(key, st, enqueue);
 }
 

@@ -1295,9 +1295,11 @@ int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, cons
               const int32_t* a_idx, const uint16_t* W, const float* bias, int gelu,
               const uint16_t* res, const int32_t* res_idx, void* out, int out_f32, int* status) {
   *g = GemmParams{};
-  // 256-column tiles unless that leaves fewer than two tiles per SM (the row
-  // count is a bound: rows are counted on the device) and A is not gathered
-  // (a gathered A is fetched again for every column tile)
+  // Column-tile width: with a gathered A, 256 (A is fetched again for every
+  // column tile); otherwise the width among 256, 192 and 128 (dividing N) with
+  // the least (whole rounds of tiles over the SMs) x (width + 32), the 32 a
+  // per-tile cost in columns' worth of time.  The row count is a bound (rows
+  // are counted on the device).
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) != cudaSuccess ||
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
@@ -1305,7 +1307,19 @@ int make_gemm(GemmParams* g, int B, int L, int N, int K, const uint16_t* A, cons
     sms = 152;
   }
   const long long row_tiles = static_cast<long long>(B) * ((L + kTile - 1) / kTile);
-  const int bn = (!a_idx && row_tiles * ((N + 255) / 256) < 2ll * sms) ? 128 : 256;
+  int bn = 256;
+  if (!a_idx) {
+    long long best = -1;
+    for (int c : {256, 192, 128}) {
+      if (c != 256 && N % c != 0) continue;
+      const long long tiles = row_tiles * ((N + c - 1) / c);
+      const long long cost = (tiles + sms - 1) / sms * (c + 32);
+      if (best < 0 || cost < best) {
+        best = cost;
+        bn = c;
+      }
+    }
+  }
   const int wbox = N < bn ? N : bn;
   if (!encode_2d(&g->map_a, A, static_cast<long long>(B) * L, K, 1) ||
       !encode_2d(&g->map_at, A, static_cast<long long>(B) * L, K, kTile) ||

@@ -33,7 +33,7 @@ constexpr int kGemmThreads = 320;   // warp 0 loads, warp 1 issues, warps 2-9 wr
 constexpr int kGemmEpiWarps = 8;    // two per tensor-memory lane quarter, one column half each
 constexpr int kGemmStages = 4;
 constexpr int kGemmBK = 64;         // K per stage: one 128-byte swizzle atom of bf16
-constexpr int kGemmBN = 256;        // output columns per tile (one MMA, N = 256)
+constexpr int kGemmBN = 256;        // most output columns per tile (one MMA, N <= 256)
 constexpr uint32_t kGemmABytes = kTileBytes;              // 128 rows x 64
 constexpr uint32_t kGemmWBytes = kGemmBN * kGemmBK * 2;   // 256 rows x 64
 constexpr uint32_t kGemmStageBytes = kGemmABytes + kGemmWBytes;

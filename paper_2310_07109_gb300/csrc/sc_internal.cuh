@@ -257,14 +257,15 @@ struct TailParams {
 // One GEMM of the encoder layer: out[(b, r)][n] = epi(sum_k A[row_a][k] W[n][k])
 // for r < rows[b], row_a = b L + (a_idx ? a_idx[b L + r] : r); epi adds bias[n],
 // then GELU (gelu != 0), then the bf16 residual res[row][n] (row = b L +
-// (res_idx ? res_idx[b L + r] : r)).  N % 128 == 0, K % 64 == 0; 128 x 256 tiles.
+// (res_idx ? res_idx[b L + r] : r)).  N % 128 == 0, K % 64 == 0; tiles of 128 rows
+// by bn columns.
 struct GemmParams {
   CUtensorMap map_a;               // 2-D [B L][K] bf16, box 64 x 1 (four-row gathers)
   CUtensorMap map_at;              // the same matrix, box 64 x 128 (consecutive rows)
   CUtensorMap map_w;               // 2-D [N][K] bf16, box 64 x wbox
   int B, L, N, K;
-  int bn;                          // output columns per tile: 256, or 128 when that gives
-                                   // too few tiles for the SMs
+  int bn;                          // output columns per tile: 256, 192 or 128 (the width
+                                   // that fills the SMs' rounds of tiles best)
   int wbox;                        // W rows per copy: min(bn, N)
   const int32_t* rows;             // [B] rows per sequence, or nullptr (L)
   const int32_t* a_idx;            // [B][L] A row of output row (b, r), or nullptr

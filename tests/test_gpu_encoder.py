@@ -54,6 +54,10 @@ LINEAR_CASES = [
     (2, 256, [200, 256], 384, 192, False, True, False, False, False),
     (3, 130, [130, 1, 129], 768, 3072, False, False, True, False, True),
     (1, 512, [431], 3072, 768, True, True, False, False, False),
+    # 192-column tiles (the width that fills whole rounds of tiles best here)
+    (8, 1024, [1024, 1000, 517, 3, 1024, 900, 128, 129], 768, 768, False, False, True, False,
+     False),
+    (4, 1664, [1664, 1600, 1, 830], 384, 128, False, True, False, False, True),
 ]
 
 

@@ -236,14 +236,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const GemmTile g = gemm_tile(p, t);
       if (g.skip) continue;
       const int acc = j & 1;
-      ok = ok && warp_wait_gemm(&sm.tfull[acc], (j >> 1) & 1, abort_flag);
       const int r = g.r0 + 32 * q + lane;
-      const bool valid = ok && r < g.rows;
+      const bool in_rows = r < g.rows;
       const size_t orow = static_cast<size_t>(g.b) * p.L + r;
       const int rsrc =
-          valid ? (p.res_idx ? __ldcg(p.res_idx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
+          in_rows ? (p.res_idx ? __ldcg(p.res_idx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
       const uint16_t* res =
           p.res ? p.res + (static_cast<size_t>(g.b) * p.L + rsrc) * p.N + g.n0 : nullptr;
+      const int cbeg = ch * (p.bn / 2), cend = min(g.nw, (ch + 1) * (p.bn / 2));
+      // this row's residual over the warp's columns (at most 4 x 32), loaded
+      // before the accumulator is ready so that its latency overlaps the MMAs
+      uint4 rpf[4][4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = cbeg + 32 * u;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          rpf[u][k] = (res != nullptr && c < cend)
+                          ? __ldcg(reinterpret_cast<const uint4*>(res + c + 8 * k))
+                          : make_uint4(0u, 0u, 0u, 0u);
+      }
+      ok = ok && warp_wait_gemm(&sm.tfull[acc], (j >> 1) & 1, abort_flag);
+      const bool valid = ok && in_rows;
       int nb = g.n0, ldo = p.N;
       void* outp = p.out;
       if (p.out_split > 0) {
@@ -253,12 +267,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         ldo = p.out_split;
       }
       tc_fence_after();
-#pragma unroll 1
-      for (int c = ch * (p.bn / 2); c < min(g.nw, (ch + 1) * (p.bn / 2)); c += 32) {
+      // one 32-column chunk: bias, GELU, the residual (rv: its 32 values, or
+      // nullptr), store
+      auto chunk = [&](int c, const uint4* rv) {
         float v[32];
         tmem_ld32(tm + acc * kGemmBN + (static_cast<uint32_t>(32 * q) << 16) + c, v);
         tmem_ld_wait();
-        if (!valid) continue;
+        if (!valid) return;
         const float4* bp = reinterpret_cast<const float4*>(p.bias + g.n0 + c);
 #pragma unroll
         for (int k = 0; k < 32; k += 4) {
@@ -271,11 +286,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (p.gelu)
 #pragma unroll
           for (int k = 0; k < 32; k += 2) gelu_erf2(v[k], v[k + 1]);
-        if (res) {
+        if (rv != nullptr) {
 #pragma unroll
           for (int k = 0; k < 32; k += 8) {
-            const uint4 u = __ldcg(reinterpret_cast<const uint4*>(res + c + k));
-            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+            const uint4 r4 = rv[k / 8];
+            const uint32_t w4[4] = {r4.x, r4.y, r4.z, r4.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               v[k + 2 * e] += __uint_as_float(w4[e] << 16);
@@ -296,6 +311,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
                            pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
         }
+      };
+      if (res == nullptr) {
+#pragma unroll 1
+        for (int c = cbeg; c < cend; c += 32) chunk(c, nullptr);
+      } else {
+        // unrolled, so that the prefetched residual stays in registers
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (cbeg + 32 * u < cend) chunk(cbeg + 32 * u, rpf[u]);
       }
       // the buffer may take the tile after next
       tc_fence_before();

@@ -23,6 +23,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>
+#include <type_traits>
 
 #include "sc_internal.cuh"
 #include "sm103_primitives.cuh"
@@ -37,7 +38,10 @@ constexpr int kGemmBN = 256;        // most output columns per tile (one MMA, N 
 constexpr uint32_t kGemmABytes = kTileBytes;              // 128 rows x 64
 constexpr uint32_t kGemmWBytes = kGemmBN * kGemmBK * 2;   // 256 rows x 64
 constexpr uint32_t kGemmStageBytes = kGemmABytes + kGemmWBytes;
-constexpr uint32_t kGemmDyn = kGemmStages * kGemmStageBytes + 1024;
+// after the ring: a 4 KB staging area per write-back warp (32 rows of 128 bytes),
+// through which the stores of a chunk leave as whole row segments
+constexpr uint32_t kGemmStageOut = 4096;
+constexpr uint32_t kGemmDyn = kGemmStages * kGemmStageBytes + kGemmEpiWarps * kGemmStageOut + 1024;
 
 struct GemmSmem {
   uint64_t full[kGemmStages], empty[kGemmStages];
@@ -230,6 +234,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ------------------------------------------------------------- write back
     const int q = warp & 3;                  // tensor-memory lane quarter of this warp
     const int ch = (warp - 2) / 4;           // column half of the tile
+    uint8_t* const stg = base + kGemmStages * kGemmStageBytes + (warp - 2) * kGemmStageOut;
     bool ok = true;
     int j = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
@@ -238,26 +243,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const int acc = j & 1;
       const int r = g.r0 + 32 * q + lane;
       const bool in_rows = r < g.rows;
-      const size_t orow = static_cast<size_t>(g.b) * p.L + r;
       const int rsrc =
           in_rows ? (p.res_idx ? __ldcg(p.res_idx + static_cast<size_t>(g.b) * p.L + r) : r) : 0;
       const uint16_t* res =
           p.res ? p.res + (static_cast<size_t>(g.b) * p.L + rsrc) * p.N + g.n0 : nullptr;
       const int cbeg = ch * (p.bn / 2), cend = min(g.nw, (ch + 1) * (p.bn / 2));
-      // this row's residual over the warp's columns (at most 4 x 32), loaded
-      // before the accumulator is ready so that its latency overlaps the MMAs
-      uint4 rpf[4][4];
+      // without GELU, this row's residual over the warp's first three chunks
+      // of 32 columns is loaded before the accumulator is ready, so that its
+      // latency overlaps the MMAs (a fourth chunk, 256-column tiles only, and
+      // GEMMs with GELU load theirs chunk by chunk)
+      const bool res_ahead = res != nullptr && !p.gelu;
+      uint4 rpf[2][4];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 2; ++u) {
         const int c = cbeg + 32 * u;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          rpf[u][k] = (res != nullptr && c < cend)
+          rpf[u][k] = (res_ahead && c < cend)
                           ? __ldcg(reinterpret_cast<const uint4*>(res + c + 8 * k))
                           : make_uint4(0u, 0u, 0u, 0u);
       }
       ok = ok && warp_wait_gemm(&sm.tfull[acc], (j >> 1) & 1, abort_flag);
-      const bool valid = ok && in_rows;
+      const uint32_t rows_mask = __ballot_sync(0xffffffffu, ok && in_rows);
+      const size_t orow0 = static_cast<size_t>(g.b) * p.L + g.r0 + 32 * q;   // the warp's row 0
       int nb = g.n0, ldo = p.N;
       void* outp = p.out;
       if (p.out_split > 0) {
@@ -267,13 +275,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         ldo = p.out_split;
       }
       tc_fence_after();
-      // one 32-column chunk: bias, GELU, the residual (rv: its 32 values, or
-      // nullptr), store
-      auto chunk = [&](int c, const uint4* rv) {
+      // one 32-column chunk: bias, GELU (only where may_gelu is true), the
+      // residual (rv: its 32 values, or nullptr: loaded here), store
+      auto chunk = [&](int c, const uint4* rv, auto may_gelu) {
         float v[32];
         tmem_ld32(tm + acc * kGemmBN + (static_cast<uint32_t>(32 * q) << 16) + c, v);
         tmem_ld_wait();
-        if (!valid) return;
+        if (rows_mask == 0u) return;   // warp-uniform
         const float4* bp = reinterpret_cast<const float4*>(p.bias + g.n0 + c);
 #pragma unroll
         for (int k = 0; k < 32; k += 4) {
@@ -283,13 +291,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           v[k + 2] += b4.z;
           v[k + 3] += b4.w;
         }
-        if (p.gelu)
+        if constexpr (decltype(may_gelu)::value) {
+          if (p.gelu)
 #pragma unroll
-          for (int k = 0; k < 32; k += 2) gelu_erf2(v[k], v[k + 1]);
-        if (rv != nullptr) {
+            for (int k = 0; k < 32; k += 2) gelu_erf2(v[k], v[k + 1]);
+        }
+        if (res != nullptr) {
 #pragma unroll
           for (int k = 0; k < 32; k += 8) {
-            const uint4 r4 = rv[k / 8];
+            const uint4 r4 = rv != nullptr ? rv[k / 8]
+                                           : __ldcg(reinterpret_cast<const uint4*>(res + c + k));
             const uint32_t w4[4] = {r4.x, r4.y, r4.z, r4.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -298,28 +309,36 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
           }
         }
+        // the warp's 32 rows leave as whole 128-byte (fp32) or 64-byte (bf16)
+        // row segments; rows past the sequence are not written
         if (p.out_f32) {
-          float* o = static_cast<float*>(outp) + orow * ldo + nb + c;
 #pragma unroll
           for (int k = 0; k < 32; k += 4)
-            *reinterpret_cast<float4*>(o + k) = make_float4(v[k], v[k + 1], v[k + 2], v[k + 3]);
+            stage_row_piece<8>(stg, k / 4,
+                               make_uint4(__float_as_uint(v[k]), __float_as_uint(v[k + 1]),
+                                          __float_as_uint(v[k + 2]), __float_as_uint(v[k + 3])));
+          flush_staged_rows<8>(
+              stg, reinterpret_cast<uint16_t*>(static_cast<float*>(outp) + orow0 * ldo + nb + c),
+              2 * static_cast<size_t>(ldo), rows_mask);
         } else {
-          uint16_t* o = static_cast<uint16_t*>(outp) + orow * ldo + nb + c;
 #pragma unroll
           for (int k = 0; k < 32; k += 8)
-            *reinterpret_cast<uint4*>(o + k) =
-                make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
-                           pack_bf16x2(v[k + 4], v[k + 5]), pack_bf16x2(v[k + 6], v[k + 7]));
+            stage_row_piece<4>(stg, k / 8,
+                               make_uint4(pack_bf16x2(v[k], v[k + 1]), pack_bf16x2(v[k + 2], v[k + 3]),
+                                          pack_bf16x2(v[k + 4], v[k + 5]),
+                                          pack_bf16x2(v[k + 6], v[k + 7])));
+          flush_staged_rows<4>(stg, static_cast<uint16_t*>(outp) + orow0 * ldo + nb + c,
+                               static_cast<size_t>(ldo), rows_mask);
         }
       };
-      if (res == nullptr) {
+      if (!res_ahead) {
 #pragma unroll 1
-        for (int c = cbeg; c < cend; c += 32) chunk(c, nullptr);
+        for (int c = cbeg; c < cend; c += 32) chunk(c, nullptr, std::true_type{});
       } else {
         // unrolled, so that the prefetched residual stays in registers
 #pragma unroll
         for (int u = 0; u < 4; ++u)
-          if (cbeg + 32 * u < cend) chunk(cbeg + 32 * u, rpf[u]);
+          if (cbeg + 32 * u < cend) chunk(cbeg + 32 * u, u < 2 ? rpf[u] : nullptr, std::false_type{});
       }
       // the buffer may take the tile after next
       tc_fence_before();

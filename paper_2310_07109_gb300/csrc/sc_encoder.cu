@@ -248,10 +248,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const uint16_t* res =
           p.res ? p.res + (static_cast<size_t>(g.b) * p.L + rsrc) * p.N + g.n0 : nullptr;
       const int cbeg = ch * (p.bn / 2), cend = min(g.nw, (ch + 1) * (p.bn / 2));
-      // without GELU, this row's residual over the warp's first three chunks
-      // of 32 columns is loaded before the accumulator is ready, so that its
-      // latency overlaps the MMAs (a fourth chunk, 256-column tiles only, and
-      // GEMMs with GELU load theirs chunk by chunk)
+      // without GELU, this row's residual over the warp's first two chunks of
+      // 32 columns is loaded before the accumulator is ready, so that its
+      // latency overlaps the MMAs (later chunks, and GEMMs with GELU, load
+      // theirs chunk by chunk)
       const bool res_ahead = res != nullptr && !p.gelu;
       uint4 rpf[2][4];
 #pragma unroll

@@ -8,7 +8,8 @@ the kept graph without recording.  Checked here: the graph route gives the
 results of the plain-launch route (SC_STACK_PLAIN_LAUNCHES) bit for bit and the
 oracle's; an identical call reuses the kept graph; a call that changes what
 the host reads at enqueue (the alpha values, the global list, an output
-address, the rows design) records a new graph and follows the change.
+address, the rows design) records a new graph and follows the change; more
+argument sets than kept graphs replace the least recently used ones.
 """
 import numpy as np
 import pytest
@@ -201,3 +202,26 @@ def test_graph_route_on_a_side_stream(sc):
     stream.synchronize()
     assert sc.workspace_status(ws) == 0
     check_stack(WL, res, _numpy(out))
+
+
+def test_more_argument_sets_than_kept_graphs(sc):
+    """18 output sets cycled twice through the 16 kept graphs: the least
+    recently used graphs are replaced (and destroyed while the stream may still
+    run them), and every call's results are those of the first."""
+    wl = wk.Workload("eager_lru", n_layers=3, B=2, L=500, w=64, n_extra_global=2, seed=67)
+    inp, res, _ = resample_stack(wl)
+    t = {k: bits_to_torch(inp[k], "cuda") for k in ("Q", "K", "V")}
+    ws = sc.new_workspace(wl.B, wl.L, wl.H)
+    outs = [_outputs(wl) for _ in range(18)]
+    r0, _ = sc.debug_graph_counts()
+    for _ in range(2):
+        for o in outs:
+            sc.stack_forward(t["Q"], t["K"], t["V"], None, inp["global_pos"], wl.w, inp["alpha"],
+                             out=o, workspace=ws)
+    torch.cuda.synchronize()
+    r1, _ = sc.debug_graph_counts()
+    assert r1 - r0 == 36          # LRU over 18 sets in a cycle: every call records
+    assert sc.workspace_status(ws) == 0
+    check_stack(wl, res, _numpy(outs[0]))
+    for o in outs[1:]:
+        _same_defined_slots(wl, outs[0], o)

@@ -13,13 +13,15 @@
 // compaction of the kept rows is the A-operand gather of the output
 // projection (Y is the next layer's X, already compacted).
 //
-// GEMM: 128 x 256 output tiles of one sequence each (rows are (sequence, row)
-// pairs, row < rows[b] read on the device), one persistent CTA per SM walking
-// the tiles; K in steps of 64 through a four-stage TMA ring: A's 128 rows by
-// four-row gathers (tile::gather4, any row order), W's 256 rows by one tiled
-// copy, both 128B-swizzled and K-major; one thread issues the MMAs (N = 256)
-// into one of two 256-column fp32 accumulators in tensor memory while four
-// warps read the other back and apply bias, GELU and the residual.
+// GEMM: output tiles of 128 rows of one sequence (rows are (sequence, row)
+// pairs, row < rows[b] read on the device) by 256, 192 or 128 columns (chosen
+// on the host), one persistent CTA per SM walking the tiles; K in steps of 64
+// through a four-stage TMA ring: A's 128 rows by one tiled copy, or by
+// four-row gathers (tile::gather4, any row order) when A is gathered, W's rows
+// by one tiled copy, both 128B-swizzled and K-major; one thread issues the
+// MMAs (M = 128) into one of two 256-column fp32 accumulators in tensor memory
+// while eight warps read the other back, apply bias, GELU and the residual,
+// and store each 32-column chunk through shared memory as whole row segments.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <cstdint>

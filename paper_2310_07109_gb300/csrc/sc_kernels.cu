@@ -9,18 +9,21 @@
 //     the tensor cores (tcgen05, bf16 -> fp32 in tensor memory); each 16 KB
 //     operand tile is one TMA copy.  Row softmax in fp32 (base 2, lazily
 //     rescaled running max); P (bf16) goes back to tensor memory and P V
-//     accumulates there.  Writes O, the row log-sum-exp LSE_i, the far-row
-//     column sums of the global keys, and (max, sum) of the global rows over
-//     this tile's keys.
+//     accumulates there.  Then the band pass: S^T = K Q^T of each key tile of
+//     the band (the tiles are still resident) and, per key column j, the sum
+//     over the tile's rows of exp2(S_ij - LSE_i) (one thread per column, no
+//     cross-thread reduction), one partial per (key, query tile).  Writes O,
+//     the row log-sum-exp LSE_i, those partials, the far-row column sums of
+//     the global keys, and (max, sum) of the global rows over this tile's keys.
 //
 //   cols kernel   (one CTA per pair of 128-key tiles; one warpgroup per tile)
-//     S^T = K Q^T for the query tiles whose band reaches this key tile, then
-//     P[i,j] = exp2(S_ij - LSE_i) summed down each key column j (one thread
-//     per column, so no cross-thread reduction), plus the global rows'
-//     probabilities and their P V outputs.  The last CTA of a key tile sums
-//     the heads in a fixed order and applies the threshold; the last tile of a
-//     sequence compacts the survivors in order.  No CTA waits for another: the
-//     "last" CTA is found by an atomic counter.
+//     The global rows' probabilities over the pair's keys and their P V
+//     outputs, and each key's column sum: the band partials added in tile
+//     order, plus the global rows' share.  The last CTA of a key-tile pair
+//     sums the heads in a fixed order and applies the threshold; the last pair
+//     of a sequence compacts the survivors in order.  Each CTA waits (bounded)
+//     only for the rows CTAs of its own (sequence, head); the "last" CTAs are
+//     found by atomic counters.
 //
 //   gather kernel copies the survivors' next-layer Q, K, V rows into compacted
 //   buffers (coalesced 16-byte vectors) when they are not already in place.
